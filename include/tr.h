@@ -1,0 +1,173 @@
+/*
+ * tr.h -- C ABI of the ALTR visual-token reducer for GB300 (sm_103a).
+ *
+ * ALTR (arxiv 2607.13500, Section IV) keeps K of the N visual tokens of an
+ * image: the K1 = floor(lambda K) tokens with the highest second-order Renyi
+ * entropy of their channel-magnitude distribution (Stage I, Eq. 3-4), plus
+ * K2 = K - K1 tokens taken at a fixed stride along the remaining tokens sorted
+ * by the cosine between the final-layer MLP input x' and output x'' (Stage II,
+ * Eq. 5-6), returned as X* = X_imp union X_div (Eq. 7, Algorithm 1).
+ *
+ * Conventions shared by every entry point:
+ *  - Device pointers are owned by the caller; the library never allocates,
+ *    frees or synchronises.  Every call enqueues work on `stream` (a
+ *    cudaStream_t; NULL is the legacy default stream) and returns at once.
+ *  - Host-detectable errors (null or misaligned pointers, bad sizes, too small
+ *    a workspace) are returned before anything is launched; outputs are left
+ *    untouched.  A launch failure returns TR_ERR_CUDA.
+ *  - Data-dependent conditions are counted in the optional device status
+ *    words (int32[TR_STATUS_WORDS], accumulated with atomics; zero them before
+ *    the call): [0] rows found to hold a non-finite value in an input the
+ *    selection (or a requested H2 / s output) needed, [1] rows whose
+ *    exact sums did not fit the exact representation (ordering of such a row
+ *    falls back to its float key), [2] rows recomputed exactly to settle a
+ *    near-tie, [3] images skipped because their budget was invalid
+ *    (K < 0, K > N, K1 < 0 or K1 > K).
+ *  - Kept indices are local to their image, ascending, and image b's
+ *    occupy positions [cu_k[b], cu_k[b+1]) of `idx` and of `y`.
+ *  - Ties go to the lower token index, in the top-K1 and in the sort.
+ *  - The library keeps no global state besides a per-device "shared memory
+ *    limit already raised" flag; calls on different streams may run
+ *    concurrently when they use different workspaces.
+ */
+#ifndef TR_H
+#define TR_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  TR_OK = 0,
+  TR_ERR_ARG = 1,         /* null pointer, negative or inconsistent size       */
+  TR_ERR_BUDGET = 2,      /* K > N, lambda or ratio outside [0, 1] (host)      */
+  TR_ERR_DTYPE = 3,       /* dtype not one of tr_dtype                         */
+  TR_ERR_ALIGN = 4,       /* d * sizeof(elem) % 16 != 0 or a base not 16-B aligned */
+  TR_ERR_WORKSPACE = 5,   /* workspace NULL, too small or not 256-B aligned    */
+  TR_ERR_CUDA = 6,        /* a kernel launch failed                            */
+  TR_ERR_UNSUPPORTED = 7  /* N_b > TR_MAX_N or d > TR_MAX_D                    */
+} tr_status;
+
+typedef enum { TR_F32 = 0, TR_BF16 = 1 } tr_dtype;
+
+#define TR_MAX_N 16384        /* tokens per image (keys of one image stay in shared memory) */
+#define TR_MAX_D 16384        /* channels per token                                  */
+#define TR_STATS_WORDS 8      /* fp32 words of the per-row statistics record         */
+#define TR_STATUS_WORDS 4
+
+/*
+ * The token tensors of a batch of images, packed row-major as [total, d]:
+ * image b owns rows [cu_seqlens[b], cu_seqlens[b+1]) (ragged), or
+ * [b*n, (b+1)*n) when cu_seqlens is NULL (uniform).
+ */
+typedef struct {
+  const void *x;              /* visual tokens X, the Stage-I input and gather source (Sec. III-A) */
+  const void *x_pre;          /* final-layer MLP input x' (Eq. 5); NULL means x' = x               */
+  const void *x_post;         /* final-layer MLP output x'' (Eq. 5); required                      */
+  int32_t dtype;              /* tr_dtype of all three tensors                                     */
+  int32_t d;                  /* channels D                                                         */
+  int32_t batch;              /* images B                                                           */
+  int32_t n;                  /* tokens per image N when cu_seqlens is NULL                         */
+  const int32_t *cu_seqlens;  /* device int32[batch+1] row offsets, or NULL                         */
+  int32_t total;              /* total rows T (ragged: must equal cu_seqlens[batch])                */
+  int32_t max_n;              /* ragged: max_b N_b (host-known); ignored when uniform              */
+} tr_tokens;
+
+/* Name of a status code (static string). */
+const char *tr_status_string(int32_t status);
+
+/* Library version string. */
+const char *tr_version(void);
+
+/*
+ * Budgets of Algorithm 1, first step, and Eq. 7 (host only, no device work).
+ * Per image b with N_b = h_seqlens[b] tokens:
+ *   K_b  = k                          when k > 0,
+ *        = max(1, floor(N_b r_num / r_den)) (0 if N_b = 0) when k <= 0;
+ *   K1_b = floor(K_b lam_num / lam_den), K2_b = K_b - K1_b;
+ *   h_cu_k[0] = 0, h_cu_k[b+1] = h_cu_k[b] + K_b.
+ * lambda = lam_num / lam_den must lie in [0, 1] (the paper's split of K = 192
+ * into 64 + 128 tokens, Section V-C, is lambda = 1/3).  Returns TR_ERR_BUDGET
+ * when K_b > N_b, a ratio lies outside (0, 1] or lambda outside [0, 1];
+ * TR_ERR_ARG for null pointers or batch < 0.  h_k, h_k1: int32[batch];
+ * h_cu_k: int32[batch+1].
+ */
+tr_status tr_budgets(int32_t batch, const int32_t *h_seqlens, int32_t k, int32_t r_num, int32_t r_den,
+                     int32_t lam_num, int32_t lam_den, int32_t *h_k, int32_t *h_k1, int32_t *h_cu_k);
+
+/* Device workspace bytes that tr_select and tr_reduce need for `in`
+ * (0 on invalid input).  The workspace must be 256-byte aligned. */
+size_t tr_workspace_bytes(const tr_tokens *in);
+
+/*
+ * Scoring pass (Eq. 3, 4 and 6 for every token): one read of x, x', x''.
+ *   stats: device fp32[total, TR_STATS_WORDS] (16-byte aligned), per row
+ *          [0] L1 = sum_j |x_j|, [1] S2 = sum_j x_j^2, [2] A = sum_j x'_j^2,
+ *          [3] B = sum_j x''_j^2, [4] P_hi, [5] P_lo with P = sum_j x'_j x''_j
+ *          = P_hi + P_lo (double-float), [6..7] zero.  L1, S2, A, B are fp32
+ *          sums of bounded rounding depth; P is accumulated error-free up to
+ *          a ~1e-10 relative residue.
+ *   h2:    device fp32[total] or NULL: H2 = -log sum_j p_j^2 = log(L1^2 / S2)
+ *          (Eq. 3-4); 0 for an all-zero row.
+ *   s:     device fp32[total] or NULL: s = P / sqrt(A B) (Eq. 6); 0 when
+ *          x' or x'' is all zero.
+ * h2 and s come from the fp32 sums; rows whose sums overflow fp32 (inputs
+ * above ~2^63 in magnitude) or hold non-finite inputs get non-finite values
+ * here and are settled exactly by tr_select / tr_reduce.
+ */
+tr_status tr_score(const tr_tokens *in, float *stats, float *h2, float *s, void *stream);
+
+/*
+ * Selection (Stage I top-K1, Stage II sort and stride pick, Algorithm 1)
+ * from the statistics of tr_score.  Decisions are exact: keys whose float
+ * bounds overlap are recomputed from the inputs in exact integer arithmetic,
+ * so the result is the selection defined by the real-valued H2 and s with
+ * the lower-index tie-break.
+ *   d_k, d_k1:  device int32[batch] budgets K_b, K1_b (see tr_budgets).
+ *   d_cu_k:     device int32[batch+1] prefix sums of K_b.
+ *   idx:        device int32[cu_k[batch]] kept local indices (ascending).
+ *   role:       device uint8[total] or NULL: 0 dropped, 1 X_imp, 2 X_div.
+ *   h2, s:      device fp32[total] or NULL: when given, rows whose fp32 sums
+ *               were unreliable (non-finite, overflowed or underflowed) and
+ *               rows recomputed for a near-tie get H2 / s rewritten from the
+ *               exact sums (-inf H2 / +inf s for non-finite inputs).
+ *   ws:         device workspace of tr_workspace_bytes(in) bytes.
+ *   d_status:   device int32[TR_STATUS_WORDS] or NULL.
+ */
+tr_status tr_select(const tr_tokens *in, const float *stats, const int32_t *d_k, const int32_t *d_k1,
+                    const int32_t *d_cu_k, int32_t *idx, uint8_t *role, float *h2, float *s, void *ws,
+                    size_t ws_bytes, int32_t *d_status, void *stream);
+
+/*
+ * Gather of the kept tokens (Eq. 7: X* holds the original token vectors):
+ * y[r] = x[first row of image b + idx[r]] for cu_k[b] <= r < cu_k[b+1], a
+ * bit copy of d elements in the input dtype.
+ *   d_cu_k:   device int32[batch+1] prefix sums of K_b (as for tr_select).
+ *   idx:      device int32[total_k] local kept indices (tr_select's output).
+ *   total_k:  host int, = cu_k[batch].
+ *   y:        device [total_k, d] in the input dtype, 16-byte aligned.
+ * A row whose index falls outside its image's tokens is written as zeros.
+ */
+tr_status tr_gather(const tr_tokens *in, const int32_t *d_cu_k, const int32_t *idx, int32_t total_k, void *y,
+                    void *stream);
+
+/*
+ * The whole path in one call: tr_score, tr_select and tr_gather on `stream`
+ * (three kernel launches), with the statistics kept in the workspace.
+ *   total_k:  host int, = cu_k[batch] (the number of output rows).
+ *   y:        device [total_k, d] in the input dtype, 16-byte aligned.
+ *   idx, h2, s, d_status: as in tr_select (role is not produced); h2 and s
+ *             may be NULL.
+ */
+tr_status tr_reduce(const tr_tokens *in, const int32_t *d_k, const int32_t *d_k1, const int32_t *d_cu_k,
+                    int32_t total_k, void *y, int32_t *idx, float *h2, float *s, void *ws, size_t ws_bytes,
+                    int32_t *d_status, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TR_H */

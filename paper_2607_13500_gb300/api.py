@@ -1,0 +1,259 @@
+"""Python binding of libtr with the C ABI's names (argument marshalling only).
+
+Every step of the path runs in libtr's CUDA kernels; PyTorch only provides
+device memory and the current stream.  There is no CPU path: the calls raise
+when libtr.so is missing or a tensor is not on a CUDA device.
+"""
+from __future__ import annotations
+
+import ctypes
+from dataclasses import dataclass
+
+import torch
+
+from . import _lib
+from ._lib import TR_BF16, TR_F32, TR_STATS_WORDS, TR_STATUS_WORDS, TrTokens, check, load
+
+_I32 = ctypes.c_int32
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.bfloat16:
+        return TR_BF16
+    if t.dtype == torch.float32:
+        return TR_F32
+    raise TypeError(f"unsupported dtype {t.dtype}: expected torch.bfloat16 or torch.float32")
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(device) -> ctypes.c_void_p:
+    return ctypes.c_void_p(torch.cuda.current_stream(device).cuda_stream)
+
+
+def _flatten(x, x_pre, x_post, seqlens):
+    """[B, N, D] or [T, D] (+ seqlens) -> packed [T, D] tensors and seqlens."""
+    if x.dim() == 3:
+        b, n, d = x.shape
+        seqlens = [n] * b
+        x = x.reshape(b * n, d)
+        x_pre = None if x_pre is None else x_pre.reshape(b * n, d)
+        x_post = x_post.reshape(b * n, d)
+    elif x.dim() == 2:
+        if seqlens is None:
+            seqlens = [x.shape[0]]
+        seqlens = [int(v) for v in seqlens]
+        if sum(seqlens) != x.shape[0]:
+            raise ValueError("seqlens must sum to the number of rows of x")
+    else:
+        raise ValueError("x must be [B, N, D] or [T, D]")
+    for t in (x, x_pre, x_post):
+        if t is None:
+            continue
+        if t.shape != x.shape or t.dtype != x.dtype or t.device != x.device:
+            raise ValueError("x, x_pre and x_post must share shape, dtype and device")
+        if not t.is_contiguous():
+            raise ValueError("token tensors must be contiguous")
+    if x.device.type != "cuda":
+        raise ValueError("token tensors must live on a CUDA device (libtr has no CPU path)")
+    return x, x_pre, x_post, seqlens
+
+
+class _Tokens:
+    """A TrTokens struct plus the device tensors it points into."""
+
+    def __init__(self, x, x_pre, x_post, seqlens):
+        self.x, self.x_pre, self.x_post, self.seqlens = x, x_pre, x_post, seqlens
+        uniform = len(set(seqlens)) <= 1
+        self.cu = None
+        if not uniform:
+            cu = [0]
+            for n in seqlens:
+                cu.append(cu[-1] + n)
+            self.cu = torch.tensor(cu, dtype=torch.int32, device=x.device)
+        self.s = TrTokens(
+            x=x.data_ptr(), x_pre=None if x_pre is None else x_pre.data_ptr(), x_post=x_post.data_ptr(),
+            dtype=_dtype_code(x), d=x.shape[1], batch=len(seqlens),
+            n=seqlens[0] if (uniform and seqlens) else 0,
+            cu_seqlens=None if self.cu is None else self.cu.data_ptr(),
+            total=x.shape[0], max_n=max(seqlens) if seqlens else 0)
+
+    def ref(self):
+        return ctypes.byref(self.s)
+
+
+def budgets(seqlens, k=None, ratio=None, lam=(1, 3)):
+    """K_b, K1_b and cu_k per Algorithm 1's first step (tr_budgets)."""
+    lib = load()
+    b = len(seqlens)
+    arr = (_I32 * max(b, 1))(*seqlens)
+    hk, hk1, hcu = (_I32 * max(b, 1))(), (_I32 * max(b, 1))(), (_I32 * (b + 1))()
+    kk = int(k) if k else 0
+    rn, rd = ratio if ratio else (0, 0)
+    check("tr_budgets", lib.tr_budgets(b, arr, kk, rn, rd, lam[0], lam[1], hk, hk1, hcu))
+    return list(hk)[:b], list(hk1)[:b], list(hcu)
+
+
+def workspace_bytes(x, x_pre, x_post, seqlens=None) -> int:
+    x, x_pre, x_post, seqlens = _flatten(x, x_pre, x_post, seqlens)
+    return load().tr_workspace_bytes(_Tokens(x, x_pre, x_post, seqlens).ref())
+
+
+def score(x, x_pre, x_post, seqlens=None):
+    """tr_score: returns (stats [T, 8] fp32, h2 [T] fp32, s [T] fp32)."""
+    lib = load()
+    x, x_pre, x_post, seqlens = _flatten(x, x_pre, x_post, seqlens)
+    tok = _Tokens(x, x_pre, x_post, seqlens)
+    t = x.shape[0]
+    stats = torch.empty(t, TR_STATS_WORDS, dtype=torch.float32, device=x.device)
+    h2 = torch.empty(t, dtype=torch.float32, device=x.device)
+    s = torch.empty(t, dtype=torch.float32, device=x.device)
+    check("tr_score", lib.tr_score(tok.ref(), _ptr(stats), _ptr(h2), _ptr(s), _stream(x.device)))
+    return stats, h2, s
+
+
+def _workspace(lib, tok, device):
+    nbytes = lib.tr_workspace_bytes(tok.ref())
+    ws = torch.empty(max(nbytes, 256), dtype=torch.uint8, device=device)
+    assert ws.data_ptr() % 256 == 0
+    return ws, nbytes
+
+
+def select(x, x_pre, x_post, stats, k=None, ratio=None, lam=(1, 3), seqlens=None, h2=None, s=None, budget=None):
+    """tr_select: returns (idx int32 [sum K], role uint8 [T], cu_k list, status int32 [4]).
+
+    ``budget`` may pass explicit (ks, k1s, cu_k) lists instead of k/ratio/lam."""
+    lib = load()
+    x, x_pre, x_post, seqlens = _flatten(x, x_pre, x_post, seqlens)
+    tok = _Tokens(x, x_pre, x_post, seqlens)
+    ks, k1s, cu_k = budget if budget is not None else budgets(seqlens, k, ratio, lam)
+    dev = x.device
+    d_k = torch.tensor(ks, dtype=torch.int32, device=dev)
+    d_k1 = torch.tensor(k1s, dtype=torch.int32, device=dev)
+    d_cu = torch.tensor(cu_k, dtype=torch.int32, device=dev)
+    idx = torch.empty(max(cu_k[-1], 1), dtype=torch.int32, device=dev)
+    role = torch.empty(x.shape[0], dtype=torch.uint8, device=dev)
+    status = torch.zeros(TR_STATUS_WORDS, dtype=torch.int32, device=dev)
+    ws, nbytes = _workspace(lib, tok, dev)
+    check("tr_select", lib.tr_select(tok.ref(), _ptr(stats), _ptr(d_k), _ptr(d_k1), _ptr(d_cu), _ptr(idx),
+                                     _ptr(role), _ptr(h2), _ptr(s), _ptr(ws), nbytes, _ptr(status),
+                                     _stream(dev)))
+    return idx[:cu_k[-1]], role, cu_k, status
+
+
+@dataclass
+class ReduceResult:
+    y: torch.Tensor        # [sum K, D] kept tokens, input dtype
+    idx: torch.Tensor      # [sum K] int32 local indices, ascending per image
+    cu_k: list             # prefix sums of K_b
+    h2: torch.Tensor | None
+    s: torch.Tensor | None
+    status: torch.Tensor   # int32[4], see include/tr.h
+
+
+class Reducer:
+    """tr_reduce with buffers allocated once for a fixed batch shape.
+
+    ``run`` takes device tensors (inputs already in HBM); ``run_host`` takes
+    pinned host tensors, copies them in, reduces, and copies y and idx back.
+    """
+
+    def __init__(self, seqlens, d, dtype, device, k=None, ratio=None, lam=(1, 3), alias_pre=False, scores=False,
+                 budget=None):
+        self.lib = load()
+        self.seqlens = [int(v) for v in seqlens]
+        self.device = torch.device(device)
+        self.d, self.dtype, self.alias_pre = d, dtype, alias_pre
+        self.ks, self.k1s, self.cu_k = budget if budget is not None else budgets(self.seqlens, k, ratio, lam)
+        self.total_k = self.cu_k[-1]
+        t = sum(self.seqlens)
+        dev = self.device
+        self.d_k = torch.tensor(self.ks, dtype=torch.int32, device=dev)
+        self.d_k1 = torch.tensor(self.k1s, dtype=torch.int32, device=dev)
+        self.d_cu = torch.tensor(self.cu_k, dtype=torch.int32, device=dev)
+        self.y = torch.empty(max(self.total_k, 1), d, dtype=dtype, device=dev)
+        self.idx = torch.empty(max(self.total_k, 1), dtype=torch.int32, device=dev)
+        self.h2 = torch.empty(t, dtype=torch.float32, device=dev) if scores else None
+        self.s = torch.empty(t, dtype=torch.float32, device=dev) if scores else None
+        self.status = torch.zeros(TR_STATUS_WORDS, dtype=torch.int32, device=dev)
+        self._tok = None
+        self._ws = None
+        self._in = None
+
+    def _bind(self, x, x_pre, x_post):
+        x, x_pre, x_post, _ = _flatten(x, x_pre, x_post, self.seqlens)
+        key = (x.data_ptr(), None if x_pre is None else x_pre.data_ptr(), x_post.data_ptr())
+        if self._tok is None or self._in != key:
+            self._tok = _Tokens(x, x_pre, x_post, self.seqlens)
+            self._in = key
+            if self._ws is None:
+                self._ws, self._ws_bytes = _workspace(self.lib, self._tok, self.device)
+        return self._tok
+
+    def run(self, x, x_pre, x_post) -> ReduceResult:
+        tok = self._bind(x, x_pre, x_post)
+        check("tr_reduce", self.lib.tr_reduce(
+            tok.ref(), _ptr(self.d_k), _ptr(self.d_k1), _ptr(self.d_cu), self.total_k, _ptr(self.y),
+            _ptr(self.idx), _ptr(self.h2), _ptr(self.s), _ptr(self._ws), self._ws_bytes, _ptr(self.status),
+            _stream(self.device)))
+        return ReduceResult(self.y[:self.total_k], self.idx[:self.total_k], self.cu_k, self.h2, self.s,
+                            self.status)
+
+    def run_split(self, x, x_pre, x_post, events=None):
+        """The same three kernels as ``run`` through the three separate entry
+        points tr_score, tr_select and tr_gather, with ``events`` (four
+        torch.cuda.Event, or None) recorded before, between and after them on
+        the current stream, so each kernel can be timed inside a step."""
+        tok = self._bind(x, x_pre, x_post)
+        st = _stream(self.device)
+        lib = self.lib
+        stats = self._stats_view()
+        if events:
+            events[0].record()
+        check("tr_score", lib.tr_score(tok.ref(), _ptr(stats), _ptr(self.h2), _ptr(self.s), st))
+        if events:
+            events[1].record()
+        check("tr_select", lib.tr_select(tok.ref(), _ptr(stats), _ptr(self.d_k), _ptr(self.d_k1), _ptr(self.d_cu),
+                                         _ptr(self.idx), None, _ptr(self.h2), _ptr(self.s), _ptr(self._ws),
+                                         self._ws_bytes, _ptr(self.status), st))
+        if events:
+            events[2].record()
+        check("tr_gather", lib.tr_gather(tok.ref(), _ptr(self.d_cu), _ptr(self.idx), self.total_k, _ptr(self.y), st))
+        if events:
+            events[3].record()
+        return ReduceResult(self.y[:self.total_k], self.idx[:self.total_k], self.cu_k, self.h2, self.s,
+                            self.status)
+
+    def _stats_view(self):
+        # tr_reduce keeps the statistics at the start of the workspace; the
+        # split path uses the same bytes.
+        t = sum(self.seqlens)
+        return self._ws[: t * TR_STATS_WORDS * 4].view(torch.float32)
+
+    def alloc_device_inputs(self):
+        t = sum(self.seqlens)
+        mk = lambda: torch.empty(t, self.d, dtype=self.dtype, device=self.device)
+        return mk(), (None if self.alias_pre else mk()), mk()
+
+    def run_host(self, x_h, x_pre_h, x_post_h, dev_in, y_h, idx_h) -> ReduceResult:
+        """End-to-end: pinned host inputs -> device -> reduce -> pinned host y, idx."""
+        dx, dp, dq = dev_in
+        dx.copy_(x_h, non_blocking=True)
+        if dp is not None:
+            dp.copy_(x_pre_h, non_blocking=True)
+        dq.copy_(x_post_h, non_blocking=True)
+        r = self.run(dx, dp, dq)
+        y_h.copy_(r.y, non_blocking=True)
+        idx_h.copy_(r.idx, non_blocking=True)
+        return r
+
+
+def reduce(x, x_pre, x_post, k=None, ratio=None, lam=(1, 3), seqlens=None, scores=False, budget=None):
+    """tr_reduce in one call: returns a ReduceResult (device tensors)."""
+    x2, p2, q2, seqlens = _flatten(x, x_pre, x_post, seqlens)
+    r = Reducer(seqlens, x2.shape[1], x2.dtype, x2.device, k=k, ratio=ratio, lam=lam, alias_pre=p2 is None,
+                scores=scores, budget=budget)
+    out = r.run(x2, p2, q2)
+    return out

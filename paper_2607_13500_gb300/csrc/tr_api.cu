@@ -1,0 +1,185 @@
+// Host side of the C ABI declared in include/tr.h: argument checks, budgets,
+// workspace carving and the launch sequence score -> select -> gather.
+#include <climits>
+
+#include "tr_internal.cuh"
+
+using namespace tr;
+
+namespace {
+
+bool misaligned(const void *p, uintptr_t a) { return p && (reinterpret_cast<uintptr_t>(p) % a) != 0; }
+
+struct Shape {
+  long long total;
+  int max_n;
+};
+
+tr_status check_tokens(const tr_tokens *in, Shape *sh) {
+  if (!in || !in->x || !in->x_post) return TR_ERR_ARG;
+  if (in->dtype != TR_F32 && in->dtype != TR_BF16) return TR_ERR_DTYPE;
+  if (in->d <= 0 || in->batch < 0) return TR_ERR_ARG;
+  if (in->d > TR_MAX_D) return TR_ERR_UNSUPPORTED;
+  if ((in->d * elem_bytes(in->dtype)) % 16 != 0) return TR_ERR_ALIGN;
+  if (misaligned(in->x, 16) || misaligned(in->x_pre, 16) || misaligned(in->x_post, 16)) return TR_ERR_ALIGN;
+  if (in->cu_seqlens) {
+    if (in->total < 0 || in->max_n < 0) return TR_ERR_ARG;
+    sh->total = in->total;
+    sh->max_n = in->max_n;
+  } else {
+    if (in->n < 0) return TR_ERR_ARG;
+    sh->total = (long long)in->batch * in->n;
+    sh->max_n = in->n;
+  }
+  if (sh->max_n > TR_MAX_N) return TR_ERR_UNSUPPORTED;
+  if (sh->total > INT_MAX) return TR_ERR_UNSUPPORTED;  // kept rows are int32
+  return TR_OK;
+}
+
+tr_status check_ws(const Shape &sh, const void *ws, size_t ws_bytes) {
+  if (!ws || misaligned(ws, 256)) return TR_ERR_WORKSPACE;
+  if (ws_bytes < ws_layout(sh.total).total) return TR_ERR_WORKSPACE;
+  return TR_OK;
+}
+
+SelectArgs select_args(const tr_tokens *in, const Shape &sh, const float *stats, const int32_t *d_k,
+                       const int32_t *d_k1, const int32_t *d_cu_k, int32_t *idx, uint8_t *role,
+                       float *h2, float *s, void *ws, int32_t *d_status) {
+  SelectArgs a;
+  a.x = in->x;
+  a.x_pre = in->x_pre;
+  a.x_post = in->x_post;
+  a.dtype = in->dtype;
+  a.d = in->d;
+  a.batch = in->batch;
+  a.n_uniform = in->cu_seqlens ? 0 : in->n;
+  a.cu_seqlens = in->cu_seqlens;
+  a.stats = stats;
+  a.k = d_k;
+  a.k1 = d_k1;
+  a.cu_k = d_cu_k;
+  a.idx = idx;
+  a.role = role;
+  a.h2 = h2;
+  a.s = s;
+  a.exact = reinterpret_cast<ExactRec *>(static_cast<char *>(ws) + ws_layout(sh.total).exact);
+  a.status = d_status;
+  a.bounds = certification_bounds(in->d, in->dtype);
+  a.max_n = sh.max_n;
+  return a;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *tr_status_string(int32_t status) {
+  switch (status) {
+    case TR_OK: return "ok";
+    case TR_ERR_ARG: return "invalid argument";
+    case TR_ERR_BUDGET: return "invalid budget";
+    case TR_ERR_DTYPE: return "unsupported dtype";
+    case TR_ERR_ALIGN: return "misaligned row or pointer (rows must be a multiple of 16 bytes)";
+    case TR_ERR_WORKSPACE: return "workspace missing, misaligned or too small";
+    case TR_ERR_CUDA: return "CUDA launch failed";
+    case TR_ERR_UNSUPPORTED: return "size above the supported maximum";
+    default: return "unknown status";
+  }
+}
+
+const char *tr_version(void) { return "libtr 0.1 (sm_103a)"; }
+
+tr_status tr_budgets(int32_t batch, const int32_t *h_seqlens, int32_t k, int32_t r_num, int32_t r_den,
+                     int32_t lam_num, int32_t lam_den, int32_t *h_k, int32_t *h_k1, int32_t *h_cu_k) {
+  if (batch < 0 || !h_cu_k || (batch > 0 && (!h_seqlens || !h_k || !h_k1))) return TR_ERR_ARG;
+  if (lam_den <= 0 || lam_num < 0 || lam_num > lam_den) return TR_ERR_BUDGET;
+  if (k <= 0 && (r_den <= 0 || r_num <= 0 || r_num > r_den)) return TR_ERR_BUDGET;
+  long long cum = 0;
+  h_cu_k[0] = 0;
+  for (int b = 0; b < batch; ++b) {
+    const long long n = h_seqlens[b];
+    if (n < 0) return TR_ERR_ARG;
+    long long kb;
+    if (k > 0)
+      kb = k;
+    else
+      kb = n == 0 ? 0 : (n * r_num / r_den > 0 ? n * r_num / r_den : 1);
+    if (kb > n) return TR_ERR_BUDGET;
+    cum += kb;
+    if (cum > INT_MAX) return TR_ERR_UNSUPPORTED;
+    h_k[b] = (int32_t)kb;
+    h_k1[b] = (int32_t)(kb * lam_num / lam_den);
+    h_cu_k[b + 1] = (int32_t)cum;
+  }
+  return TR_OK;
+}
+
+size_t tr_workspace_bytes(const tr_tokens *in) {
+  Shape sh;
+  if (check_tokens(in, &sh) != TR_OK) return 0;
+  return ws_layout(sh.total).total;
+}
+
+tr_status tr_score(const tr_tokens *in, float *stats, float *h2, float *s, void *stream) {
+  Shape sh;
+  tr_status rc = check_tokens(in, &sh);
+  if (rc != TR_OK) return rc;
+  if (!stats) return TR_ERR_ARG;
+  if (misaligned(stats, 16) || misaligned(h2, 4) || misaligned(s, 4)) return TR_ERR_ALIGN;
+  cudaError_t err = launch_score(in->x, in->x_pre, in->x_post, in->dtype, in->d, sh.total, stats, h2, s,
+                                 static_cast<cudaStream_t>(stream));
+  return err == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+}
+
+tr_status tr_select(const tr_tokens *in, const float *stats, const int32_t *d_k, const int32_t *d_k1,
+                    const int32_t *d_cu_k, int32_t *idx, uint8_t *role, float *h2, float *s, void *ws,
+                    size_t ws_bytes, int32_t *d_status, void *stream) {
+  Shape sh;
+  tr_status rc = check_tokens(in, &sh);
+  if (rc != TR_OK) return rc;
+  if (in->batch > 0 && (!stats || !d_k || !d_k1 || !d_cu_k || !idx)) return TR_ERR_ARG;
+  if (misaligned(stats, 16)) return TR_ERR_ALIGN;
+  if ((rc = check_ws(sh, ws, ws_bytes)) != TR_OK) return rc;
+  SelectArgs a = select_args(in, sh, stats, d_k, d_k1, d_cu_k, idx, role, h2, s, ws, d_status);
+  cudaError_t err = launch_select(a, static_cast<cudaStream_t>(stream));
+  return err == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+}
+
+tr_status tr_reduce(const tr_tokens *in, const int32_t *d_k, const int32_t *d_k1, const int32_t *d_cu_k,
+                    int32_t total_k, void *y, int32_t *idx, float *h2, float *s, void *ws, size_t ws_bytes,
+                    int32_t *d_status, void *stream) {
+  Shape sh;
+  tr_status rc = check_tokens(in, &sh);
+  if (rc != TR_OK) return rc;
+  if (total_k < 0 || total_k > sh.total) return TR_ERR_BUDGET;
+  if (in->batch > 0 && (!d_k || !d_k1 || !d_cu_k || !idx || (total_k > 0 && !y))) return TR_ERR_ARG;
+  if (misaligned(y, 16)) return TR_ERR_ALIGN;
+  if ((rc = check_ws(sh, ws, ws_bytes)) != TR_OK) return rc;
+  const WsLayout lay = ws_layout(sh.total);
+  char *w = static_cast<char *>(ws);
+  float *stats = reinterpret_cast<float *>(w + lay.stats);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t err = launch_score(in->x, in->x_pre, in->x_post, in->dtype, in->d, sh.total, stats, h2, s, st);
+  if (err != cudaSuccess) return TR_ERR_CUDA;
+  SelectArgs a = select_args(in, sh, stats, d_k, d_k1, d_cu_k, idx, nullptr, h2, s, ws, d_status);
+  err = launch_select(a, st);
+  if (err != cudaSuccess) return TR_ERR_CUDA;
+  err = launch_gather(in->x, sh.total, in->dtype, in->d, in->batch, in->cu_seqlens ? 0 : in->n, in->cu_seqlens,
+                      d_cu_k, idx, total_k, y, st);
+  return err == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+}
+
+tr_status tr_gather(const tr_tokens *in, const int32_t *d_cu_k, const int32_t *idx, int32_t total_k, void *y,
+                    void *stream) {
+  Shape sh;
+  tr_status rc = check_tokens(in, &sh);
+  if (rc != TR_OK) return rc;
+  if (total_k < 0 || total_k > sh.total) return TR_ERR_BUDGET;
+  if (total_k > 0 && (!d_cu_k || !idx || !y || in->batch == 0)) return TR_ERR_ARG;
+  if (misaligned(y, 16)) return TR_ERR_ALIGN;
+  cudaError_t err = launch_gather(in->x, sh.total, in->dtype, in->d, in->batch, in->cu_seqlens ? 0 : in->n,
+                                  in->cu_seqlens, d_cu_k, idx, total_k, y, static_cast<cudaStream_t>(stream));
+  return err == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+}
+
+}  // extern "C"

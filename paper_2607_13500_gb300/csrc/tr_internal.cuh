@@ -1,0 +1,140 @@
+// Internal declarations shared by the CUDA translation units of libtr.
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+#include "tr.h"
+
+namespace tr {
+
+// ---------------------------------------------------------------- launch shapes
+constexpr int kScoreWarps = 8;        // rows (one per warp) in flight per score CTA
+constexpr int kScoreBatch = 4;        // 16-byte chunks a lane loads per stream before it computes
+constexpr int kSelectThreads = 1024;  // one select CTA per image
+constexpr int kGatherWarps = 8;
+
+// ---------------------------------------------------------------- exact sums
+// A non-negative integer magnitude times a power of two, with a sign:
+//   value = (-1)^neg * sum_i l[i] * 2^(32 * (i + e)),  n limbs in use (n = 0 means 0).
+constexpr int kBigLimbs = 8;
+struct Big {
+  uint32_t l[kBigLimbs];
+  int16_t e;
+  uint8_t n;
+  uint8_t neg;
+};
+
+// Exact per-row sums of Eq. 3-4 (L1 = sum|x|, S2 = sum x^2) and of Eq. 6
+// (P = sum x'x'', A = sum x'^2, B = sum x''^2).
+enum : uint32_t {
+  kRecNonFiniteX = 1u,   // x holds Inf/NaN: ranks last by importance
+  kRecNonFiniteS = 2u,   // x' or x'' holds Inf/NaN: sorts last by s
+  kRecOverflowL = 4u,    // L1 or S2 did not fit kBigLimbs limbs
+  kRecOverflowS = 8u,    // P, A or B did not fit kBigLimbs limbs
+};
+struct ExactRec {
+  Big l1, s2, a, b, p;
+  uint32_t flags_l;  // kRecNonFiniteX | kRecOverflowL, valid once L1, S2 are filled
+  uint32_t flags_s;  // kRecNonFiniteS | kRecOverflowS, valid once P, A, B are filled
+  uint32_t pad;
+};
+static_assert(sizeof(ExactRec) % 16 == 0, "ExactRec records keep 16-byte alignment");
+
+// ---------------------------------------------------------------- error bounds
+// Rounding depth of the fp32 sums L1, S2, A, B in the score kernel: each term
+// goes through at most this many rounded additions (tree inside a 16-byte
+// chunk, one accumulation per batch of kScoreBatch chunks, the tree over the
+// kScoreBatch accumulators, the 32-lane butterfly), plus one rounding of the
+// square itself for fp32 inputs (bf16 squares and products are exact in fp32).
+__host__ __device__ inline int elem_bytes(int dtype) { return dtype == TR_BF16 ? 2 : 4; }
+
+__host__ __device__ inline int score_depth(int d, int dtype) {
+  const int per_chunk = 16 / elem_bytes(dtype);
+  const int tree = dtype == TR_BF16 ? 3 : 2;
+  const int nchunks = d / per_chunk;
+  const int lane_chunks = (nchunks + 31) / 32;
+  const int batches = (lane_chunks + kScoreBatch - 1) / kScoreBatch;
+  int log_batch = 0;
+  while ((1 << log_batch) < kScoreBatch) ++log_batch;
+  return tree + batches + log_batch + 5 + (dtype == TR_BF16 ? 0 : 1);
+}
+
+// Certification bounds for the float selection keys (see the select kernel):
+//  * importance key R32 = fp32(L1^2 / S2): R32 = R (1 + delta), |delta| <= rho_r;
+//  * consistency key s32 = fp32(P / sqrt(A B)): |s32 - s| <= es_abs + es_rel |s32|.
+struct Bounds {
+  double rho_r;
+  double es_abs;
+  double es_rel;
+};
+
+inline Bounds certification_bounds(int d, int dtype) {
+  const double u = 1.0 / 16777216.0;  // fp32 unit roundoff 2^-24
+  const int h = score_depth(d, dtype);
+  const double g = h * u / (1.0 - h * u);  // gamma_h
+  const int per_chunk = 16 / elem_bytes(dtype);
+  const double lane_terms = (double)((d / per_chunk + 31) / 32) * per_chunk;
+  // P = P_hi + P_lo is exact up to the rounding of the P_lo additions:
+  // at most u^2 (lane_terms^2 / 2 + 12 d) sum|x'x''| (doubled for fp32
+  // inputs, whose product errors also enter P_lo), and sum|x'x''| <= sqrt(A B).
+  double ep = 2.0 * u * u * (lane_terms * lane_terms + 12.0 * d) + 0x1p-52;
+  if (dtype != TR_BF16) ep *= 2.0;
+  Bounds b;
+  // R^ = L1^2(1+d1)^2 / (S2(1+d2)) rounded twice (fp64 division, fp32 key);
+  // 2^-30 covers the absolute error of subnormal squares when S2 >= 2^-100.
+  b.rho_r = (1.0 + g) * (1.0 + g) / (1.0 - g) * (1.0 + 0x1p-52) * (1.0 + u) - 1.0 + 0x1p-30;
+  // s^ = (P + e_p sqrt(AB)) / sqrt(A B (1+da)(1+db)), then rounded to fp32;
+  // 2^-34 covers underflowed squares and products when A, B >= 2^-100.
+  b.es_rel = 1.02 * (g / (1.0 - g) + u + 0x1p-34);
+  b.es_abs = 1.02 * (ep / (1.0 - g)) + 0x1p-34;
+  return b;
+}
+
+// Sums below kTiny or above kHuge (or non-finite) are outside the fp32 error
+// model above (underflow, overflow): such rows are settled exactly.
+constexpr float kTiny = 0x1p-100f;
+constexpr float kHuge = 0x1p+100f;
+
+// ---------------------------------------------------------------- workspace
+inline size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// [stats: total x TR_STATS_WORDS fp32][exact records: total x ExactRec]
+struct WsLayout {
+  size_t stats, exact, total;
+};
+inline WsLayout ws_layout(long long total_rows) {
+  WsLayout w;
+  w.stats = 0;
+  w.exact = align_up(w.stats + (size_t)total_rows * TR_STATS_WORDS * sizeof(float), 256);
+  w.total = align_up(w.exact + (size_t)total_rows * sizeof(ExactRec), 256);
+  return w;
+}
+
+// ---------------------------------------------------------------- launchers
+struct SelectArgs {
+  const void *x, *x_pre, *x_post;
+  int dtype, d, batch, n_uniform;
+  const int32_t *cu_seqlens;
+  const float *stats;
+  const int32_t *k, *k1, *cu_k;
+  int32_t *idx;
+  uint8_t *role;      // or NULL
+  float *h2, *s;      // exact fix-ups, or NULL
+  ExactRec *exact;    // [total] scratch
+  int32_t *status;    // or NULL
+  Bounds bounds;
+  int max_n;
+};
+
+size_t select_smem_bytes(int max_n);  // dynamic shared memory of one select CTA
+cudaError_t launch_score(const void *x, const void *x_pre, const void *x_post, int dtype, int d, long long total,
+                         float *stats, float *h2, float *s, cudaStream_t st);
+cudaError_t launch_select(const SelectArgs &a, cudaStream_t st);
+cudaError_t launch_gather(const void *x, long long total_rows, int dtype, int d, int batch, int n_uniform,
+                          const int32_t *cu_seqlens, const int32_t *cu_k, const int32_t *idx, int total_k, void *y,
+                          cudaStream_t st);
+
+}  // namespace tr

@@ -1,0 +1,202 @@
+// Scoring pass: per-token sums for the Renyi-2 entropy (Eq. 3-4) and the
+// consistency signal (Eq. 6) in one read of x, x', x''.
+//
+// One warp per row; lane l reads 16-byte chunks l, l+32, l+64, ... of each of
+// the three streams (fully coalesced 512-byte warp requests), kScoreBatch
+// chunks per stream in flight before any arithmetic.  L1, S2, A, B are fp32
+// sums with a fixed, shallow rounding depth (score_depth); P = x'.x'' is
+// accumulated error-free as a double-float (P_hi + P_lo) with TwoSum, since
+// the ordering by s needs it far more precisely than fp32 gives.
+#include <cmath>
+
+#include "tr_internal.cuh"
+
+namespace tr {
+namespace {
+
+__device__ __forceinline__ uint4 ld_stream(const uint4 *p) {
+  uint4 r;
+  asm("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+      : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+      : "l"(p));
+  return r;
+}
+
+// Error-free sum: s + e = a + b exactly (Knuth's TwoSum, no ordering assumption).
+__device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
+  s = __fadd_rn(a, b);
+  const float bb = __fsub_rn(s, a);
+  const float aa = __fsub_rn(s, bb);
+  e = __fadd_rn(__fsub_rn(a, aa), __fsub_rn(b, bb));
+}
+
+__device__ __forceinline__ float lo_bf16(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float hi_bf16(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+
+struct Acc {
+  float l1, s2, a, b;
+};
+
+// Eight bf16 elements of each stream: tree sums of depth 3 for L1, S2, A, B
+// (bf16 squares are exact in fp32); P terms (exact products) go through TwoSum.
+__device__ __forceinline__ void chunk_bf16(const uint4 &vx, const uint4 &vp, const uint4 &vq, Acc &acc, float &ph,
+                                           float &pl) {
+  const uint32_t wx[4] = {vx.x, vx.y, vx.z, vx.w};
+  const uint32_t wp[4] = {vp.x, vp.y, vp.z, vp.w};
+  const uint32_t wq[4] = {vq.x, vq.y, vq.z, vq.w};
+  float l[4], s[4], a[4], b[4];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float x0 = lo_bf16(wx[i]), x1 = hi_bf16(wx[i]);
+    const float p0 = lo_bf16(wp[i]), p1 = hi_bf16(wp[i]);
+    const float q0 = lo_bf16(wq[i]), q1 = hi_bf16(wq[i]);
+    l[i] = fabsf(x0) + fabsf(x1);
+    s[i] = fmaf(x0, x0, x1 * x1);
+    a[i] = fmaf(p0, p0, p1 * p1);
+    b[i] = fmaf(q0, q0, q1 * q1);
+    float t, e;
+    two_sum(ph, p0 * q0, t, e);
+    ph = t;
+    pl += e;
+    two_sum(ph, p1 * q1, t, e);
+    ph = t;
+    pl += e;
+  }
+  acc.l1 += (l[0] + l[1]) + (l[2] + l[3]);
+  acc.s2 += (s[0] + s[1]) + (s[2] + s[3]);
+  acc.a += (a[0] + a[1]) + (a[2] + a[3]);
+  acc.b += (b[0] + b[1]) + (b[2] + b[3]);
+}
+
+// Four fp32 elements of each stream: tree depth 2; products split exactly
+// into p + pe with an FMA, both parts enter the double-float P.
+__device__ __forceinline__ void chunk_f32(const uint4 &vx, const uint4 &vp, const uint4 &vq, Acc &acc, float &ph,
+                                          float &pl) {
+  const float x[4] = {__uint_as_float(vx.x), __uint_as_float(vx.y), __uint_as_float(vx.z), __uint_as_float(vx.w)};
+  const float p[4] = {__uint_as_float(vp.x), __uint_as_float(vp.y), __uint_as_float(vp.z), __uint_as_float(vp.w)};
+  const float q[4] = {__uint_as_float(vq.x), __uint_as_float(vq.y), __uint_as_float(vq.z), __uint_as_float(vq.w)};
+  acc.l1 += (fabsf(x[0]) + fabsf(x[1])) + (fabsf(x[2]) + fabsf(x[3]));
+  acc.s2 += fmaf(x[0], x[0], x[1] * x[1]) + fmaf(x[2], x[2], x[3] * x[3]);
+  acc.a += fmaf(p[0], p[0], p[1] * p[1]) + fmaf(p[2], p[2], p[3] * p[3]);
+  acc.b += fmaf(q[0], q[0], q[1] * q[1]) + fmaf(q[2], q[2], q[3] * q[3]);
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const float pr = p[i] * q[i];
+    const float pe = fmaf(p[i], q[i], -pr);
+    float t, e;
+    two_sum(ph, pr, t, e);
+    ph = t;
+    pl += e + pe;
+  }
+}
+
+template <bool kBf16>
+__global__ void __launch_bounds__(kScoreWarps * 32)
+    k_score(const uint4 *__restrict__ x, const uint4 *__restrict__ xp, const uint4 *__restrict__ xq, int nchunks,
+            long long total, float4 *__restrict__ stats, float *__restrict__ h2, float *__restrict__ s_out) {
+  const int lane = threadIdx.x & 31;
+  const long long stride = (long long)gridDim.x * kScoreWarps;
+  for (long long row = (long long)blockIdx.x * kScoreWarps + (threadIdx.x >> 5); row < total; row += stride) {
+    const uint4 *rx = x + row * nchunks;
+    const uint4 *rp = xp + row * nchunks;
+    const uint4 *rq = xq + row * nchunks;
+    Acc acc[kScoreBatch];
+#pragma unroll
+    for (int u = 0; u < kScoreBatch; ++u) acc[u] = Acc{0.f, 0.f, 0.f, 0.f};
+    float ph = 0.f, pl = 0.f;
+    for (int c0 = lane; c0 < nchunks; c0 += 32 * kScoreBatch) {
+      uint4 vx[kScoreBatch], vp[kScoreBatch], vq[kScoreBatch];
+#pragma unroll
+      for (int u = 0; u < kScoreBatch; ++u) {
+        const int c = c0 + 32 * u;
+        if (c < nchunks) {
+          vx[u] = ld_stream(rx + c);
+          vp[u] = ld_stream(rp + c);
+          vq[u] = ld_stream(rq + c);
+        } else {
+          vx[u] = vp[u] = vq[u] = make_uint4(0u, 0u, 0u, 0u);
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kScoreBatch; ++u) {
+        if (kBf16)
+          chunk_bf16(vx[u], vp[u], vq[u], acc[u], ph, pl);
+        else
+          chunk_f32(vx[u], vp[u], vq[u], acc[u], ph, pl);
+      }
+    }
+    static_assert(kScoreBatch == 4, "the accumulator tree below assumes 4 accumulators");
+    float l1 = (acc[0].l1 + acc[1].l1) + (acc[2].l1 + acc[3].l1);
+    float s2 = (acc[0].s2 + acc[1].s2) + (acc[2].s2 + acc[3].s2);
+    float sa = (acc[0].a + acc[1].a) + (acc[2].a + acc[3].a);
+    float sb = (acc[0].b + acc[1].b) + (acc[2].b + acc[3].b);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      l1 += __shfl_xor_sync(0xffffffffu, l1, o);
+      s2 += __shfl_xor_sync(0xffffffffu, s2, o);
+      sa += __shfl_xor_sync(0xffffffffu, sa, o);
+      sb += __shfl_xor_sync(0xffffffffu, sb, o);
+      const float oh = __shfl_xor_sync(0xffffffffu, ph, o);
+      const float ol = __shfl_xor_sync(0xffffffffu, pl, o);
+      float t, e;
+      two_sum(ph, oh, t, e);
+      ph = t;
+      pl = pl + ol + e;
+    }
+    if (lane == 0) {
+      stats[2 * row] = make_float4(l1, s2, sa, sb);
+      stats[2 * row + 1] = make_float4(ph, pl, 0.f, 0.f);
+      if (h2) h2[row] = l1 > 0.f ? (float)log((double)l1 * (double)l1 / (double)s2) : 0.f;
+      if (s_out)
+        s_out[row] = (sa > 0.f && sb > 0.f) ? (float)(((double)ph + (double)pl) / sqrt((double)sa * (double)sb)) : 0.f;
+    }
+  }
+}
+
+struct DevInfo {
+  int sms = 0;
+  int blocks_per_sm[2] = {0, 0};
+};
+
+DevInfo &dev_info(int dev) {
+  static DevInfo info[64];
+  return info[dev & 63];
+}
+
+}  // namespace
+
+cudaError_t launch_score(const void *x, const void *x_pre, const void *x_post, int dtype, int d, long long total,
+                         float *stats, float *h2, float *s, cudaStream_t st) {
+  if (total == 0) return cudaSuccess;
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err != cudaSuccess) return err;
+  DevInfo &info = dev_info(dev);
+  const int which = dtype == TR_BF16 ? 1 : 0;
+  if (info.blocks_per_sm[which] == 0) {
+    // Benign race: concurrent first calls compute the same numbers.
+    int sms = 0, bps = 0;
+    err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (err != cudaSuccess) return err;
+    err = which ? cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, k_score<true>, kScoreWarps * 32, 0)
+                : cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, k_score<false>, kScoreWarps * 32, 0);
+    if (err != cudaSuccess) return err;
+    info.sms = sms;
+    info.blocks_per_sm[which] = bps > 0 ? bps : 1;
+  }
+  const long long need = (total + kScoreWarps - 1) / kScoreWarps;
+  const long long cap = (long long)info.sms * info.blocks_per_sm[which];
+  const int grid = (int)(need < cap ? need : cap);
+  const int nchunks = d * elem_bytes(dtype) / 16;
+  const uint4 *px = static_cast<const uint4 *>(x);
+  const uint4 *pp = static_cast<const uint4 *>(x_pre ? x_pre : x);
+  const uint4 *pq = static_cast<const uint4 *>(x_post);
+  float4 *ps = reinterpret_cast<float4 *>(stats);
+  if (which)
+    k_score<true><<<grid, kScoreWarps * 32, 0, st>>>(px, pp, pq, nchunks, total, ps, h2, s);
+  else
+    k_score<false><<<grid, kScoreWarps * 32, 0, st>>>(px, pp, pq, nchunks, total, ps, h2, s);
+  return cudaGetLastError();
+}
+
+}  // namespace tr

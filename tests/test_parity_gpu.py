@@ -1,0 +1,220 @@
+"""CUDA path versus the CPU oracle, element by element, through the C ABI.
+
+Kept indices and gathered rows must match bit for bit; H2 within 1e-5
+relative (fp32 inputs) or 2e-3 relative (bf16 inputs) and s within 1e-5
+absolute.  Small cases check every image; the full-size workloads (the
+launch configuration bench.py times) check sampled images one by one.
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+
+pytestmark = pytest.mark.gpu
+
+H2_RTOL = {torch.float32: 1e-5, torch.bfloat16: 2e-3}
+S_ATOL = 1e-5
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("needs a CUDA GPU")
+    from paper_2607_13500_gb300 import _build
+    _build.build()
+
+
+def _alt():
+    import paper_2607_13500_gb300 as altr
+    return altr
+
+
+def _f64(t):
+    return t.float().cpu().numpy().astype(np.float64)
+
+
+def _bits(t):
+    return t.view(torch.int16) if t.dtype == torch.bfloat16 else t.view(torch.int32)
+
+
+def check_reduce(x, x_pre, x_post, seqlens, budget, images=None, alias=False, expect_nonfinite=False):
+    """Runs tr_reduce on the device and compares sampled images with the oracle."""
+    altr = _alt()
+    dev = torch.device("cuda")
+    dx, dq = x.to(dev), x_post.to(dev)
+    dp = None if alias else x_pre.to(dev)
+    r = altr.reduce(dx, dp, dq, seqlens=seqlens, budget=budget, scores=True)
+    torch.cuda.synchronize()
+    ks, k1s, cu = budget
+    status = r.status.cpu().tolist()
+    assert status[1] == 0, f"unresolved rows: {status}"
+    assert status[3] == 0, f"invalid budget or kept-count mismatch: {status}"
+    if expect_nonfinite:
+        assert status[0] > 0
+    idx = r.idx.cpu().numpy()
+    y = r.y.cpu()
+    h2 = r.h2.cpu().numpy().astype(np.float64)
+    s = r.s.cpu().numpy().astype(np.float64)
+    offs = np.concatenate([[0], np.cumsum(seqlens)]).astype(np.int64)
+    images = range(len(seqlens)) if images is None else images
+    pre = x if alias else x_pre
+    for b in images:
+        o0, o1 = int(offs[b]), int(offs[b + 1])
+        xb, pb, qb = _f64(x[o0:o1]), _f64(pre[o0:o1]), _f64(x_post[o0:o1])
+        ref = oracle.select_image(xb, pb, qb, ks[b], k1s[b])
+        got = idx[cu[b]:cu[b + 1]]
+        assert np.array_equal(got, ref["kept"]), (b, np.setdiff1d(got, ref["kept"]), np.setdiff1d(ref["kept"], got))
+        want_rows = x[o0:o1][torch.from_numpy(ref["kept"].astype(np.int64))]
+        assert torch.equal(_bits(y[cu[b]:cu[b + 1]]), _bits(want_rows)), b
+        fin = np.isfinite(ref["h2"])
+        rt = H2_RTOL[x.dtype]
+        assert np.all(np.abs(h2[o0:o1][fin] - ref["h2"][fin]) <= rt * np.abs(ref["h2"][fin]) + 1e-6), b
+        assert np.array_equal(np.isneginf(h2[o0:o1][~fin]), np.ones((~fin).sum(), bool))
+        sf = np.isfinite(ref["s"])
+        assert np.all(np.abs(s[o0:o1][sf] - ref["s"][sf]) <= S_ATOL), b
+    return status
+
+
+def _budget(w, k=None, ratio=None, lam=(1, 3)):
+    return _alt().budgets(w.seqlens, k=k, ratio=ratio, lam=lam)
+
+
+# ---------------------------------------------------------------- the five workloads, shrunk
+SMALL = [
+    ("single_clip336", {}, [dict(k=64)]),
+    ("llava576", dict(batch=6), [dict(k=64), dict(k=128), dict(k=192)]),
+    ("multitile2880", dict(batch=2), [dict(k=160), dict(k=320)]),
+    ("ragged_dynres", dict(batch=5, n=(256, 3000)), [dict(ratio=(1, 9)), dict(ratio=(2, 9))]),
+    ("video6272", dict(batch=2), [dict(ratio=(1, 8))]),
+]
+
+
+@pytest.mark.parametrize("name,over,budgets", SMALL, ids=[s[0] for s in SMALL])
+def test_workloads_small(name, over, budgets):
+    w = synth.make(name, seed=11, device="cuda", **over)
+    x, xp, xq = w.x.cpu(), w.x_pre.cpu(), w.x_post.cpu()
+    for bk in budgets:
+        check_reduce(x, xp, xq, w.seqlens, _budget(w, **bk))
+
+
+def test_lambda_extremes_and_alias():
+    w = synth.make("llava576", seed=12, device="cuda", batch=3, d=1024)
+    x, xp, xq = w.x.cpu(), w.x_pre.cpu(), w.x_post.cpu()
+    for lam in [(0, 1), (1, 1), (1, 2)]:
+        check_reduce(x, xp, xq, w.seqlens, _budget(w, k=100, lam=lam))
+    check_reduce(x, x, xq, w.seqlens, _budget(w, k=100), alias=True)
+
+
+def test_score_and_select_entry_points():
+    altr = _alt()
+    w = synth.make("llava576", seed=13, device="cuda", batch=2, d=2048)
+    stats, h2, s = altr.score(w.x, w.x_pre, w.x_post, seqlens=w.seqlens)
+    ks, k1s, cu = _budget(w, k=96)
+    idx, role, cu_k, status = altr.select(w.x, w.x_pre, w.x_post, stats, seqlens=w.seqlens, budget=(ks, k1s, cu))
+    torch.cuda.synchronize()
+    role = role.cpu().numpy()
+    for b in range(2):
+        sl = slice(b * 576, (b + 1) * 576)
+        ref = oracle.select_image(_f64(w.x[sl]), _f64(w.x_pre[sl]), _f64(w.x_post[sl]), ks[b], k1s[b])
+        assert set(np.nonzero(role[sl] == 1)[0].tolist()) == set(ref["imp"].tolist())
+        assert set(np.nonzero(role[sl] == 2)[0].tolist()) == set(ref["div"].tolist())
+        assert np.array_equal(idx[cu[b]:cu[b + 1]].cpu().numpy(), ref["kept"])
+    st = stats.cpu().numpy().astype(np.float64)
+    xx = _f64(w.x)
+    assert np.allclose(st[:, 0], np.abs(xx).sum(1), rtol=2e-6)
+    assert np.allclose(st[:, 1], (xx * xx).sum(1), rtol=2e-6)
+    p = (_f64(w.x_pre) * _f64(w.x_post)).sum(1)
+    scale = np.sqrt((_f64(w.x_pre) ** 2).sum(1) * (_f64(w.x_post) ** 2).sum(1))
+    assert np.all(np.abs(st[:, 4] + st[:, 5] - p) <= 1e-9 * scale)
+
+
+# ---------------------------------------------------------------- edge cases
+def _rows(n, d, seed, dtype=torch.bfloat16):
+    g = torch.Generator().manual_seed(seed)
+    mk = lambda: torch.randn(n, d, generator=g).to(dtype)
+    return mk(), mk(), mk()
+
+
+def test_edge_budgets_and_sizes():
+    d = 256
+    x, xp, xq = _rows(40, d, 1)
+    # K = N, K = 0 (explicit), N = 1, an empty image in a ragged batch
+    check_reduce(x, xp, xq, [40], ([40], [13], [0, 40]))
+    check_reduce(x, xp, xq, [40], ([0], [0], [0, 0]))
+    check_reduce(x, xp, xq, [1, 39], ([1, 5], [0, 1], [0, 1, 6]))
+    check_reduce(x, xp, xq, [20, 0, 20], ([7, 0, 20], [2, 0, 6], [0, 7, 7, 27]))
+    # several tiles and a ragged tail: N not a multiple of anything
+    x, xp, xq = _rows(1000, 1032, 2)
+    check_reduce(x, xp, xq, [333, 1, 666], ([100, 1, 66], [33, 0, 22], [0, 100, 101, 167]))
+
+
+def test_exact_ties_and_degenerate_rows():
+    d, n = 512, 96
+    g = torch.Generator().manual_seed(3)
+    base = torch.randn(d, generator=g).to(torch.bfloat16)
+    x = torch.stack([base[torch.randperm(d, generator=g)] for _ in range(n)])  # channel permutations: R ties
+    other = torch.randn(d, generator=g).to(torch.bfloat16)
+    perms = [torch.randperm(d, generator=g) for _ in range(n)]
+    xp = torch.stack([base[p] for p in perms])
+    xq = torch.stack([other[p] for p in perms])                                # P, A, B tie exactly
+    x[5] = 0
+    x[6] = 0
+    x[7, :] = 0
+    x[7, 3] = 2.5                                                               # one-hot: R = 1 like zero rows
+    x[8] = x[9]                                                                 # duplicate rows
+    xq[10] = 0                                                                  # zero norm: s = 0
+    for k, k1 in [(30, 10), (96, 32), (50, 50), (40, 0)]:
+        check_reduce(x, xp, xq, [n], ([k], [k1], [0, k]))
+    # equal magnitudes with random signs: every row has R = D exactly
+    sgn = torch.randint(0, 2, (n, d), generator=g) * 2 - 1
+    mags = torch.tensor([0.375, 1.5, 3.0]).repeat(n // 3 + 1)[:n, None]
+    xe = (sgn * mags).to(torch.bfloat16)
+    check_reduce(xe, xp, xq, [n], ([40], [13], [0, 40]))
+
+
+def test_nonfinite_huge_and_tiny_rows():
+    n, d = 64, 256
+    x, xp, xq = _rows(n, d, 4)
+    x[3, 17] = float("nan")
+    x[4, 0] = float("inf")
+    xp[5, 2] = float("-inf")
+    xq[6, 9] = float("nan")
+    x[10] *= 2.0 ** 70                   # squares overflow fp32: settled exactly
+    x[11] *= 2.0 ** -70                  # squares underflow fp32: settled exactly
+    xp[12] *= 2.0 ** 80
+    xq[13] *= 2.0 ** -75
+    for k, k1 in [(64, 60), (40, 13), (20, 0)]:
+        check_reduce(x, xp, xq, [n], ([k], [k1], [0, k]), expect_nonfinite=True)
+
+
+def test_fp32_wide_range():
+    n, d = 300, 1024
+    g = torch.Generator().manual_seed(5)
+    x = torch.randn(n, d, generator=g) * torch.exp2(torch.randint(-20, 20, (n, d), generator=g).float())
+    xp = torch.randn(n, d, generator=g)
+    xq = 0.5 * xp + torch.randn(n, d, generator=g) * torch.exp2(torch.randint(-10, 10, (n, d), generator=g).float())
+    check_reduce(x, xp, xq, [n], ([90], [30], [0, 90]))
+    check_reduce(x, xp, xq, [100, 200], ([33, 66], [11, 22], [0, 33, 99]))
+
+
+# ---------------------------------------------------------------- full-size workloads (sampled)
+FULL = [
+    ("llava576", dict(k=192), None),
+    ("multitile2880", dict(k=320), None),
+    ("ragged_dynres", dict(ratio=(2, 9)), "largest3"),
+    ("video6272", dict(ratio=(1, 8)), [0, 7]),
+    ("single_clip336", dict(k=64), None),
+]
+
+
+@pytest.mark.parametrize("name,bk,sample", FULL, ids=[f[0] for f in FULL])
+def test_workloads_full_size(name, bk, sample):
+    w = synth.make(name, seed=0, device="cuda")
+    if sample == "largest3":
+        sample = sorted(range(w.batch), key=lambda b: -w.seqlens[b])[:2] + [0]
+    x, xp, xq = w.x.cpu(), w.x_pre.cpu(), w.x_post.cpu()
+    del w.x, w.x_pre, w.x_post
+    torch.cuda.empty_cache()
+    check_reduce(x, xp, xq, w.seqlens, _alt().budgets(w.seqlens, **bk), images=sample)
