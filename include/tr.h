@@ -166,6 +166,29 @@ tr_status tr_reduce(const tr_tokens *in, const int32_t *d_k, const int32_t *d_k1
                     int32_t total_k, void *y, int32_t *idx, float *h2, float *s, void *ws, size_t ws_bytes,
                     int32_t *d_status, void *stream);
 
+/*
+ * tr_reduce without a caller-provided workspace, for callers that cannot
+ * allocate device memory (code running inside a host framework whose
+ * allocator it cannot reach, plugins or callbacks that must not call
+ * cudaMalloc, loops that must not allocate once they run).  The paper has
+ * no counterpart: this is a deployment convenience of this library.
+ *
+ * Same arguments and results as tr_reduce, minus ws / ws_bytes.  Its scratch
+ * is a device array of TR_NOALLOC_SCRATCH_BYTES bytes inside libtr, present
+ * on every GPU that loads the library until the process exits; batches of
+ * more than TR_NOALLOC_MAX_ROWS token rows are rejected with
+ * TR_ERR_UNSUPPORTED.  The call allocates nothing.  The first call on a
+ * device looks up that array's device address (with the device current),
+ * so make the first call on each device before any stream capture.  All
+ * calls share the array: calls whose work may overlap on the GPU race and
+ * must be serialised by the caller.
+ */
+#define TR_NOALLOC_MAX_ROWS 32768
+#define TR_NOALLOC_SCRATCH_BYTES (8u << 20)
+tr_status tr_reduce_noalloc(const tr_tokens *in, const int32_t *d_k, const int32_t *d_k1, const int32_t *d_cu_k,
+                            int32_t total_k, void *y, int32_t *idx, float *h2, float *s, int32_t *d_status,
+                            void *stream);
+
 #ifdef __cplusplus
 }
 #endif
