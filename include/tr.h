@@ -107,9 +107,12 @@ size_t tr_workspace_bytes(const tr_tokens *in);
  *   stats: device fp32[total, TR_STATS_WORDS] (16-byte aligned), per row
  *          [0] L1 = sum_j |x_j|, [1] S2 = sum_j x_j^2, [2] A = sum_j x'_j^2,
  *          [3] B = sum_j x''_j^2, [4] P_hi, [5] P_lo with P = sum_j x'_j x''_j
- *          = P_hi + P_lo (double-float), [6..7] zero.  L1, S2, A, B are fp32
- *          sums of bounded rounding depth; P is accumulated error-free up to
- *          a ~1e-10 relative residue.
+ *          = P_hi + P_lo (double-float), [6] the importance key L1^2 / S2
+ *          and [7] the consistency key P / sqrt(A B), both rounded once to
+ *          fp32 and NaN when the row's sums left the fp32 error model
+ *          (non-finite, or S2, A or B outside [2^-100, 2^100]).  L1, S2, A, B
+ *          are fp32 sums of bounded rounding depth; P is accumulated
+ *          error-free up to a ~1e-10 relative residue.
  *   h2:    device fp32[total] or NULL: H2 = -log sum_j p_j^2 = log(L1^2 / S2)
  *          (Eq. 3-4); 0 for an all-zero row.
  *   s:     device fp32[total] or NULL: s = P / sqrt(A B) (Eq. 6); 0 when

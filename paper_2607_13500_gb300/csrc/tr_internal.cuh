@@ -13,7 +13,7 @@ namespace tr {
 // ---------------------------------------------------------------- launch shapes
 constexpr int kScoreWarps = 8;        // rows (one per warp) in flight per score CTA
 constexpr int kScoreBatch = 4;        // 16-byte chunks a lane loads per stream before it computes
-constexpr int kSelectThreads = 1024;  // one select CTA per image
+constexpr int kSelectThreads = 512;   // one select CTA per image
 constexpr int kGatherWarps = 8;
 
 // ---------------------------------------------------------------- exact sums
@@ -45,21 +45,16 @@ static_assert(sizeof(ExactRec) % 16 == 0, "ExactRec records keep 16-byte alignme
 
 // ---------------------------------------------------------------- error bounds
 // Rounding depth of the fp32 sums L1, S2, A, B in the score kernel: each term
-// goes through at most this many rounded additions (tree inside a 16-byte
-// chunk, one accumulation per batch of kScoreBatch chunks, the tree over the
-// kScoreBatch accumulators, the 32-lane butterfly), plus one rounding of the
-// square itself for fp32 inputs (bf16 squares and products are exact in fp32).
+// goes through the depth-3 (bf16) or depth-2 (fp32) tree of its 16-byte chunk
+// (plus the rounding of the square itself for fp32 inputs, bf16 squares being
+// exact), the chunk partials are accumulated error-free (TwoSum into a
+// double-float whose low part's own rounding is bounded separately), and the
+// final hi + lo is rounded once to fp32.
 __host__ __device__ inline int elem_bytes(int dtype) { return dtype == TR_BF16 ? 2 : 4; }
 
 __host__ __device__ inline int score_depth(int d, int dtype) {
-  const int per_chunk = 16 / elem_bytes(dtype);
-  const int tree = dtype == TR_BF16 ? 3 : 2;
-  const int nchunks = d / per_chunk;
-  const int lane_chunks = (nchunks + 31) / 32;
-  const int batches = (lane_chunks + kScoreBatch - 1) / kScoreBatch;
-  int log_batch = 0;
-  while ((1 << log_batch) < kScoreBatch) ++log_batch;
-  return tree + batches + log_batch + 5 + (dtype == TR_BF16 ? 0 : 1);
+  (void)d;
+  return dtype == TR_BF16 ? 3 + 1 : 2 + 1 + 1;
 }
 
 // Certification bounds for the float selection keys (see the select kernel):
@@ -69,27 +64,43 @@ struct Bounds {
   double rho_r;
   double es_abs;
   double es_rel;
+  // the same bounds as fp32 factors rounded outward, for tests evaluated
+  // with directed rounding:  R >= R32 * r_lo,  R <= R32 * r_hi,
+  // |s - s32| <= s_abs + s_rel |s32|
+  float r_lo, r_hi, s_abs, s_rel;
 };
 
 inline Bounds certification_bounds(int d, int dtype) {
   const double u = 1.0 / 16777216.0;  // fp32 unit roundoff 2^-24
   const int h = score_depth(d, dtype);
-  const double g = h * u / (1.0 - h * u);  // gamma_h
   const int per_chunk = 16 / elem_bytes(dtype);
-  const double lane_terms = (double)((d / per_chunk + 31) / 32) * per_chunk;
+  const double lane_chunks = (double)((d / per_chunk + 31) / 32);
+  const double lane_terms = lane_chunks * per_chunk;
+  // Double-float low parts: m additions of error terms each below u times the
+  // running sum leave at most m^2 u^2 of the sum (m = the low part's additions).
+  const double m = lane_chunks + 12.0;
+  const double g = h * u / (1.0 - h * u) + m * m * u * u + 0x1p-34;  // relative error of L1, S2, A, B
   // P = P_hi + P_lo is exact up to the rounding of the P_lo additions:
   // at most u^2 (lane_terms^2 / 2 + 12 d) sum|x'x''| (doubled for fp32
   // inputs, whose product errors also enter P_lo), and sum|x'x''| <= sqrt(A B).
   double ep = 2.0 * u * u * (lane_terms * lane_terms + 12.0 * d) + 0x1p-52;
   if (dtype != TR_BF16) ep *= 2.0;
   Bounds b;
-  // R^ = L1^2(1+d1)^2 / (S2(1+d2)) rounded twice (fp64 division, fp32 key);
-  // 2^-30 covers the absolute error of subnormal squares when S2 >= 2^-100.
-  b.rho_r = (1.0 + g) * (1.0 + g) / (1.0 - g) * (1.0 + 0x1p-52) * (1.0 + u) - 1.0 + 0x1p-30;
-  // s^ = (P + e_p sqrt(AB)) / sqrt(A B (1+da)(1+db)), then rounded to fp32;
-  // 2^-34 covers underflowed squares and products when A, B >= 2^-100.
-  b.es_rel = 1.02 * (g / (1.0 - g) + u + 0x1p-34);
+  // R32 = fl(fl(L1^2) / S2) with L1, S2 relative g: R32 / R within
+  // (1 + g)^2 / (1 - g) (1 + u)^2; 2^-30 covers subnormal squares (S2 >= 2^-100).
+  b.rho_r = (1.0 + g) * (1.0 + g) / (1.0 - g) * (1.0 + u) * (1.0 + u) - 1.0 + 0x1p-30;
+  // s32 = fl(fl(P_hi + P_lo) / fl(fl(sqrt A) fl(sqrt B))): the sums contribute
+  // g (half from A, half from B), the five fp32 roundings 5u, P's residue
+  // e_p sqrt(A B) an absolute term; 2^-34 covers underflowed squares and
+  // products when A, B >= 2^-100.
+  b.es_rel = 1.02 * (g / (1.0 - g) + 5.0 * u + 0x1p-34);
   b.es_abs = 1.02 * (ep / (1.0 - g)) + 0x1p-34;
+  // float factors: rounding a double to float moves it by at most 2^-24
+  // relative, so widening by 2^-22 before the cast keeps each one outward.
+  b.r_lo = (float)((1.0 / (1.0 + b.rho_r)) * (1.0 - 0x1p-22));
+  b.r_hi = (float)((1.0 / (1.0 - b.rho_r)) * (1.0 + 0x1p-22));
+  b.s_abs = (float)(b.es_abs * (1.0 + 0x1p-22));
+  b.s_rel = (float)(b.es_rel * (1.0 + 0x1p-22));
   return b;
 }
 

@@ -3,10 +3,13 @@
 //
 // One warp per row; lane l reads 16-byte chunks l, l+32, l+64, ... of each of
 // the three streams (fully coalesced 512-byte warp requests), kScoreBatch
-// chunks per stream in flight before any arithmetic.  L1, S2, A, B are fp32
-// sums with a fixed, shallow rounding depth (score_depth); P = x'.x'' is
-// accumulated error-free as a double-float (P_hi + P_lo) with TwoSum, since
-// the ordering by s needs it far more precisely than fp32 gives.
+// chunks per stream in flight before any arithmetic.  Each chunk's partial
+// sums of |x|, x^2, x'^2, x''^2 come from a depth-3 fp32 tree; the partials
+// are accumulated error-free as double-floats (TwoSum), so every sum carries
+// at most score_depth() roundings whatever D is.  P = x'.x'' is accumulated
+// error-free term by term, since the ordering by s needs it to far better
+// than fp32.  The epilogue rounds the sums to fp32 and derives the fp32
+// selection keys, all without fp64 (GB300's fp64 rate would stall the warp).
 #include <cmath>
 
 #include "tr_internal.cuh"
@@ -33,14 +36,31 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
 __device__ __forceinline__ float lo_bf16(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float hi_bf16(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
 
+// Double-float accumulator: hi + lo carries the sum, hi exact in TwoSum.
+struct DF {
+  float hi, lo;
+};
+__device__ __forceinline__ void df_add(DF &a, float v) {
+  float t, e;
+  two_sum(a.hi, v, t, e);
+  a.hi = t;
+  a.lo += e;
+}
+__device__ __forceinline__ void df_merge(DF &a, float hi, float lo) {
+  float t, e;
+  two_sum(a.hi, hi, t, e);
+  a.hi = t;
+  a.lo = a.lo + lo + e;
+}
+
 struct Acc {
-  float l1, s2, a, b;
+  DF l1, s2, a, b, p;
 };
 
-// Eight bf16 elements of each stream: tree sums of depth 3 for L1, S2, A, B
-// (bf16 squares are exact in fp32); P terms (exact products) go through TwoSum.
-__device__ __forceinline__ void chunk_bf16(const uint4 &vx, const uint4 &vp, const uint4 &vq, Acc &acc, float &ph,
-                                           float &pl) {
+// Eight bf16 elements of each stream: depth-3 trees for |x|, x^2, x'^2, x''^2
+// (bf16 squares are exact in fp32, so only the additions round); the eight
+// exact products x'x'' go through TwoSum one by one.
+__device__ __forceinline__ void chunk_bf16(const uint4 &vx, const uint4 &vp, const uint4 &vq, Acc &acc) {
   const uint32_t wx[4] = {vx.x, vx.y, vx.z, vx.w};
   const uint32_t wp[4] = {vp.x, vp.y, vp.z, vp.w};
   const uint32_t wq[4] = {vq.x, vq.y, vq.z, vq.w};
@@ -54,39 +74,40 @@ __device__ __forceinline__ void chunk_bf16(const uint4 &vx, const uint4 &vp, con
     s[i] = fmaf(x0, x0, x1 * x1);
     a[i] = fmaf(p0, p0, p1 * p1);
     b[i] = fmaf(q0, q0, q1 * q1);
-    float t, e;
-    two_sum(ph, p0 * q0, t, e);
-    ph = t;
-    pl += e;
-    two_sum(ph, p1 * q1, t, e);
-    ph = t;
-    pl += e;
+    df_add(acc.p, p0 * q0);
+    df_add(acc.p, p1 * q1);
   }
-  acc.l1 += (l[0] + l[1]) + (l[2] + l[3]);
-  acc.s2 += (s[0] + s[1]) + (s[2] + s[3]);
-  acc.a += (a[0] + a[1]) + (a[2] + a[3]);
-  acc.b += (b[0] + b[1]) + (b[2] + b[3]);
+  df_add(acc.l1, (l[0] + l[1]) + (l[2] + l[3]));
+  df_add(acc.s2, (s[0] + s[1]) + (s[2] + s[3]));
+  df_add(acc.a, (a[0] + a[1]) + (a[2] + a[3]));
+  df_add(acc.b, (b[0] + b[1]) + (b[2] + b[3]));
 }
 
-// Four fp32 elements of each stream: tree depth 2; products split exactly
-// into p + pe with an FMA, both parts enter the double-float P.
-__device__ __forceinline__ void chunk_f32(const uint4 &vx, const uint4 &vp, const uint4 &vq, Acc &acc, float &ph,
-                                          float &pl) {
+// Four fp32 elements of each stream: depth-2 trees (plus the rounding of each
+// square); products split exactly into p + pe with an FMA, both enter P.
+__device__ __forceinline__ void chunk_f32(const uint4 &vx, const uint4 &vp, const uint4 &vq, Acc &acc) {
   const float x[4] = {__uint_as_float(vx.x), __uint_as_float(vx.y), __uint_as_float(vx.z), __uint_as_float(vx.w)};
   const float p[4] = {__uint_as_float(vp.x), __uint_as_float(vp.y), __uint_as_float(vp.z), __uint_as_float(vp.w)};
   const float q[4] = {__uint_as_float(vq.x), __uint_as_float(vq.y), __uint_as_float(vq.z), __uint_as_float(vq.w)};
-  acc.l1 += (fabsf(x[0]) + fabsf(x[1])) + (fabsf(x[2]) + fabsf(x[3]));
-  acc.s2 += fmaf(x[0], x[0], x[1] * x[1]) + fmaf(x[2], x[2], x[3] * x[3]);
-  acc.a += fmaf(p[0], p[0], p[1] * p[1]) + fmaf(p[2], p[2], p[3] * p[3]);
-  acc.b += fmaf(q[0], q[0], q[1] * q[1]) + fmaf(q[2], q[2], q[3] * q[3]);
+  df_add(acc.l1, (fabsf(x[0]) + fabsf(x[1])) + (fabsf(x[2]) + fabsf(x[3])));
+  df_add(acc.s2, fmaf(x[0], x[0], x[1] * x[1]) + fmaf(x[2], x[2], x[3] * x[3]));
+  df_add(acc.a, fmaf(p[0], p[0], p[1] * p[1]) + fmaf(p[2], p[2], p[3] * p[3]));
+  df_add(acc.b, fmaf(q[0], q[0], q[1] * q[1]) + fmaf(q[2], q[2], q[3] * q[3]));
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
     const float pr = p[i] * q[i];
     const float pe = fmaf(p[i], q[i], -pr);
-    float t, e;
-    two_sum(ph, pr, t, e);
-    ph = t;
-    pl += e + pe;
+    df_add(acc.p, pr);
+    acc.p.lo += pe;
+  }
+}
+
+__device__ __forceinline__ void df_warp_sum(DF &v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float oh = __shfl_xor_sync(0xffffffffu, v.hi, o);
+    const float ol = __shfl_xor_sync(0xffffffffu, v.lo, o);
+    df_merge(v, oh, ol);
   }
 }
 
@@ -100,10 +121,7 @@ __global__ void __launch_bounds__(kScoreWarps * 32)
     const uint4 *rx = x + row * nchunks;
     const uint4 *rp = xp + row * nchunks;
     const uint4 *rq = xq + row * nchunks;
-    Acc acc[kScoreBatch];
-#pragma unroll
-    for (int u = 0; u < kScoreBatch; ++u) acc[u] = Acc{0.f, 0.f, 0.f, 0.f};
-    float ph = 0.f, pl = 0.f;
+    Acc acc{{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
     for (int c0 = lane; c0 < nchunks; c0 += 32 * kScoreBatch) {
       uint4 vx[kScoreBatch], vp[kScoreBatch], vq[kScoreBatch];
 #pragma unroll
@@ -120,35 +138,34 @@ __global__ void __launch_bounds__(kScoreWarps * 32)
 #pragma unroll
       for (int u = 0; u < kScoreBatch; ++u) {
         if (kBf16)
-          chunk_bf16(vx[u], vp[u], vq[u], acc[u], ph, pl);
+          chunk_bf16(vx[u], vp[u], vq[u], acc);
         else
-          chunk_f32(vx[u], vp[u], vq[u], acc[u], ph, pl);
+          chunk_f32(vx[u], vp[u], vq[u], acc);
       }
     }
-    static_assert(kScoreBatch == 4, "the accumulator tree below assumes 4 accumulators");
-    float l1 = (acc[0].l1 + acc[1].l1) + (acc[2].l1 + acc[3].l1);
-    float s2 = (acc[0].s2 + acc[1].s2) + (acc[2].s2 + acc[3].s2);
-    float sa = (acc[0].a + acc[1].a) + (acc[2].a + acc[3].a);
-    float sb = (acc[0].b + acc[1].b) + (acc[2].b + acc[3].b);
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      l1 += __shfl_xor_sync(0xffffffffu, l1, o);
-      s2 += __shfl_xor_sync(0xffffffffu, s2, o);
-      sa += __shfl_xor_sync(0xffffffffu, sa, o);
-      sb += __shfl_xor_sync(0xffffffffu, sb, o);
-      const float oh = __shfl_xor_sync(0xffffffffu, ph, o);
-      const float ol = __shfl_xor_sync(0xffffffffu, pl, o);
-      float t, e;
-      two_sum(ph, oh, t, e);
-      ph = t;
-      pl = pl + ol + e;
-    }
+    df_warp_sum(acc.l1);
+    df_warp_sum(acc.s2);
+    df_warp_sum(acc.a);
+    df_warp_sum(acc.b);
+    df_warp_sum(acc.p);
     if (lane == 0) {
+      const float l1 = acc.l1.hi + acc.l1.lo, s2 = acc.s2.hi + acc.s2.lo;
+      const float sa = acc.a.hi + acc.a.lo, sb = acc.b.hi + acc.b.lo;
+      const float ph = acc.p.hi, pl = acc.p.lo;
+      // Selection keys, fp32 only: R = L1^2 / S2 (H2 = log R, Eq. 3-4) and
+      // s = P / (sqrt(A) sqrt(B)) (Eq. 6).  NaN marks a row whose sums left
+      // the fp32 error model (non-finite, overflowed or underflowed): the
+      // selection recomputes it exactly.
+      const bool bad_r = !(isfinite(l1) && isfinite(s2)) || (l1 != 0.f && (s2 < kTiny || s2 > kHuge));
+      const bool bad_s = !(isfinite(sa) && isfinite(sb) && isfinite(ph) && isfinite(pl)) || sa < kTiny ||
+                         sb < kTiny || sa > kHuge || sb > kHuge;
+      const float r = l1 == 0.f ? 1.f : __fdiv_rn(__fmul_rn(l1, l1), s2);
+      const float sv = __fdiv_rn(__fadd_rn(ph, pl), __fmul_rn(__fsqrt_rn(sa), __fsqrt_rn(sb)));
+      const float nan = __int_as_float(0x7fc00000);
       stats[2 * row] = make_float4(l1, s2, sa, sb);
-      stats[2 * row + 1] = make_float4(ph, pl, 0.f, 0.f);
-      if (h2) h2[row] = l1 > 0.f ? (float)log((double)l1 * (double)l1 / (double)s2) : 0.f;
-      if (s_out)
-        s_out[row] = (sa > 0.f && sb > 0.f) ? (float)(((double)ph + (double)pl) / sqrt((double)sa * (double)sb)) : 0.f;
+      stats[2 * row + 1] = make_float4(ph, pl, bad_r ? nan : r, bad_s ? nan : sv);
+      if (h2) h2[row] = l1 > 0.f ? logf(r) : 0.f;
+      if (s_out) s_out[row] = (sa > 0.f && sb > 0.f) ? sv : 0.f;
     }
   }
 }

@@ -2,10 +2,10 @@
 // and stride pick), one CTA per image, with exact decisions.
 //
 // Keys.  H2 = log R with R = L1^2 / S2 (Eq. 3-4: sum_j p_j^2 = S2 / L1^2),
-// so ranking by H2 is ranking by R; s = P / sqrt(A B) (Eq. 6).  The CTA sorts
-// fp32 keys R32 (descending) and s32 (ascending) built from the score pass's
-// sums, packed with the token index into 64-bit words so that equal keys
-// order by the lower index.
+// so ranking by H2 is ranking by R; s = P / sqrt(A B) (Eq. 6).  The score
+// pass leaves fp32 keys R32 and s32 in each row's statistics record; the CTA
+// sorts them (R descending, s ascending) packed with the token index into
+// 64-bit words so that equal keys order by the lower index.
 //
 // Certification.  The score pass's sums carry proven error bounds (Bounds),
 // so a cut between sorted neighbours is certain when their key intervals do
@@ -44,63 +44,105 @@ __device__ __forceinline__ uint32_t ord32(float f) {
 __device__ __forceinline__ float unord32(uint32_t o) {
   return __uint_as_float((o & 0x80000000u) ? (o & 0x7fffffffu) : ~o);
 }
-__device__ __forceinline__ int row_at(const unsigned long long *keys, int q) { return (int)(keys[q] & 0xffffffffu); }
-__device__ __forceinline__ float r_at(const unsigned long long *keys, int q) {
-  return unord32(~(uint32_t)(keys[q] >> 32));
+// fp32 keys from the statistics record; NaN = outside the fp32 error model.
+__device__ __forceinline__ float key_r(const float *st) { return st[6]; }
+__device__ __forceinline__ float key_s(const float *st) { return st[7]; }
+
+// ---- a Big truncated to a 64-bit mantissa: value in [m 2^e, (m + 1) 2^e) ----
+// Integer-only (the GPU's fp64 rate is far too low for this path).
+struct Fx {
+  unsigned long long m;  // top bit set, or 0 for the value 0
+  int e;
+};
+__device__ __forceinline__ Fx big_fx(const Big &b) {
+  if (b.n == 0) return Fx{0ull, 0};
+  const int n = b.n;
+  const unsigned long long top = ((unsigned long long)b.l[n - 1] << 32) | (n >= 2 ? b.l[n - 2] : 0u);
+  const uint32_t third = n >= 3 ? b.l[n - 3] : 0u;
+  const int z = __clzll(top);  // < 32: the top limb is non-zero
+  const unsigned long long m = z ? (top << z) | ((unsigned long long)third >> (32 - z)) : top;
+  return Fx{m, 32 * (b.e + n - 2) - z};
 }
-__device__ __forceinline__ float s_at(const unsigned long long *keys, int q) {
-  return unord32((uint32_t)(keys[q] >> 32));
+__device__ __forceinline__ Fx fx_one() { return Fx{1ull << 63, -63}; }
+// Product truncated to 64 bits (relative error below 2^-63).
+__device__ __forceinline__ Fx fx_mul(const Fx &a, const Fx &b) {
+  if (!a.m || !b.m) return Fx{0ull, 0};
+  const unsigned long long hi = __umul64hi(a.m, b.m), lo = a.m * b.m;
+  if (hi >> 63) return Fx{hi, a.e + b.e + 64};
+  return Fx{(hi << 1) | (lo >> 63), a.e + b.e + 63};
+}
+// sign(x - y) when |x - y| exceeds 2^-57 of max(x, y), else 0 (too close to
+// call: each side is a product of at most four truncated factors, within
+// 2^-60 of its value).
+__device__ __forceinline__ int fx_cmp(const Fx &x, const Fx &y) {
+  if (!x.m || !y.m) return (x.m != 0) - (y.m != 0);
+  const bool xbig = x.e >= y.e;
+  const Fx &b = xbig ? x : y, &s = xbig ? y : x;
+  const int sh = b.e - s.e;
+  const unsigned long long sm = sh >= 64 ? 0ull : s.m >> sh;
+  if (b.m > sm && b.m - sm > 128ull) return xbig ? 1 : -1;
+  if (sm > b.m && sm - b.m > 128ull) return xbig ? -1 : 1;
+  return 0;
+}
+// Mantissa of a non-zero Fx as a float in [1, 2], rounded to nearest: the Fx
+// value is fx_mant(x) * 2^(x.e + 63).
+__device__ __forceinline__ float fx_mant(const Fx &x) { return __ull2float_rn(x.m) * 0x1p-63f; }
+__device__ __forceinline__ float fx_log(const Fx &x) {  // natural log of a non-zero Fx
+  return logf(fx_mant(x)) + (float)(x.e + 63) * 0.69314718f;
 }
 
-__device__ __forceinline__ bool force_l(const float *st) {
-  const float l1 = st[0], s2 = st[1];
-  if (!(isfinite(l1) && isfinite(s2))) return true;
-  return l1 != 0.f && (s2 < kTiny || s2 > kHuge);
+// Keys and reported scores of a row settled exactly, in fp32 from the
+// truncated exact sums (relative error a few 2^-24, inside the bounds).
+__device__ __forceinline__ float exact_r_key(const ExactRec &r) {
+  if (r.flags_l & kRecNonFiniteX) return 0.f;
+  if (r.l1.n == 0) return 1.f;
+  const Fx l1 = big_fx(r.l1), s2 = big_fx(r.s2);
+  // R = (l1.m / 2^63)^2 / (s2.m / 2^63) * 2^(2 (l1.e + 63) - (s2.e + 63))
+  const float ml = fx_mant(l1), ms = fx_mant(s2);
+  return ldexpf(ml * ml / ms, 2 * (l1.e + 63) - (s2.e + 63));
 }
-__device__ __forceinline__ bool force_s(const float *st) {
-  const float a = st[2], b = st[3], ph = st[4], pl = st[5];
-  if (!(isfinite(a) && isfinite(b) && isfinite(ph) && isfinite(pl))) return true;
-  return a < kTiny || b < kTiny || a > kHuge || b > kHuge;
+__device__ __forceinline__ float exact_h2(const ExactRec &r) {
+  if (r.flags_l & kRecNonFiniteX) return -INFINITY;
+  if (r.l1.n == 0) return 0.f;
+  const Fx l1 = big_fx(r.l1), s2 = big_fx(r.s2);
+  return 2.f * fx_log(l1) - fx_log(s2);
 }
-__device__ __forceinline__ float approx_r(const float *st) {
-  const float l1 = st[0], s2 = st[1];
-  return l1 == 0.f ? 1.f : (float)((double)l1 * (double)l1 / (double)s2);
-}
-__device__ __forceinline__ float approx_s(const float *st) {
-  return (float)(((double)st[4] + (double)st[5]) / sqrt((double)st[2] * (double)st[3]));
-}
-
-__device__ double big_to_double(const Big &b) {
-  if (b.n == 0) return 0.0;
-  const int top = b.n - 1, bot = b.n >= 3 ? b.n - 3 : 0;
-  double v = 0.0;
-  for (int i = top; i >= bot; --i) v = v * 4294967296.0 + (double)b.l[i];
-  v = ldexp(v, 32 * (b.e + bot));
-  return b.neg ? -v : v;
-}
-__device__ __forceinline__ double exact_r_value(const ExactRec &r) {
-  if (r.flags_l & kRecNonFiniteX) return 0.0;
-  if (r.l1.n == 0) return 1.0;
-  const double l1 = big_to_double(r.l1);
-  return l1 * l1 / big_to_double(r.s2);
-}
-__device__ __forceinline__ double exact_s_value(const ExactRec &r) {
-  if (r.flags_s & kRecNonFiniteS) return 2.0;
-  if (r.a.n == 0 || r.b.n == 0) return 0.0;
-  return big_to_double(r.p) / sqrt(big_to_double(r.a) * big_to_double(r.b));
+__device__ __forceinline__ float exact_s_key(const ExactRec &r) {
+  if (r.flags_s & kRecNonFiniteS) return 2.f;
+  if (r.a.n == 0 || r.b.n == 0 || r.p.n == 0) return 0.f;
+  const Fx p = big_fx(r.p), a = big_fx(r.a), b = big_fx(r.b);
+  // s = P / sqrt(A B); scale A and B to even exponents so the roots are exact powers of two
+  const float mp = fx_mant(p);
+  int ea = a.e + 63, eb = b.e + 63;
+  float ma = fx_mant(a), mb = fx_mant(b);
+  if (ea & 1) { ma *= 2.f; --ea; }
+  if (eb & 1) { mb *= 2.f; --eb; }
+  const float v = ldexpf(mp / (sqrtf(ma) * sqrtf(mb)), (p.e + 63) - ea / 2 - eb / 2);
+  return r.p.neg ? -v : v;
 }
 
-// Cut between importance-sorted positions q-1 and q (descending R32) is
-// certain when R(q-1) > R(q) for every value the bounds allow.
-__device__ __forceinline__ bool cert_r(const unsigned long long *keys, int q, double rho) {
-  const double ra = r_at(keys, q - 1), rb = r_at(keys, q);
-  return ra / (1.0 + rho) > rb / (1.0 - rho);
+// Sorted order: ord[q] is the row at position q, key[row] its 32-bit sort
+// key: ~ord32(R32) for the importance order (ascending key = descending R),
+// ord32(s32) for the consistency order.
+__device__ __forceinline__ float r_of(const uint32_t *key, const uint16_t *ord, int q) {
+  return unord32(~key[ord[q]]);
+}
+__device__ __forceinline__ float s_of(const uint32_t *key, const uint16_t *ord, int q) {
+  return unord32(key[ord[q]]);
+}
+
+// Cut between importance-sorted positions q-1 and q is certain when the
+// smallest R the bounds allow at q-1 exceeds the largest R they allow at q;
+// evaluated in fp32 with rounding toward the safe side.
+__device__ __forceinline__ bool cert_r(const uint32_t *key, const uint16_t *ord, int q, const Bounds &bd) {
+  return __fmul_rd(r_of(key, ord, q - 1), bd.r_lo) > __fmul_ru(r_of(key, ord, q), bd.r_hi);
 }
 // Cut between consistency-sorted positions q-1 and q (ascending s32).
-__device__ __forceinline__ bool cert_s(const unsigned long long *keys, int q, const Bounds &bd) {
-  const double sa = s_at(keys, q - 1), sb = s_at(keys, q);
-  const double ea = bd.es_abs + bd.es_rel * fabs(sa), eb = bd.es_abs + bd.es_rel * fabs(sb);
-  return sa + ea < sb - eb;
+__device__ __forceinline__ bool cert_s(const uint32_t *key, const uint16_t *ord, int q, const Bounds &bd) {
+  const float sa = s_of(key, ord, q - 1), sb = s_of(key, ord, q);
+  const float hi_a = __fadd_ru(sa, __fmaf_ru(bd.s_rel, fabsf(sa), bd.s_abs));
+  const float lo_b = __fsub_rd(sb, __fmaf_ru(bd.s_rel, fabsf(sb), bd.s_abs));
+  return lo_b > hi_a;
 }
 
 // ---------------------------------------------------------------- exact sums
@@ -207,7 +249,7 @@ __device__ __forceinline__ void warp_sum_digits(long long *dg) {
 // S2 = sum x^2; mode 1: A = sum x'^2, B = sum x''^2, P = sum x'x''.
 // Digit bases (multiples of 32): |x| has exponent >= -133 (bf16) or -149
 // (fp32), products >= -266 or -298; the top digit stays below kDig.
-__device__ void exact_row(const SelectArgs &a, long long row, int mode, ExactRec *rec, int lane) {
+__device__ __noinline__ void exact_row(const SelectArgs &a, long long row, int mode, ExactRec *rec, int lane) {
   const bool bf16 = a.dtype == TR_BF16;
   const int base1 = -160;
   const int base2 = bf16 ? -288 : -320;
@@ -265,26 +307,243 @@ __device__ void exact_row(const SelectArgs &a, long long row, int mode, ExactRec
   }
 }
 
-// Every warp takes 32-row groups round-robin and recomputes the rows whose
-// flags request it; clears the request and records what is now exact.
-__device__ void refine_pending(const SelectArgs &a, long long off, int n, uint8_t *fl, ExactRec *rec) {
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
-  for (int g = warp; g * 32 < n; g += nwarps) {
-    const int i = g * 32 + lane;
-    const uint8_t f = i < n ? fl[i] : 0;
-    unsigned mask = __ballot_sync(0xffffffffu, (f & (F_NEEDL | F_NEEDS)) != 0);
-    while (mask) {
-      const int r = __ffs(mask) - 1;
-      mask &= mask - 1;
-      const int row = g * 32 + r;
-      const uint8_t fr = (uint8_t)__shfl_sync(0xffffffffu, (int)f, r);
-      if (fr & F_NEEDL) exact_row(a, off + row, 0, rec + row, lane);
-      if (fr & F_NEEDS) exact_row(a, off + row, 1, rec + row, lane);
-      if (lane == 0) {
-        fl[row] = (uint8_t)((fr & ~(F_NEEDL | F_NEEDS)) | ((fr & F_NEEDL) ? F_XL : 0) | ((fr & F_NEEDS) ? F_XS : 0));
-        if (a.status) atomicAdd(&a.status[2], 1);
+// ---- fast exact sums: one 128-bit integer per sum, in registers ----------
+// Every term is m * 2^e with an integer m of at most 2 * kMant bits.  With
+// the row's smallest exponent as the base, term m * 2^(e - base) and the sum
+// of all d terms fit 127 bits whenever the row's exponent span is moderate
+// (always for ordinary activations); the warp checks that first and falls
+// back to the digit accumulator above otherwise.
+struct Dec {
+  uint32_t m;
+  int e;
+  bool neg, nf;
+};
+__device__ __forceinline__ Dec dec16(uint32_t h) {
+  const uint32_t ex = (h >> 7) & 0xffu, mant = h & 0x7fu;
+  return Dec{ex ? (mant | 0x80u) : mant, (ex ? (int)ex : 1) - 134, (h >> 15) != 0, ex == 0xffu};
+}
+__device__ __forceinline__ Dec dec32(uint32_t b) {
+  const uint32_t ex = (b >> 23) & 0xffu, mant = b & 0x7fffffu;
+  return Dec{ex ? (mant | 0x800000u) : mant, (ex ? (int)ex : 1) - 150, (b >> 31) != 0, ex == 0xffu};
+}
+
+template <bool kBf16>
+__device__ __forceinline__ void unpack(const uint4 &v, Dec *out) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  if (kBf16) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      out[2 * i] = dec16(w[i] & 0xffffu);
+      out[2 * i + 1] = dec16(w[i] >> 16);
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) out[i] = dec32(w[i]);
+  }
+}
+
+__device__ __forceinline__ void add128(__int128 &acc, unsigned long long m, int sh, bool neg) {
+  const __int128 v = (__int128)((unsigned __int128)m << sh);
+  acc = neg ? acc - v : acc + v;
+}
+__device__ __forceinline__ __int128 warp_sum128(__int128 v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const unsigned long long lo = __shfl_xor_sync(0xffffffffu, (unsigned long long)v, o);
+    const unsigned long long hi = __shfl_xor_sync(0xffffffffu, (unsigned long long)((unsigned __int128)v >> 64), o);
+    v += (__int128)(((unsigned __int128)hi << 64) | lo);
+  }
+  return v;
+}
+
+// value = v * 2^base as a trimmed Big (|v| < 2^127, so at most 5 limbs).
+__device__ void int128_to_big(__int128 v, int base, Big &out) {
+  const bool neg = v < 0;
+  const unsigned __int128 mag = neg ? (unsigned __int128)(-v) : (unsigned __int128)v;
+  out.neg = neg ? 1 : 0;
+  if (mag == 0) {
+    out.n = 0;
+    out.e = 0;
+    out.neg = 0;
+    return;
+  }
+  const int q = base >> 5, r = base & 31;  // base = 32 q + r, 0 <= r < 32
+  const unsigned __int128 lo = mag << r;
+  uint32_t limb[5] = {(uint32_t)lo, (uint32_t)(lo >> 32), (uint32_t)(lo >> 64), (uint32_t)(lo >> 96),
+                      r ? (uint32_t)(mag >> (128 - r)) : 0u};
+  int hi = 4;
+  while (limb[hi] == 0) --hi;
+  int l = 0;
+  while (limb[l] == 0) ++l;
+  out.n = (uint8_t)(hi - l + 1);
+  for (int i = 0; i < out.n; ++i) out.l[i] = limb[l + i];
+  out.e = (int16_t)(q + l);
+}
+
+// Window for one exact sum: every term and the sum are below 2^top, where
+// 2^top exceeds 1.5 x (the fp32 sum of |terms|, itself within 1e-6 of the
+// truth); terms are integers times 2^bottom with bottom = top - 126, so the
+// signed 128-bit accumulator cannot overflow.  A term with a lower bit below
+// 2^bottom does not fit (the row spans > ~95 binades): the caller falls back.
+__device__ __forceinline__ int window_bottom(float bound) {
+  int ex;
+  frexpf(bound * 1.5f, &ex);  // bound * 1.5 < 2^ex
+  return ex - 126;
+}
+
+constexpr int kWarps = kSelectThreads / 32;
+
+// 128-bit partial sums of the warps, reduced by thread 0.
+struct Part128 {
+  unsigned long long lo[kWarps * 3], hi[kWarps * 3];
+};
+__device__ __forceinline__ void part_put(Part128 &p, int slot, __int128 v) {
+  p.lo[slot] = (unsigned long long)v;
+  p.hi[slot] = (unsigned long long)((unsigned __int128)v >> 64);
+}
+__device__ __forceinline__ __int128 part_sum(const Part128 &p, int which) {
+  __int128 v = 0;
+  for (int w = 0; w < kWarps; ++w)
+    v += (__int128)(((unsigned __int128)p.hi[w * 3 + which] << 64) | p.lo[w * 3 + which]);
+  return v;
+}
+
+// Exact sums of one row computed by the whole CTA (one 16-byte chunk of each
+// stream per thread and pass), in three 128-bit windows; false (uniformly)
+// when a term does not fit its window.
+template <bool kBf16>
+__device__ bool exact_row_block(const SelectArgs &a, long long row, int mode, const float *st, ExactRec *rec,
+                                Part128 &part) {
+  constexpr int kPer = kBf16 ? 8 : 4;  // elements per 16-byte chunk
+  const int nchunks = a.d / kPer;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  bool fits = true;
+  Dec e0[kPer], e1[kPer];
+  __int128 s0 = 0, s1 = 0, s2 = 0;
+  int b0, b1, b2 = 0;
+  if (mode == 0) {
+    b0 = window_bottom(st[0]);
+    b1 = window_bottom(st[1]);
+    const uint4 *px = static_cast<const uint4 *>(a.x) + row * nchunks;
+#pragma unroll 4
+    for (int c = threadIdx.x; c < nchunks; c += blockDim.x) {
+      unpack<kBf16>(__ldg(px + c), e0);
+#pragma unroll
+      for (int i = 0; i < kPer; ++i) {
+        const Dec &t = e0[i];
+        if (!t.m) continue;
+        if (t.nf || t.e < b0 || 2 * t.e < b1) {
+          fits = false;
+          continue;
+        }
+        add128(s0, t.m, t.e - b0, false);
+        add128(s1, (unsigned long long)t.m * t.m, 2 * t.e - b1, false);
       }
     }
+  } else {
+    b0 = window_bottom(st[2]);
+    b1 = window_bottom(st[3]);
+    b2 = window_bottom(__fsqrt_ru(st[2]) * __fsqrt_ru(st[3]));
+    const uint4 *pp = static_cast<const uint4 *>(a.x_pre ? a.x_pre : a.x) + row * nchunks;
+    const uint4 *pq = static_cast<const uint4 *>(a.x_post) + row * nchunks;
+#pragma unroll 4
+    for (int c = threadIdx.x; c < nchunks; c += blockDim.x) {
+      unpack<kBf16>(__ldg(pp + c), e0);
+      unpack<kBf16>(__ldg(pq + c), e1);
+#pragma unroll
+      for (int i = 0; i < kPer; ++i) {
+        const Dec &p = e0[i], &q = e1[i];
+        if (p.nf || q.nf) {
+          fits = false;
+          continue;
+        }
+        if (p.m) {
+          if (2 * p.e < b0) fits = false; else add128(s0, (unsigned long long)p.m * p.m, 2 * p.e - b0, false);
+        }
+        if (q.m) {
+          if (2 * q.e < b1) fits = false; else add128(s1, (unsigned long long)q.m * q.m, 2 * q.e - b1, false);
+        }
+        if (p.m && q.m) {
+          if (p.e + q.e < b2) fits = false;
+          else add128(s2, (unsigned long long)p.m * q.m, p.e + q.e - b2, p.neg != q.neg);
+        }
+      }
+    }
+  }
+  if (!__syncthreads_and(fits)) return false;
+  s0 = warp_sum128(s0);
+  s1 = warp_sum128(s1);
+  s2 = warp_sum128(s2);
+  if (lane == 0) {
+    part_put(part, warp * 3 + 0, s0);
+    part_put(part, warp * 3 + 1, s1);
+    part_put(part, warp * 3 + 2, s2);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    if (mode == 0) {
+      int128_to_big(part_sum(part, 0), b0, rec->l1);
+      int128_to_big(part_sum(part, 1), b1, rec->s2);
+      rec->flags_l = 0u;
+    } else {
+      int128_to_big(part_sum(part, 0), b0, rec->a);
+      int128_to_big(part_sum(part, 1), b1, rec->b);
+      int128_to_big(part_sum(part, 2), b2, rec->p);
+      rec->flags_s = 0u;
+    }
+  }
+  __syncthreads();
+  return true;
+}
+
+// Exact sums of one row by the whole CTA: the 128-bit windows when the row's
+// fp32 sums are trustworthy and its terms fit, else warp 0 runs the digit
+// accumulator (non-finite or extreme rows).
+__device__ __noinline__ void exact_row_any(const SelectArgs &a, long long row, int mode, const float *st,
+                                           ExactRec *rec, Part128 &part) {
+  const bool trusted = mode == 0 ? !isnan(st[6]) : !isnan(st[7]);
+  bool ok = false;
+  if (trusted)
+    ok = a.dtype == TR_BF16 ? exact_row_block<true>(a, row, mode, st, rec, part)
+                            : exact_row_block<false>(a, row, mode, st, rec, part);
+  if (!ok) {
+    if ((threadIdx.x >> 5) == 0) exact_row(a, row, mode, rec, threadIdx.x & 31);
+    __syncthreads();
+  }
+}
+
+// Recomputes, one row at a time with the whole CTA, the rows whose flags
+// request it; clears the request and records what is now exact.  A single
+// block-wide vote skips the scan when nothing is pending.
+__device__ void refine_pending(const SelectArgs &a, long long off, int n, uint8_t *fl, ExactRec *rec) {
+  __shared__ unsigned wmask[kWarps];
+  __shared__ Part128 part;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  bool any = false;
+  for (int i = threadIdx.x; i < n; i += blockDim.x) any |= (fl[i] & (F_NEEDL | F_NEEDS)) != 0;
+  if (!__syncthreads_or(any)) return;
+  for (int base = 0; base < n; base += blockDim.x) {
+    const int i = base + threadIdx.x;
+    const unsigned m = __ballot_sync(0xffffffffu, i < n && (fl[i] & (F_NEEDL | F_NEEDS)) != 0);
+    if (lane == 0) wmask[warp] = m;
+    __syncthreads();
+    for (int w = 0; w < kWarps; ++w) {
+      unsigned mm = wmask[w];
+      while (mm) {
+        const int r = __ffs(mm) - 1;
+        mm &= mm - 1;
+        const int row = base + 32 * w + r;
+        const uint8_t fr = fl[row];
+        const float *st = a.stats + (off + row) * TR_STATS_WORDS;
+        if (fr & F_NEEDL) exact_row_any(a, off + row, 0, st, rec + row, part);
+        if (fr & F_NEEDS) exact_row_any(a, off + row, 1, st, rec + row, part);
+        if (threadIdx.x == 0) {
+          fl[row] = (uint8_t)((fr & ~(F_NEEDL | F_NEEDS)) | ((fr & F_NEEDL) ? F_XL : 0) | ((fr & F_NEEDS) ? F_XS : 0));
+          if (a.status) atomicAdd(&a.status[2], 1);
+        }
+      }
+    }
+    __syncthreads();
   }
 }
 
@@ -340,8 +599,9 @@ __device__ int wide_cmp(const Wide &x, const Wide &y) {
   return 0;
 }
 
-// sign(R_a - R_b), R = L1^2 / S2 (R = 1 for an all-zero row, non-finite rows lowest).
-__device__ int cmp_r(const ExactRec &ra, const ExactRec &rb) {
+// sign(R_a - R_b), R = L1^2 / S2 (R = 1 for an all-zero row, non-finite rows
+// lowest), by big-integer cross products.
+__device__ __noinline__ int cmp_r_big(const ExactRec &ra, const ExactRec &rb) {
   const bool na = ra.flags_l & kRecNonFiniteX, nb = rb.flags_l & kRecNonFiniteX;
   if (na || nb) return na == nb ? 0 : (na ? -1 : 1);
   Wide l1a, s2a, l1b, s2b, t, x, y;
@@ -367,8 +627,8 @@ __device__ int cmp_r(const ExactRec &ra, const ExactRec &rb) {
 }
 
 // sign(s_a - s_b) through sigma = sign(P) P^2 / (A B) (s = 0 when A or B is 0,
-// non-finite rows highest).
-__device__ int cmp_s(const ExactRec &ra, const ExactRec &rb) {
+// non-finite rows highest), by big-integer cross products.
+__device__ __noinline__ int cmp_s_big(const ExactRec &ra, const ExactRec &rb) {
   const bool na = ra.flags_s & kRecNonFiniteS, nb = rb.flags_s & kRecNonFiniteS;
   if (na || nb) return na == nb ? 0 : (na ? 1 : -1);
   const int sa = (ra.a.n == 0 || ra.b.n == 0 || ra.p.n == 0) ? 0 : (ra.p.neg ? -1 : 1);
@@ -392,29 +652,37 @@ __device__ int cmp_s(const ExactRec &ra, const ExactRec &rb) {
   return sa > 0 ? c : -c;
 }
 
-// ---------------------------------------------------------------- block helpers
-__device__ void bitonic_sort(unsigned long long *keys, int np) {
-  for (int k = 2; k <= np; k <<= 1) {
-    for (int j = k >> 1; j > 0; j >>= 1) {
-      for (int i = threadIdx.x; i < np; i += blockDim.x) {
-        const int ixj = i ^ j;
-        if (ixj > i) {
-          const unsigned long long u = keys[i], v = keys[ixj];
-          const bool up = (i & k) == 0;
-          if ((u > v) == up) {
-            keys[i] = v;
-            keys[ixj] = u;
-          }
-        }
-      }
-      __syncthreads();
-    }
-  }
+// The same comparisons screened first with 64-bit truncated mantissas
+// (integer arithmetic only); only gaps below 2^-57 relative -- in practice
+// exact ties -- go on to the big-integer cross products.
+__device__ int cmp_r(const ExactRec &ra, const ExactRec &rb) {
+  const bool na = ra.flags_l & kRecNonFiniteX, nb = rb.flags_l & kRecNonFiniteX;
+  if (na || nb) return na == nb ? 0 : (na ? -1 : 1);
+  const Fx l1a = ra.l1.n ? big_fx(ra.l1) : fx_one(), s2a = ra.l1.n ? big_fx(ra.s2) : fx_one();
+  const Fx l1b = rb.l1.n ? big_fx(rb.l1) : fx_one(), s2b = rb.l1.n ? big_fx(rb.s2) : fx_one();
+  const int c = fx_cmp(fx_mul(fx_mul(l1a, l1a), s2b), fx_mul(fx_mul(l1b, l1b), s2a));
+  return c ? c : cmp_r_big(ra, rb);
 }
+__device__ int cmp_s(const ExactRec &ra, const ExactRec &rb) {
+  const bool na = ra.flags_s & kRecNonFiniteS, nb = rb.flags_s & kRecNonFiniteS;
+  if (na || nb) return na == nb ? 0 : (na ? 1 : -1);
+  const int sa = (ra.a.n == 0 || ra.b.n == 0 || ra.p.n == 0) ? 0 : (ra.p.neg ? -1 : 1);
+  const int sb = (rb.a.n == 0 || rb.b.n == 0 || rb.p.n == 0) ? 0 : (rb.p.neg ? -1 : 1);
+  if (sa != sb) return sa > sb ? 1 : -1;
+  if (sa == 0) return 0;
+  const Fx pa = big_fx(ra.p), pb = big_fx(rb.p);
+  const Fx x = fx_mul(fx_mul(fx_mul(pa, pa), big_fx(rb.a)), big_fx(rb.b));
+  const Fx y = fx_mul(fx_mul(fx_mul(pb, pb), big_fx(ra.a)), big_fx(ra.b));
+  const int c = fx_cmp(x, y);
+  return c ? c * sa : cmp_s_big(ra, rb);
+}
+
+// ---------------------------------------------------------------- block helpers
 
 __device__ int block_exclusive_scan(int v, int *total) {
   __shared__ int wsum[32];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  __syncthreads();  // wsum may still be read by a previous call
   int x = v;
 #pragma unroll
   for (int o = 1; o < 32; o <<= 1) {
@@ -437,11 +705,79 @@ __device__ int block_exclusive_scan(int v, int *total) {
   return (warp ? wsum[warp - 1] : 0) + x - v;
 }
 
-__host__ __device__ inline int next_pow2(int n) {
-  int p = 1;
-  while (p < n) p <<= 1;
-  return p;
+// Stable ascending LSD radix sort (8-bit digits) of the m rows listed in a
+// by key[row]; b is scratch of the same size and hist holds kWarps x 256
+// counters.  Warp w owns the contiguous stretch w of the current order:
+// per-warp digit counts, a column scan (digit-major, then warp), then each
+// warp scatters its stretch in order, ranking equal digits within 32 lanes
+// with match-any, which keeps the sort stable.  A pass whose digit is the
+// same for every row is skipped.  Returns the buffer holding the order.
+__device__ uint16_t *radix_sort(const uint32_t *key, uint16_t *a, uint16_t *b, int m, uint32_t *hist) {
+  __shared__ int skip;
+  __shared__ uint32_t dsum[8];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int seg = (m + kWarps - 1) / kWarps;
+  const int s0 = min(m, warp * seg), s1 = min(m, s0 + seg);
+  uint32_t *h = hist + warp * 256;
+  const unsigned lt = (1u << lane) - 1u;
+  if (m < 2) return a;
+  for (int shift = 0; shift < 32; shift += 8) {
+    for (int d = lane; d < 256; d += 32) h[d] = 0u;
+    if (tid == 0) skip = 0;
+    __syncwarp();
+    for (int q = s0 + lane; q < s1; q += 32) atomicAdd(&h[(key[a[q]] >> shift) & 0xffu], 1u);
+    __syncthreads();
+    uint32_t total = 0;
+    if (tid < 256) {
+      for (int w = 0; w < kWarps; ++w) {
+        const uint32_t c = hist[w * 256 + tid];
+        hist[w * 256 + tid] = total;
+        total += c;
+      }
+      if (total == (uint32_t)m) skip = 1;
+    }
+    uint32_t incl = total;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    if (tid < 256 && lane == 31) dsum[warp] = incl;
+    __syncthreads();
+    if (tid < 256) {
+      uint32_t base = 0;
+      for (int w = 0; w < warp; ++w) base += dsum[w];
+      const uint32_t excl = base + incl - total;
+      for (int w = 0; w < kWarps; ++w) hist[w * 256 + tid] += excl;
+    }
+    __syncthreads();
+    if (!skip) {
+      for (int q0 = s0; q0 < s1; q0 += 32) {
+        const int q = q0 + lane;
+        const bool act = q < s1;
+        const unsigned am = __ballot_sync(0xffffffffu, act);
+        if (act) {
+          const uint16_t row = a[q];
+          const uint32_t d = (key[row] >> shift) & 0xffu;
+          const unsigned peers = __match_any_sync(am, d);
+          const int rank = __popc(peers & lt);
+          const uint32_t base = h[d];
+          b[base + rank] = row;
+          __syncwarp(am);
+          if (rank == 0) h[d] = base + __popc(peers);
+        }
+        __syncwarp();
+      }
+      uint16_t *t = a;
+      a = b;
+      b = t;
+    }
+    __syncthreads();
+  }
+  return a;
 }
+
+__host__ __device__ inline int row_capacity(int max_n) { return (max_n + 15) / 16 * 16; }
 
 // ---------------------------------------------------------------- the kernel
 __global__ void __launch_bounds__(kSelectThreads, 1) k_select(const SelectArgs a) {
@@ -464,9 +800,12 @@ __global__ void __launch_bounds__(kSelectThreads, 1) k_select(const SelectArgs a
     return;
   }
   if (n == 0) return;
-  const int np = next_pow2(n);
-  unsigned long long *keys = reinterpret_cast<unsigned long long *>(smem);
-  uint8_t *fl = reinterpret_cast<uint8_t *>(keys + next_pow2(a.max_n));
+  const int cap = row_capacity(a.max_n);
+  uint32_t *key = reinterpret_cast<uint32_t *>(smem);        // [cap] sort key per row
+  uint16_t *ia = reinterpret_cast<uint16_t *>(key + cap);    // [cap] order buffers
+  uint16_t *ib = ia + cap;                                   // [cap]
+  uint32_t *hist = reinterpret_cast<uint32_t *>(ib + cap);   // [kWarps x 256]
+  uint8_t *fl = reinterpret_cast<uint8_t *>(hist + kWarps * 256);  // [cap] row flags
   const float *st = a.stats + off * TR_STATS_WORDS;
   ExactRec *rec = a.exact + off;
   const bool need_r = k1 > 0 && k1 < n;  // the importance order decides something
@@ -477,8 +816,8 @@ __global__ void __launch_bounds__(kSelectThreads, 1) k_select(const SelectArgs a
   for (int i = tid; i < n; i += nthr) {
     const float *r = st + (long long)i * TR_STATS_WORDS;
     uint8_t f = 0;
-    if ((need_r || a.h2) && force_l(r)) f |= F_NEEDL;
-    if ((need_s || a.s) && force_s(r)) f |= F_NEEDS;
+    if ((need_r || a.h2) && isnan(key_r(r))) f |= F_NEEDL;
+    if ((need_s || a.s) && isnan(key_s(r))) f |= F_NEEDS;
     fl[i] = f;
   }
   __syncthreads();
@@ -487,45 +826,42 @@ __global__ void __launch_bounds__(kSelectThreads, 1) k_select(const SelectArgs a
 
   // 2. Stage I: top-K1 by R (equivalently H2), descending, lower index first.
   if (need_r) {
-    for (int i = tid; i < np; i += nthr) {
-      unsigned long long key = ~0ull;
-      if (i < n) {
-        const float r = (fl[i] & F_XL) ? (float)exact_r_value(rec[i]) : approx_r(st + (long long)i * TR_STATS_WORDS);
-        key = ((unsigned long long)(~ord32(r)) << 32) | (unsigned)i;
-      }
-      keys[i] = key;
+    for (int i = tid; i < n; i += nthr) {
+      const float r = (fl[i] & F_XL) ? exact_r_key(rec[i]) : key_r(st + (long long)i * TR_STATS_WORDS);
+      key[i] = ~ord32(r);
+      ia[i] = (uint16_t)i;
     }
     __syncthreads();
-    bitonic_sort(keys, np);
+    const uint16_t *ord = radix_sort(key, ia, ib, n, hist);
     if (tid == 0) {
       int lo = k1, hi = k1;
-      if (!cert_r(keys, k1, a.bounds.rho_r)) {
+      if (!cert_r(key, ord, k1, a.bounds)) {
         lo = k1 - 1;
-        while (lo > 0 && !cert_r(keys, lo, a.bounds.rho_r)) --lo;
+        while (lo > 0 && !cert_r(key, ord, lo, a.bounds)) --lo;
         hi = k1 + 1;
-        while (hi < n && !cert_r(keys, hi, a.bounds.rho_r)) ++hi;
+        while (hi < n && !cert_r(key, ord, hi, a.bounds)) ++hi;
       }
       sh_lo = lo;
       sh_hi = hi;
     }
     __syncthreads();
     const int lo = sh_lo, hi = sh_hi;
-    for (int q = tid; q < lo; q += nthr) fl[row_at(keys, q)] |= F_IMP;
+    for (int q = tid; q < lo; q += nthr) fl[ord[q]] |= F_IMP;
     if (hi > lo) {
       for (int q = lo + tid; q < hi; q += nthr) {
-        const int r = row_at(keys, q);
+        const int r = ord[q];
         if (!(fl[r] & F_XL)) fl[r] |= F_NEEDL;
       }
       __syncthreads();
       refine_pending(a, off, n, fl, rec);
       __syncthreads();
       for (int q = lo + tid; q < hi; q += nthr) {
-        const int r = row_at(keys, q);
+        const int r = ord[q];
         const bool ovf = rec[r].flags_l & kRecOverflowL;
         int rank = 0;
         for (int q2 = lo; q2 < hi; ++q2) {
           if (q2 == q) continue;
-          const int r2 = row_at(keys, q2);
+          const int r2 = ord[q2];
           int c;
           if (ovf || (rec[r2].flags_l & kRecOverflowL))
             c = q2 < q ? 1 : -1;  // no exact value: keep the float order
@@ -544,32 +880,36 @@ __global__ void __launch_bounds__(kSelectThreads, 1) k_select(const SelectArgs a
 
   // 3. Stage II: sort X_rem by s ascending, pick positions 0, t, 2t, ...
   if (need_s) {
-    const int m = n - k1;
-    for (int i = tid; i < np; i += nthr) {
-      unsigned long long key = ~0ull;
-      if (i < n && !(fl[i] & F_IMP)) {
-        const float sv = (fl[i] & F_XS) ? (float)exact_s_value(rec[i]) : approx_s(st + (long long)i * TR_STATS_WORDS);
-        key = ((unsigned long long)ord32(sv) << 32) | (unsigned)i;
-      }
-      keys[i] = key;
+    // X_rem in ascending index order (the stable sort's tie order)
+    const int per = (n + nthr - 1) / nthr;
+    const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
+    int cnt = 0;
+    for (int i = i0; i < i1; ++i) cnt += !(fl[i] & F_IMP);
+    int m = 0;
+    int pos = block_exclusive_scan(cnt, &m);
+    for (int i = i0; i < i1; ++i) {
+      if (fl[i] & F_IMP) continue;
+      ia[pos++] = (uint16_t)i;
+      const float sv = (fl[i] & F_XS) ? exact_s_key(rec[i]) : key_s(st + (long long)i * TR_STATS_WORDS);
+      key[i] = ord32(sv);
     }
     __syncthreads();
-    bitonic_sort(keys, np);
+    const uint16_t *ord = radix_sort(key, ia, ib, m, hist);
     const int t = max(1, m / k2);
     for (int j = tid; j < k2; j += nthr) {
       const int p = j * t;
-      const bool c0 = p == 0 || cert_s(keys, p, a.bounds);
-      const bool c1 = p + 1 >= m || cert_s(keys, p + 1, a.bounds);
+      const bool c0 = p == 0 || cert_s(key, ord, p, a.bounds);
+      const bool c1 = p + 1 >= m || cert_s(key, ord, p + 1, a.bounds);
       if (c0 && c1) {
-        fl[row_at(keys, p)] |= F_DIV;
+        fl[ord[p]] |= F_DIV;
       } else {
         int lo = p;
-        while (lo > 0 && !cert_s(keys, lo, a.bounds)) --lo;
+        while (lo > 0 && !cert_s(key, ord, lo, a.bounds)) --lo;
         int hi = p + 1;
-        while (hi < m && !cert_s(keys, hi, a.bounds)) ++hi;
+        while (hi < m && !cert_s(key, ord, hi, a.bounds)) ++hi;
         // Threads whose runs coincide write the same bits: the races are benign.
         for (int q = lo; q < hi; ++q) {
-          const int r = row_at(keys, q);
+          const int r = ord[q];
           fl[r] |= (uint8_t)(F_RUN | ((fl[r] & F_XS) ? 0 : F_NEEDS));
         }
       }
@@ -578,17 +918,17 @@ __global__ void __launch_bounds__(kSelectThreads, 1) k_select(const SelectArgs a
     refine_pending(a, off, n, fl, rec);
     __syncthreads();
     for (int q = tid; q < m; q += nthr) {
-      const int r = row_at(keys, q);
+      const int r = ord[q];
       if (!(fl[r] & F_RUN)) continue;
       int lo = q;
-      while (lo > 0 && !cert_s(keys, lo, a.bounds)) --lo;
+      while (lo > 0 && !cert_s(key, ord, lo, a.bounds)) --lo;
       int hi = q + 1;
-      while (hi < m && !cert_s(keys, hi, a.bounds)) ++hi;
+      while (hi < m && !cert_s(key, ord, hi, a.bounds)) ++hi;
       const bool ovf = rec[r].flags_s & kRecOverflowS;
       int rank = 0;
       for (int q2 = lo; q2 < hi; ++q2) {
         if (q2 == q) continue;
-        const int r2 = row_at(keys, q2);
+        const int r2 = ord[q2];
         int c;
         if (ovf || (rec[r2].flags_s & kRecOverflowS))
           c = q2 < q ? -1 : 1;
@@ -596,8 +936,8 @@ __global__ void __launch_bounds__(kSelectThreads, 1) k_select(const SelectArgs a
           c = cmp_s(rec[r2], rec[r]);
         if (c < 0 || (c == 0 && r2 < r)) ++rank;
       }
-      const int pos = lo + rank;
-      if (pos % t == 0 && pos / t < k2) fl[r] |= F_DIV;
+      const int pp = lo + rank;
+      if (pp % t == 0 && pp / t < k2) fl[r] |= F_DIV;
     }
     __syncthreads();
   }
@@ -622,14 +962,14 @@ __global__ void __launch_bounds__(kSelectThreads, 1) k_select(const SelectArgs a
       nonfinite |= (r.flags_l & kRecNonFiniteX) != 0;
       overflow |= (r.flags_l & kRecOverflowL) != 0;
       if (a.h2 && !(r.flags_l & kRecOverflowL))
-        a.h2[off + i] = (r.flags_l & kRecNonFiniteX) ? -INFINITY : (float)log(exact_r_value(r));
+        a.h2[off + i] = exact_h2(r);
     }
     if (f & F_XS) {
       const ExactRec &r = rec[i];
       nonfinite |= (r.flags_s & kRecNonFiniteS) != 0;
       overflow |= (r.flags_s & kRecOverflowS) != 0;
       if (a.s && !(r.flags_s & kRecOverflowS))
-        a.s[off + i] = (r.flags_s & kRecNonFiniteS) ? INFINITY : (float)exact_s_value(r);
+        a.s[off + i] = (r.flags_s & kRecNonFiniteS) ? INFINITY : exact_s_key(r);
     }
     if (a.status) {
       if (nonfinite) atomicAdd(&a.status[0], 1);
@@ -644,7 +984,8 @@ int g_smem_set[64];  // per device: dynamic shared memory limit already raised
 }  // namespace
 
 size_t select_smem_bytes(int max_n) {
-  return (size_t)next_pow2(max_n > 0 ? max_n : 1) * sizeof(unsigned long long) + align_up((size_t)max_n, 16);
+  const size_t cap = (size_t)row_capacity(max_n > 0 ? max_n : 1);
+  return cap * (sizeof(uint32_t) + 2 * sizeof(uint16_t) + sizeof(uint8_t)) + kWarps * 256 * sizeof(uint32_t);
 }
 
 cudaError_t launch_select(const SelectArgs &a, cudaStream_t st) {
