@@ -44,17 +44,17 @@ struct ExactRec {
 static_assert(sizeof(ExactRec) % 16 == 0, "ExactRec records keep 16-byte alignment");
 
 // ---------------------------------------------------------------- error bounds
-// Rounding depth of the fp32 sums L1, S2, A, B in the score kernel: each term
-// goes through the depth-3 (bf16) or depth-2 (fp32) tree of its 16-byte chunk
-// (plus the rounding of the square itself for fp32 inputs, bf16 squares being
-// exact), the chunk partials are accumulated error-free (TwoSum into a
-// double-float whose low part's own rounding is bounded separately), and the
-// final hi + lo is rounded once to fp32.
+// Rounding depth of the sums L1, S2, A, B in the score kernel: each term goes
+// through the depth-3 (bf16) or depth-2 (fp32, plus the rounding of the square
+// itself) tree of its 16-byte chunk; the chunk partials are accumulated
+// error-free into a double-float whose low part's own rounding is bounded
+// separately, and the keys are computed from the unrounded double-float.
 __host__ __device__ inline int elem_bytes(int dtype) { return dtype == TR_BF16 ? 2 : 4; }
 
 __host__ __device__ inline int score_depth(int d, int dtype) {
   (void)d;
-  return dtype == TR_BF16 ? 3 + 1 : 2 + 1 + 1;
+  (void)dtype;
+  return 3;
 }
 
 // Certification bounds for the float selection keys (see the select kernel):
@@ -86,14 +86,16 @@ inline Bounds certification_bounds(int d, int dtype) {
   double ep = 2.0 * u * u * (lane_terms * lane_terms + 12.0 * d) + 0x1p-52;
   if (dtype != TR_BF16) ep *= 2.0;
   Bounds b;
-  // R32 = fl(fl(L1^2) / S2) with L1, S2 relative g: R32 / R within
-  // (1 + g)^2 / (1 - g) (1 + u)^2; 2^-30 covers subnormal squares (S2 >= 2^-100).
-  b.rho_r = (1.0 + g) * (1.0 + g) / (1.0 - g) * (1.0 + u) * (1.0 + u) - 1.0 + 0x1p-30;
-  // s32 = fl(fl(P_hi + P_lo) / fl(fl(sqrt A) fl(sqrt B))): the sums contribute
-  // g (half from A, half from B), the five fp32 roundings 5u, P's residue
-  // e_p sqrt(A B) an absolute term; 2^-34 covers underflowed squares and
-  // products when A, B >= 2^-100.
-  b.es_rel = 1.02 * (g / (1.0 - g) + 5.0 * u + 0x1p-34);
+  // R32 = fl(R^) with R^ = L1^2 / S2 evaluated in double-float (2^-40) from
+  // sums within relative g: R32 / R within (1 + g)^2 / (1 - g) (1 + 2^-40) (1 + u);
+  // 2^-30 covers subnormal squares (S2 >= 2^-100).
+  b.rho_r = (1.0 + g) * (1.0 + g) / (1.0 - g) * (1.0 + 0x1p-40) * (1.0 + u) - 1.0 + 0x1p-30;
+  // s32 = fl(s^) with s^ = P / (sqrt(A) sqrt(B)) in double-float: A and B
+  // within g contribute g (half each through the roots), the double-float
+  // operations 2^-40, the final rounding u, P's residue e_p sqrt(A B) an
+  // absolute term; 2^-34 covers underflowed squares and products when
+  // A, B >= 2^-100.
+  b.es_rel = 1.02 * (g / (1.0 - g) + u + 0x1p-40 + 0x1p-34);
   b.es_abs = 1.02 * (ep / (1.0 - g)) + 0x1p-34;
   // float factors: rounding a double to float moves it by at most 2^-24
   // relative, so widening by 2^-22 before the cast keeps each one outward.

@@ -1,0 +1,1004 @@
+// Selection of Algorithm 1 (Stage I top-K1 by H2, Stage II ascending sort by s
+// and stride pick), one CTA per image, with exact decisions.
+//
+// Keys.  H2 = log R with R = L1^2 / S2 (Eq. 3-4: sum_j p_j^2 = S2 / L1^2),
+// so ranking by H2 is ranking by R; s = P / sqrt(A B) (Eq. 6).  The score
+// pass leaves fp32 keys R32 and s32 in each row's statistics record; the CTA
+// sorts them (R descending, s ascending) packed with the token index into
+// 64-bit words so that equal keys order by the lower index.
+//
+// Certification.  The score pass's sums carry proven error bounds (Bounds),
+// so a cut between sorted neighbours is certain when their key intervals do
+// not overlap; with a uniform relative (R) or monotone absolute (s) bound it
+// suffices to test adjacent pairs.  Only decisions matter: the cut at K1 for
+// Stage I and the neighbourhood of each stride position for Stage II.  The
+// tokens of an uncertain run (a maximal stretch of uncertain cuts around a
+// decision) are recomputed exactly -- their five sums as integers, from the
+// input bits -- and ranked by exact rational comparison (cross products of
+// big integers), ties to the lower index.  Rows whose fp32 sums left the
+// error model (non-finite, overflowed, tiny) are recomputed exactly up front.
+#pragma once
+
+#include <cfloat>
+#include <climits>
+#include <cmath>
+
+#include "tr_df.cuh"
+#include "tr_internal.cuh"
+
+namespace tr {
+namespace {
+
+enum : uint8_t {
+  F_IMP = 1,     // in X_imp
+  F_DIV = 2,     // in X_div
+  F_XL = 4,      // exact L1, S2 in the row's ExactRec
+  F_XS = 8,      // exact P, A, B in the row's ExactRec
+  F_NEEDL = 16,  // exact L1, S2 requested
+  F_NEEDS = 32,  // exact P, A, B requested
+  F_RUN = 64,    // lies in an uncertain run around a stride position
+};
+
+// ---------------------------------------------------------------- float keys
+__device__ __forceinline__ uint32_t ord32(float f) {
+  const uint32_t u = __float_as_uint(f);
+  return (u & 0x80000000u) ? ~u : (u | 0x80000000u);
+}
+__device__ __forceinline__ float unord32(uint32_t o) {
+  return __uint_as_float((o & 0x80000000u) ? (o & 0x7fffffffu) : ~o);
+}
+// fp32 keys from the statistics record; NaN = outside the fp32 error model.
+__device__ __forceinline__ float key_r(const float *st) { return __ldcg(st + 6); }
+__device__ __forceinline__ float key_s(const float *st) { return __ldcg(st + 7); }
+
+// ---- a Big truncated to a 64-bit mantissa: value in [m 2^e, (m + 1) 2^e) ----
+// Integer-only (the GPU's fp64 rate is far too low for this path).
+struct Fx {
+  unsigned long long m;  // top bit set, or 0 for the value 0
+  int e;
+};
+__device__ __forceinline__ Fx big_fx(const Big &b) {
+  if (b.n == 0) return Fx{0ull, 0};
+  const int n = b.n;
+  const unsigned long long top = ((unsigned long long)b.l[n - 1] << 32) | (n >= 2 ? b.l[n - 2] : 0u);
+  const uint32_t third = n >= 3 ? b.l[n - 3] : 0u;
+  const int z = __clzll(top);  // < 32: the top limb is non-zero
+  const unsigned long long m = z ? (top << z) | ((unsigned long long)third >> (32 - z)) : top;
+  return Fx{m, 32 * (b.e + n - 2) - z};
+}
+__device__ __forceinline__ Fx fx_one() { return Fx{1ull << 63, -63}; }
+// Product truncated to 64 bits (relative error below 2^-63).
+__device__ __forceinline__ Fx fx_mul(const Fx &a, const Fx &b) {
+  if (!a.m || !b.m) return Fx{0ull, 0};
+  const unsigned long long hi = __umul64hi(a.m, b.m), lo = a.m * b.m;
+  if (hi >> 63) return Fx{hi, a.e + b.e + 64};
+  return Fx{(hi << 1) | (lo >> 63), a.e + b.e + 63};
+}
+// sign(x - y) when |x - y| exceeds 2^-57 of max(x, y), else 0 (too close to
+// call: each side is a product of at most four truncated factors, within
+// 2^-60 of its value).
+__device__ __forceinline__ int fx_cmp(const Fx &x, const Fx &y) {
+  if (!x.m || !y.m) return (x.m != 0) - (y.m != 0);
+  const bool xbig = x.e >= y.e;
+  const Fx &b = xbig ? x : y, &s = xbig ? y : x;
+  const int sh = b.e - s.e;
+  const unsigned long long sm = sh >= 64 ? 0ull : s.m >> sh;
+  if (b.m > sm && b.m - sm > 128ull) return xbig ? 1 : -1;
+  if (sm > b.m && sm - b.m > 128ull) return xbig ? -1 : 1;
+  return 0;
+}
+// Mantissa of a non-zero Fx as a float in [1, 2], rounded to nearest: the Fx
+// value is fx_mant(x) * 2^(x.e + 63).
+__device__ __forceinline__ float fx_mant(const Fx &x) { return __ull2float_rn(x.m) * 0x1p-63f; }
+__device__ __forceinline__ float fx_log(const Fx &x) {  // natural log of a non-zero Fx
+  return logf(fx_mant(x)) + (float)(x.e + 63) * 0.69314718f;
+}
+
+// The mantissa of a non-zero Fx as a double-float in [1, 2] (within 2^-47):
+// the Fx value is fx_f2(x) * 2^(x.e + 63).
+__device__ __forceinline__ df::F2 fx_f2(const Fx &x) {
+  const float h = (float)(x.m >> 40) * 0x1p40f;             // top 24 bits, exact
+  const float l = __ull2float_rn(x.m & ((1ull << 40) - 1));  // the rest, rounded
+  const df::F2 v = df::fast_two_sum(h, l);
+  return df::F2{v.h * 0x1p-63f, v.l * 0x1p-63f};
+}
+
+// Keys of a row settled exactly: the same double-float evaluation as the
+// score pass, from the exact sums (truncated to 64 bits), rounded once.
+__device__ __forceinline__ float exact_r_key(const ExactRec &r) {
+  if (r.flags_l & kRecNonFiniteX) return 0.f;
+  if (r.l1.n == 0) return 1.f;
+  const Fx l1 = big_fx(r.l1), s2 = big_fx(r.s2);
+  const df::F2 L = fx_f2(l1), S = fx_f2(s2);
+  return ldexpf(df::round(df::div(df::mul(L, L), S)), 2 * (l1.e + 63) - (s2.e + 63));
+}
+__device__ __forceinline__ float exact_h2(const ExactRec &r) {
+  if (r.flags_l & kRecNonFiniteX) return -INFINITY;
+  if (r.l1.n == 0) return 0.f;
+  const Fx l1 = big_fx(r.l1), s2 = big_fx(r.s2);
+  return 2.f * fx_log(l1) - fx_log(s2);
+}
+__device__ __forceinline__ float exact_s_key(const ExactRec &r) {
+  if (r.flags_s & kRecNonFiniteS) return 2.f;
+  if (r.a.n == 0 || r.b.n == 0 || r.p.n == 0) return 0.f;
+  const Fx p = big_fx(r.p), a = big_fx(r.a), b = big_fx(r.b);
+  // s = P / sqrt(A B); A and B scaled to even exponents so the roots are exact powers of two
+  df::F2 A = fx_f2(a), B = fx_f2(b);
+  int ea = a.e + 63, eb = b.e + 63;
+  if (ea & 1) {
+    A = df::F2{A.h * 2.f, A.l * 2.f};
+    --ea;
+  }
+  if (eb & 1) {
+    B = df::F2{B.h * 2.f, B.l * 2.f};
+    --eb;
+  }
+  const float v = ldexpf(df::round(df::div(fx_f2(p), df::mul(df::sqrt(A), df::sqrt(B)))), (p.e + 63) - ea / 2 - eb / 2);
+  return r.p.neg ? -v : v;
+}
+
+// Sorted order: ord[q] is the row at position q, key[row] its 32-bit sort
+// key: ~ord32(R32) for the importance order (ascending key = descending R),
+// ord32(s32) for the consistency order.
+__device__ __forceinline__ float r_of(const uint32_t *key, const uint16_t *ord, int q) {
+  return unord32(~key[ord[q]]);
+}
+__device__ __forceinline__ float s_of(const uint32_t *key, const uint16_t *ord, int q) {
+  return unord32(key[ord[q]]);
+}
+
+// Cut between importance-sorted positions q-1 and q is certain when the
+// smallest R the bounds allow at q-1 exceeds the largest R they allow at q;
+// evaluated in fp32 with rounding toward the safe side.
+__device__ __forceinline__ bool cert_r(const uint32_t *key, const uint16_t *ord, int q, const Bounds &bd) {
+  return __fmul_rd(r_of(key, ord, q - 1), bd.r_lo) > __fmul_ru(r_of(key, ord, q), bd.r_hi);
+}
+// Cut between consistency-sorted positions q-1 and q (ascending s32).
+__device__ __forceinline__ bool cert_s(const uint32_t *key, const uint16_t *ord, int q, const Bounds &bd) {
+  const float sa = s_of(key, ord, q - 1), sb = s_of(key, ord, q);
+  const float hi_a = __fadd_ru(sa, __fmaf_ru(bd.s_rel, fabsf(sa), bd.s_abs));
+  const float lo_b = __fsub_rd(sb, __fmaf_ru(bd.s_rel, fabsf(sb), bd.s_abs));
+  return lo_b > hi_a;
+}
+
+// ---------------------------------------------------------------- exact sums
+constexpr int kDig = 20;  // 32-bit digit positions per exact accumulator
+
+struct Term {
+  uint32_t m;  // integer significand
+  int e;       // value = m * 2^e
+  bool nonfinite;
+};
+__device__ __forceinline__ Term decode(const void *base, long long i, bool bf16) {
+  Term t;
+  if (bf16) {
+    const uint32_t b = static_cast<const uint16_t *>(base)[i];
+    const uint32_t ex = (b >> 7) & 0xffu, mant = b & 0x7fu;
+    t.nonfinite = ex == 0xffu;
+    t.m = ex ? (mant | 0x80u) : mant;
+    t.e = (ex ? (int)ex : 1) - 134;
+  } else {
+    const uint32_t b = static_cast<const uint32_t *>(base)[i];
+    const uint32_t ex = (b >> 23) & 0xffu, mant = b & 0x7fffffu;
+    t.nonfinite = ex == 0xffu;
+    t.m = ex ? (mant | 0x800000u) : mant;
+    t.e = (ex ? (int)ex : 1) - 150;
+  }
+  return t;
+}
+__device__ __forceinline__ bool sign_bit(const void *base, long long i, bool bf16) {
+  return bf16 ? (static_cast<const uint16_t *>(base)[i] >> 15) != 0 : (static_cast<const uint32_t *>(base)[i] >> 31) != 0;
+}
+
+// Adds (+/-) m * 2^e into signed 32-bit digit positions relative to 2^base.
+__device__ __forceinline__ void add_term(long long *dg, int base, unsigned long long m, int e, bool negative) {
+  const int off = e - base;  // >= 0 for every finite input value, see the bases below
+  const int k = off >> 5, r = off & 31;
+  const unsigned long long lo = m << r;
+  const unsigned long long hi = r ? (m >> (64 - r)) : 0ull;
+  long long p0 = (long long)(lo & 0xffffffffull), p1 = (long long)(lo >> 32), p2 = (long long)hi;
+  if (negative) {
+    p0 = -p0;
+    p1 = -p1;
+    p2 = -p2;
+  }
+  dg[k] += p0;
+  dg[k + 1] += p1;
+  if (p2) dg[k + 2] += p2;
+}
+
+// Carry-propagates signed digits (value = sum dg[k] 2^(32k + base)) into a
+// trimmed sign-magnitude Big.  Returns false when more than kBigLimbs limbs
+// would be needed.
+__device__ bool normalize(const long long *dg, int base, Big &out) {
+  uint32_t limb[kDig + 2];
+  long long carry = 0;
+  for (int k = 0; k < kDig; ++k) {
+    const long long t = dg[k] + carry;
+    limb[k] = (uint32_t)t;
+    carry = t >> 32;
+  }
+  const bool neg = carry < 0;
+  if (neg) {
+    carry = 0;
+    for (int k = 0; k < kDig; ++k) {
+      const long long t = -dg[k] + carry;
+      limb[k] = (uint32_t)t;
+      carry = t >> 32;
+    }
+  }
+  limb[kDig] = (uint32_t)carry;
+  limb[kDig + 1] = (uint32_t)(carry >> 32);
+  int hi = kDig + 1;
+  while (hi >= 0 && limb[hi] == 0) --hi;
+  out.neg = 0;
+  if (hi < 0) {
+    out.n = 0;
+    out.e = 0;
+    return true;
+  }
+  int lo = 0;
+  while (limb[lo] == 0) ++lo;
+  const int n = hi - lo + 1;
+  if (n > kBigLimbs) {
+    out.n = 0;
+    out.e = 0;
+    return false;
+  }
+  for (int i = 0; i < n; ++i) out.l[i] = limb[lo + i];
+  out.n = (uint8_t)n;
+  out.e = (int16_t)(lo + base / 32);
+  out.neg = neg ? 1 : 0;
+  return true;
+}
+
+__device__ __forceinline__ void warp_sum_digits(long long *dg) {
+  for (int k = 0; k < kDig; ++k) {
+    long long v = dg[k];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    dg[k] = v;
+  }
+}
+
+// Exact sums of one row, computed by one warp.  mode 0: L1 = sum|x| and
+// S2 = sum x^2; mode 1: A = sum x'^2, B = sum x''^2, P = sum x'x''.
+// Digit bases (multiples of 32): |x| has exponent >= -133 (bf16) or -149
+// (fp32), products >= -266 or -298; the top digit stays below kDig.
+__device__ __noinline__ void exact_row(const SelectArgs &a, long long row, int mode, ExactRec *rec, int lane) {
+  const bool bf16 = a.dtype == TR_BF16;
+  const int base1 = -160;
+  const int base2 = bf16 ? -288 : -320;
+  long long d0[kDig], d1[kDig], d2[kDig];
+  for (int k = 0; k < kDig; ++k) d0[k] = d1[k] = d2[k] = 0;
+  bool nonfinite = false;
+  const long long first = row * (long long)a.d;
+  if (mode == 0) {
+    for (int j = lane; j < a.d; j += 32) {
+      const Term t = decode(a.x, first + j, bf16);
+      if (t.nonfinite) {
+        nonfinite = true;
+      } else if (t.m) {
+        add_term(d0, base1, t.m, t.e, false);
+        add_term(d1, base2, (unsigned long long)t.m * t.m, 2 * t.e, false);
+      }
+    }
+  } else {
+    const void *xp = a.x_pre ? a.x_pre : a.x;
+    for (int j = lane; j < a.d; j += 32) {
+      const Term p = decode(xp, first + j, bf16);
+      const Term q = decode(a.x_post, first + j, bf16);
+      if (p.nonfinite || q.nonfinite) {
+        nonfinite = true;
+        continue;
+      }
+      if (p.m) add_term(d0, base2, (unsigned long long)p.m * p.m, 2 * p.e, false);
+      if (q.m) add_term(d1, base2, (unsigned long long)q.m * q.m, 2 * q.e, false);
+      if (p.m && q.m) {
+        const bool neg = sign_bit(xp, first + j, bf16) != sign_bit(a.x_post, first + j, bf16);
+        add_term(d2, base2, (unsigned long long)p.m * q.m, p.e + q.e, neg);
+      }
+    }
+  }
+  nonfinite = __any_sync(0xffffffffu, nonfinite);
+  warp_sum_digits(d0);
+  warp_sum_digits(d1);
+  if (mode == 1) warp_sum_digits(d2);
+  if (lane == 0) {
+    uint32_t flags = 0;
+    if (mode == 0) {
+      if (nonfinite) flags |= kRecNonFiniteX;
+      bool ok = normalize(d0, base1, rec->l1);
+      ok = normalize(d1, base2, rec->s2) && ok;
+      if (!ok) flags |= kRecOverflowL;
+      rec->flags_l = flags;
+    } else {
+      if (nonfinite) flags |= kRecNonFiniteS;
+      bool ok = normalize(d0, base2, rec->a);
+      ok = normalize(d1, base2, rec->b) && ok;
+      ok = normalize(d2, base2, rec->p) && ok;
+      if (!ok) flags |= kRecOverflowS;
+      rec->flags_s = flags;
+    }
+  }
+}
+
+// ---- fast exact sums: one 128-bit integer per sum, in registers ----------
+// Every term is m * 2^e with an integer m of at most 2 * kMant bits.  With
+// the row's smallest exponent as the base, term m * 2^(e - base) and the sum
+// of all d terms fit 127 bits whenever the row's exponent span is moderate
+// (always for ordinary activations); the warp checks that first and falls
+// back to the digit accumulator above otherwise.
+struct Dec {
+  uint32_t m;
+  int e;
+  bool neg, nf;
+};
+__device__ __forceinline__ Dec dec16(uint32_t h) {
+  const uint32_t ex = (h >> 7) & 0xffu, mant = h & 0x7fu;
+  return Dec{ex ? (mant | 0x80u) : mant, (ex ? (int)ex : 1) - 134, (h >> 15) != 0, ex == 0xffu};
+}
+__device__ __forceinline__ Dec dec32(uint32_t b) {
+  const uint32_t ex = (b >> 23) & 0xffu, mant = b & 0x7fffffu;
+  return Dec{ex ? (mant | 0x800000u) : mant, (ex ? (int)ex : 1) - 150, (b >> 31) != 0, ex == 0xffu};
+}
+
+template <bool kBf16>
+__device__ __forceinline__ void unpack(const uint4 &v, Dec *out) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  if (kBf16) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      out[2 * i] = dec16(w[i] & 0xffffu);
+      out[2 * i + 1] = dec16(w[i] >> 16);
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) out[i] = dec32(w[i]);
+  }
+}
+
+__device__ __forceinline__ void add128(__int128 &acc, unsigned long long m, int sh, bool neg) {
+  const __int128 v = (__int128)((unsigned __int128)m << sh);
+  acc = neg ? acc - v : acc + v;
+}
+__device__ __forceinline__ __int128 warp_sum128(__int128 v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const unsigned long long lo = __shfl_xor_sync(0xffffffffu, (unsigned long long)v, o);
+    const unsigned long long hi = __shfl_xor_sync(0xffffffffu, (unsigned long long)((unsigned __int128)v >> 64), o);
+    v += (__int128)(((unsigned __int128)hi << 64) | lo);
+  }
+  return v;
+}
+
+// value = v * 2^base as a trimmed Big (|v| < 2^127, so at most 5 limbs).
+__device__ void int128_to_big(__int128 v, int base, Big &out) {
+  const bool neg = v < 0;
+  const unsigned __int128 mag = neg ? (unsigned __int128)(-v) : (unsigned __int128)v;
+  out.neg = neg ? 1 : 0;
+  if (mag == 0) {
+    out.n = 0;
+    out.e = 0;
+    out.neg = 0;
+    return;
+  }
+  const int q = base >> 5, r = base & 31;  // base = 32 q + r, 0 <= r < 32
+  const unsigned __int128 lo = mag << r;
+  uint32_t limb[5] = {(uint32_t)lo, (uint32_t)(lo >> 32), (uint32_t)(lo >> 64), (uint32_t)(lo >> 96),
+                      r ? (uint32_t)(mag >> (128 - r)) : 0u};
+  int hi = 4;
+  while (limb[hi] == 0) --hi;
+  int l = 0;
+  while (limb[l] == 0) ++l;
+  out.n = (uint8_t)(hi - l + 1);
+  for (int i = 0; i < out.n; ++i) out.l[i] = limb[l + i];
+  out.e = (int16_t)(q + l);
+}
+
+// Window for one exact sum: every term and the sum are below 2^top, where
+// 2^top exceeds 1.5 x (the fp32 sum of |terms|, itself within 1e-6 of the
+// truth); terms are integers times 2^bottom with bottom = top - 126, so the
+// signed 128-bit accumulator cannot overflow.  A term with a lower bit below
+// 2^bottom does not fit (the row spans > ~95 binades): the caller falls back.
+__device__ __forceinline__ int window_bottom(float bound) {
+  int ex;
+  frexpf(bound * 1.5f, &ex);  // bound * 1.5 < 2^ex
+  return ex - 126;
+}
+
+constexpr int kWarps = kSelectThreads / 32;
+
+// 128-bit partial sums of the warps, reduced by thread 0.
+struct Part128 {
+  unsigned long long lo[kWarps * 3], hi[kWarps * 3];
+};
+__device__ __forceinline__ void part_put(Part128 &p, int slot, __int128 v) {
+  p.lo[slot] = (unsigned long long)v;
+  p.hi[slot] = (unsigned long long)((unsigned __int128)v >> 64);
+}
+__device__ __forceinline__ __int128 part_sum(const Part128 &p, int which) {
+  __int128 v = 0;
+  for (int w = 0; w < kWarps; ++w)
+    v += (__int128)(((unsigned __int128)p.hi[w * 3 + which] << 64) | p.lo[w * 3 + which]);
+  return v;
+}
+
+// Exact sums of one row computed by the whole CTA (one 16-byte chunk of each
+// stream per thread and pass), in three 128-bit windows; false (uniformly)
+// when a term does not fit its window.
+template <bool kBf16>
+__device__ bool exact_row_block(const SelectArgs &a, long long row, int mode, const float *st, ExactRec *rec,
+                                Part128 &part) {
+  constexpr int kPer = kBf16 ? 8 : 4;  // elements per 16-byte chunk
+  const int nchunks = a.d / kPer;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  bool fits = true;
+  Dec e0[kPer], e1[kPer];
+  __int128 s0 = 0, s1 = 0, s2 = 0;
+  int b0, b1, b2 = 0;
+  if (mode == 0) {
+    b0 = window_bottom(__ldcg(st + 0));
+    b1 = window_bottom(__ldcg(st + 1));
+    const uint4 *px = static_cast<const uint4 *>(a.x) + row * nchunks;
+#pragma unroll 4
+    for (int c = threadIdx.x; c < nchunks; c += blockDim.x) {
+      unpack<kBf16>(__ldg(px + c), e0);
+#pragma unroll
+      for (int i = 0; i < kPer; ++i) {
+        const Dec &t = e0[i];
+        if (!t.m) continue;
+        if (t.nf || t.e < b0 || 2 * t.e < b1) {
+          fits = false;
+          continue;
+        }
+        add128(s0, t.m, t.e - b0, false);
+        add128(s1, (unsigned long long)t.m * t.m, 2 * t.e - b1, false);
+      }
+    }
+  } else {
+    const float sa = __ldcg(st + 2), sb = __ldcg(st + 3);
+    b0 = window_bottom(sa);
+    b1 = window_bottom(sb);
+    b2 = window_bottom(__fsqrt_ru(sa) * __fsqrt_ru(sb));
+    const uint4 *pp = static_cast<const uint4 *>(a.x_pre ? a.x_pre : a.x) + row * nchunks;
+    const uint4 *pq = static_cast<const uint4 *>(a.x_post) + row * nchunks;
+#pragma unroll 4
+    for (int c = threadIdx.x; c < nchunks; c += blockDim.x) {
+      unpack<kBf16>(__ldg(pp + c), e0);
+      unpack<kBf16>(__ldg(pq + c), e1);
+#pragma unroll
+      for (int i = 0; i < kPer; ++i) {
+        const Dec &p = e0[i], &q = e1[i];
+        if (p.nf || q.nf) {
+          fits = false;
+          continue;
+        }
+        if (p.m) {
+          if (2 * p.e < b0) fits = false; else add128(s0, (unsigned long long)p.m * p.m, 2 * p.e - b0, false);
+        }
+        if (q.m) {
+          if (2 * q.e < b1) fits = false; else add128(s1, (unsigned long long)q.m * q.m, 2 * q.e - b1, false);
+        }
+        if (p.m && q.m) {
+          if (p.e + q.e < b2) fits = false;
+          else add128(s2, (unsigned long long)p.m * q.m, p.e + q.e - b2, p.neg != q.neg);
+        }
+      }
+    }
+  }
+  if (!__syncthreads_and(fits)) return false;
+  s0 = warp_sum128(s0);
+  s1 = warp_sum128(s1);
+  s2 = warp_sum128(s2);
+  if (lane == 0) {
+    part_put(part, warp * 3 + 0, s0);
+    part_put(part, warp * 3 + 1, s1);
+    part_put(part, warp * 3 + 2, s2);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    if (mode == 0) {
+      int128_to_big(part_sum(part, 0), b0, rec->l1);
+      int128_to_big(part_sum(part, 1), b1, rec->s2);
+      rec->flags_l = 0u;
+    } else {
+      int128_to_big(part_sum(part, 0), b0, rec->a);
+      int128_to_big(part_sum(part, 1), b1, rec->b);
+      int128_to_big(part_sum(part, 2), b2, rec->p);
+      rec->flags_s = 0u;
+    }
+  }
+  __syncthreads();
+  return true;
+}
+
+// Exact sums of one row by the whole CTA: the 128-bit windows when the row's
+// fp32 sums are trustworthy and its terms fit, else warp 0 runs the digit
+// accumulator (non-finite or extreme rows).
+__device__ __forceinline__ void exact_row_any(const SelectArgs &a, long long row, int mode, const float *st,
+                                              ExactRec *rec, Part128 &part) {
+  const bool trusted = mode == 0 ? !isnan(key_r(st)) : !isnan(key_s(st));
+  bool ok = false;
+  if (trusted)
+    ok = a.dtype == TR_BF16 ? exact_row_block<true>(a, row, mode, st, rec, part)
+                            : exact_row_block<false>(a, row, mode, st, rec, part);
+  if (!ok) {
+    if ((threadIdx.x >> 5) == 0) exact_row(a, row, mode, rec, threadIdx.x & 31);
+    __syncthreads();
+  }
+}
+
+// Recomputes, one row at a time with the whole CTA, the rows whose flags
+// request it; clears the request and records what is now exact.  A single
+// block-wide vote skips the scan when nothing is pending.
+__device__ void refine_pending(const SelectArgs &a, long long off, int n, uint8_t *fl, ExactRec *rec) {
+  __shared__ unsigned wmask[kWarps];
+  __shared__ Part128 part;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  bool any = false;
+  for (int i = threadIdx.x; i < n; i += blockDim.x) any |= (fl[i] & (F_NEEDL | F_NEEDS)) != 0;
+  if (!__syncthreads_or(any)) return;
+  for (int base = 0; base < n; base += blockDim.x) {
+    const int i = base + threadIdx.x;
+    const unsigned m = __ballot_sync(0xffffffffu, i < n && (fl[i] & (F_NEEDL | F_NEEDS)) != 0);
+    if (lane == 0) wmask[warp] = m;
+    __syncthreads();
+    for (int w = 0; w < kWarps; ++w) {
+      unsigned mm = wmask[w];
+      while (mm) {
+        const int r = __ffs(mm) - 1;
+        mm &= mm - 1;
+        const int row = base + 32 * w + r;
+        const uint8_t fr = fl[row];
+        const float *st = a.stats + (off + row) * TR_STATS_WORDS;
+        if (fr & F_NEEDL) exact_row_any(a, off + row, 0, st, rec + row, part);
+        if (fr & F_NEEDS) exact_row_any(a, off + row, 1, st, rec + row, part);
+        if (threadIdx.x == 0) {
+          fl[row] = (uint8_t)((fr & ~(F_NEEDL | F_NEEDS)) | ((fr & F_NEEDL) ? F_XL : 0) | ((fr & F_NEEDS) ? F_XS : 0));
+          if (a.status) atomicAdd(&a.status[2], 1);
+        }
+      }
+    }
+    __syncthreads();
+  }
+}
+
+// ---------------------------------------------------------------- exact comparisons
+constexpr int kWide = 4 * kBigLimbs;
+struct Wide {
+  uint32_t l[kWide];
+  int n;
+  int e;
+};
+__device__ __forceinline__ void wide_from(const Big &b, Wide &w) {
+  w.n = b.n;
+  w.e = b.e;
+  for (int i = 0; i < b.n; ++i) w.l[i] = b.l[i];
+}
+__device__ __forceinline__ void wide_one(Wide &w) {
+  w.n = 1;
+  w.e = 0;
+  w.l[0] = 1u;
+}
+// out = a * b (magnitudes); a.n + b.n <= kWide at every call site.
+__device__ void wide_mul(const Wide &a, const Wide &b, Wide &out) {
+  if (a.n == 0 || b.n == 0) {
+    out.n = 0;
+    out.e = 0;
+    return;
+  }
+  out.n = a.n + b.n;
+  out.e = a.e + b.e;
+  for (int i = 0; i < out.n; ++i) out.l[i] = 0u;
+  for (int i = 0; i < a.n; ++i) {
+    unsigned long long carry = 0;
+    for (int j = 0; j < b.n; ++j) {
+      const unsigned long long t = (unsigned long long)a.l[i] * b.l[j] + out.l[i + j] + carry;
+      out.l[i + j] = (uint32_t)t;
+      carry = t >> 32;
+    }
+    out.l[i + b.n] = (uint32_t)carry;
+  }
+  while (out.n > 0 && out.l[out.n - 1] == 0u) --out.n;
+}
+__device__ int wide_cmp(const Wide &x, const Wide &y) {
+  if (x.n == 0 || y.n == 0) return (x.n != 0) - (y.n != 0);
+  const int tx = 32 * (x.e + x.n) - __clz(x.l[x.n - 1]);
+  const int ty = 32 * (y.e + y.n) - __clz(y.l[y.n - 1]);
+  if (tx != ty) return tx > ty ? 1 : -1;
+  const int hi = max(x.e + x.n, y.e + y.n) - 1, lo = min(x.e, y.e);
+  for (int p = hi; p >= lo; --p) {
+    const uint32_t u = (p >= x.e && p < x.e + x.n) ? x.l[p - x.e] : 0u;
+    const uint32_t v = (p >= y.e && p < y.e + y.n) ? y.l[p - y.e] : 0u;
+    if (u != v) return u > v ? 1 : -1;
+  }
+  return 0;
+}
+
+// sign(R_a - R_b), R = L1^2 / S2 (R = 1 for an all-zero row, non-finite rows
+// lowest), by big-integer cross products.
+__device__ __noinline__ int cmp_r_big(const ExactRec &ra, const ExactRec &rb) {
+  const bool na = ra.flags_l & kRecNonFiniteX, nb = rb.flags_l & kRecNonFiniteX;
+  if (na || nb) return na == nb ? 0 : (na ? -1 : 1);
+  Wide l1a, s2a, l1b, s2b, t, x, y;
+  if (ra.l1.n == 0) {
+    wide_one(l1a);
+    wide_one(s2a);
+  } else {
+    wide_from(ra.l1, l1a);
+    wide_from(ra.s2, s2a);
+  }
+  if (rb.l1.n == 0) {
+    wide_one(l1b);
+    wide_one(s2b);
+  } else {
+    wide_from(rb.l1, l1b);
+    wide_from(rb.s2, s2b);
+  }
+  wide_mul(l1a, l1a, t);
+  wide_mul(t, s2b, x);
+  wide_mul(l1b, l1b, t);
+  wide_mul(t, s2a, y);
+  return wide_cmp(x, y);
+}
+
+// sign(s_a - s_b) through sigma = sign(P) P^2 / (A B) (s = 0 when A or B is 0,
+// non-finite rows highest), by big-integer cross products.
+__device__ __noinline__ int cmp_s_big(const ExactRec &ra, const ExactRec &rb) {
+  const bool na = ra.flags_s & kRecNonFiniteS, nb = rb.flags_s & kRecNonFiniteS;
+  if (na || nb) return na == nb ? 0 : (na ? 1 : -1);
+  const int sa = (ra.a.n == 0 || ra.b.n == 0 || ra.p.n == 0) ? 0 : (ra.p.neg ? -1 : 1);
+  const int sb = (rb.a.n == 0 || rb.b.n == 0 || rb.p.n == 0) ? 0 : (rb.p.neg ? -1 : 1);
+  if (sa != sb) return sa > sb ? 1 : -1;
+  if (sa == 0) return 0;
+  Wide pa, aa, ba, pb, ab, bb, t, u, x, y;
+  wide_from(ra.p, pa);
+  wide_from(ra.a, aa);
+  wide_from(ra.b, ba);
+  wide_from(rb.p, pb);
+  wide_from(rb.a, ab);
+  wide_from(rb.b, bb);
+  wide_mul(pa, pa, t);
+  wide_mul(t, ab, u);
+  wide_mul(u, bb, x);
+  wide_mul(pb, pb, t);
+  wide_mul(t, aa, u);
+  wide_mul(u, ba, y);
+  const int c = wide_cmp(x, y);
+  return sa > 0 ? c : -c;
+}
+
+// The same comparisons screened first with 64-bit truncated mantissas
+// (integer arithmetic only); only gaps below 2^-57 relative -- in practice
+// exact ties -- go on to the big-integer cross products.
+__device__ int cmp_r(const ExactRec &ra, const ExactRec &rb) {
+  const bool na = ra.flags_l & kRecNonFiniteX, nb = rb.flags_l & kRecNonFiniteX;
+  if (na || nb) return na == nb ? 0 : (na ? -1 : 1);
+  const Fx l1a = ra.l1.n ? big_fx(ra.l1) : fx_one(), s2a = ra.l1.n ? big_fx(ra.s2) : fx_one();
+  const Fx l1b = rb.l1.n ? big_fx(rb.l1) : fx_one(), s2b = rb.l1.n ? big_fx(rb.s2) : fx_one();
+  const int c = fx_cmp(fx_mul(fx_mul(l1a, l1a), s2b), fx_mul(fx_mul(l1b, l1b), s2a));
+  return c ? c : cmp_r_big(ra, rb);
+}
+__device__ int cmp_s(const ExactRec &ra, const ExactRec &rb) {
+  const bool na = ra.flags_s & kRecNonFiniteS, nb = rb.flags_s & kRecNonFiniteS;
+  if (na || nb) return na == nb ? 0 : (na ? 1 : -1);
+  const int sa = (ra.a.n == 0 || ra.b.n == 0 || ra.p.n == 0) ? 0 : (ra.p.neg ? -1 : 1);
+  const int sb = (rb.a.n == 0 || rb.b.n == 0 || rb.p.n == 0) ? 0 : (rb.p.neg ? -1 : 1);
+  if (sa != sb) return sa > sb ? 1 : -1;
+  if (sa == 0) return 0;
+  const Fx pa = big_fx(ra.p), pb = big_fx(rb.p);
+  const Fx x = fx_mul(fx_mul(fx_mul(pa, pa), big_fx(rb.a)), big_fx(rb.b));
+  const Fx y = fx_mul(fx_mul(fx_mul(pb, pb), big_fx(ra.a)), big_fx(ra.b));
+  const int c = fx_cmp(x, y);
+  return c ? c * sa : cmp_s_big(ra, rb);
+}
+
+// ---------------------------------------------------------------- block helpers
+
+__device__ int block_exclusive_scan(int v, int *total) {
+  __shared__ int wsum[32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  __syncthreads();  // wsum may still be read by a previous call
+  int x = v;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int y = __shfl_up_sync(0xffffffffu, x, o);
+    if (lane >= o) x += y;
+  }
+  if (lane == 31) wsum[warp] = x;
+  __syncthreads();
+  if (warp == 0) {
+    int w = lane < nwarps ? wsum[lane] : 0;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(0xffffffffu, w, o);
+      if (lane >= o) w += y;
+    }
+    wsum[lane] = w;
+  }
+  __syncthreads();
+  *total = wsum[nwarps - 1];
+  return (warp ? wsum[warp - 1] : 0) + x - v;
+}
+
+// Stable ascending LSD radix sort (8-bit digits) of the m rows listed in a
+// by key[row]; b is scratch of the same size and hist holds kWarps x 256
+// counters.  Warp w owns the contiguous stretch w of the current order:
+// per-warp digit counts, a column scan (digit-major, then warp), then each
+// warp scatters its stretch in order, ranking equal digits within 32 lanes
+// with match-any, which keeps the sort stable.  A pass whose digit is the
+// same for every row is skipped.  Returns the buffer holding the order.
+__device__ uint16_t *radix_sort(const uint32_t *key, uint16_t *a, uint16_t *b, int m, uint32_t *hist) {
+  __shared__ int skip;
+  __shared__ uint32_t dsum[8];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int seg = (m + kWarps - 1) / kWarps;
+  const int s0 = min(m, warp * seg), s1 = min(m, s0 + seg);
+  uint32_t *h = hist + warp * 256;
+  const unsigned lt = (1u << lane) - 1u;
+  if (m < 2) return a;
+  for (int shift = 0; shift < 32; shift += 8) {
+    for (int d = lane; d < 256; d += 32) h[d] = 0u;
+    if (tid == 0) skip = 0;
+    __syncwarp();
+    for (int q = s0 + lane; q < s1; q += 32) atomicAdd(&h[(key[a[q]] >> shift) & 0xffu], 1u);
+    __syncthreads();
+    uint32_t total = 0;
+    if (tid < 256) {
+      for (int w = 0; w < kWarps; ++w) {
+        const uint32_t c = hist[w * 256 + tid];
+        hist[w * 256 + tid] = total;
+        total += c;
+      }
+      if (total == (uint32_t)m) skip = 1;
+    }
+    uint32_t incl = total;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+      if (lane >= o) incl += y;
+    }
+    if (tid < 256 && lane == 31) dsum[warp] = incl;
+    __syncthreads();
+    if (tid < 256) {
+      uint32_t base = 0;
+      for (int w = 0; w < warp; ++w) base += dsum[w];
+      const uint32_t excl = base + incl - total;
+      for (int w = 0; w < kWarps; ++w) hist[w * 256 + tid] += excl;
+    }
+    __syncthreads();
+    if (!skip) {
+      for (int q0 = s0; q0 < s1; q0 += 32) {
+        const int q = q0 + lane;
+        const bool act = q < s1;
+        const unsigned am = __ballot_sync(0xffffffffu, act);
+        if (act) {
+          const uint16_t row = a[q];
+          const uint32_t d = (key[row] >> shift) & 0xffu;
+          const unsigned peers = __match_any_sync(am, d);
+          const int rank = __popc(peers & lt);
+          const uint32_t base = h[d];
+          b[base + rank] = row;
+          __syncwarp(am);
+          if (rank == 0) h[d] = base + __popc(peers);
+        }
+        __syncwarp();
+      }
+      uint16_t *t = a;
+      a = b;
+      b = t;
+    }
+    __syncthreads();
+  }
+  return a;
+}
+
+__host__ __device__ inline int row_capacity(int max_n) { return (max_n + 15) / 16 * 16; }
+
+// ---------------------------------------------------------------- one image
+// Algorithm 1 for image b, by the whole CTA (kSelectThreads threads);
+// smem holds select_smem_bytes(a.max_n) bytes.  Reads the statistics through
+// L2 so that rows scored by other CTAs of the same launch are seen.
+__device__ void select_image(const SelectArgs &a, const int b, unsigned char *smem) {
+  __shared__ int sh_lo, sh_hi;
+  const int tid = threadIdx.x, nthr = blockDim.x;
+  long long off;
+  int n;
+  if (a.cu_seqlens) {
+    off = a.cu_seqlens[b];
+    n = a.cu_seqlens[b + 1] - a.cu_seqlens[b];
+  } else {
+    off = (long long)b * a.n_uniform;
+    n = a.n_uniform;
+  }
+  const int k = a.k[b], k1 = a.k1[b], k2 = k - k1, ko = a.cu_k[b];
+  if (n < 0 || n > a.max_n || k < 0 || k > n || k1 < 0 || k1 > k) {
+    if (tid == 0 && a.status) atomicAdd(&a.status[3], 1);
+    return;
+  }
+  if (n == 0) return;
+  const int cap = row_capacity(a.max_n);
+  uint32_t *key = reinterpret_cast<uint32_t *>(smem);        // [cap] sort key per row
+  uint16_t *ia = reinterpret_cast<uint16_t *>(key + cap);    // [cap] order buffers
+  uint16_t *ib = ia + cap;                                   // [cap]
+  uint32_t *hist = reinterpret_cast<uint32_t *>(ib + cap);   // [kWarps x 256]
+  uint8_t *fl = reinterpret_cast<uint8_t *>(hist + kWarps * 256);  // [cap] row flags
+  const float *st = a.stats + off * TR_STATS_WORDS;
+  ExactRec *rec = a.exact + off;
+  const bool need_r = k1 > 0 && k1 < n;  // the importance order decides something
+  const bool need_s = k2 > 0;
+
+  // 1. Rows whose fp32 sums left the error model are settled exactly first
+  //    (also when only their H2 / s outputs need it).
+  for (int i = tid; i < n; i += nthr) {
+    const float *r = st + (long long)i * TR_STATS_WORDS;
+    uint8_t f = 0;
+    if ((need_r || a.h2) && isnan(key_r(r))) f |= F_NEEDL;
+    if ((need_s || a.s) && isnan(key_s(r))) f |= F_NEEDS;
+    fl[i] = f;
+  }
+  __syncthreads();
+  refine_pending(a, off, n, fl, rec);
+  __syncthreads();
+
+  // 2. Stage I: top-K1 by R (equivalently H2), descending, lower index first.
+  if (need_r) {
+    for (int i = tid; i < n; i += nthr) {
+      const float r = (fl[i] & F_XL) ? exact_r_key(rec[i]) : key_r(st + (long long)i * TR_STATS_WORDS);
+      key[i] = ~ord32(r);
+      ia[i] = (uint16_t)i;
+    }
+    __syncthreads();
+    const uint16_t *ord = radix_sort(key, ia, ib, n, hist);
+    if (tid == 0) {
+      int lo = k1, hi = k1;
+      if (!cert_r(key, ord, k1, a.bounds)) {
+        lo = k1 - 1;
+        while (lo > 0 && !cert_r(key, ord, lo, a.bounds)) --lo;
+        hi = k1 + 1;
+        while (hi < n && !cert_r(key, ord, hi, a.bounds)) ++hi;
+      }
+      sh_lo = lo;
+      sh_hi = hi;
+    }
+    __syncthreads();
+    const int lo = sh_lo, hi = sh_hi;
+    for (int q = tid; q < lo; q += nthr) fl[ord[q]] |= F_IMP;
+    if (hi > lo) {
+      for (int q = lo + tid; q < hi; q += nthr) {
+        const int r = ord[q];
+        if (!(fl[r] & F_XL)) fl[r] |= F_NEEDL;
+      }
+      __syncthreads();
+      refine_pending(a, off, n, fl, rec);
+      __syncthreads();
+      for (int q = lo + tid; q < hi; q += nthr) {
+        const int r = ord[q];
+        const bool ovf = rec[r].flags_l & kRecOverflowL;
+        int rank = 0;
+        for (int q2 = lo; q2 < hi; ++q2) {
+          if (q2 == q) continue;
+          const int r2 = ord[q2];
+          int c;
+          if (ovf || (rec[r2].flags_l & kRecOverflowL))
+            c = q2 < q ? 1 : -1;  // no exact value: keep the float order
+          else
+            c = cmp_r(rec[r2], rec[r]);
+          if (c > 0 || (c == 0 && r2 < r)) ++rank;
+        }
+        if (lo + rank < k1) fl[r] |= F_IMP;
+      }
+    }
+    __syncthreads();
+  } else if (k1 == n) {
+    for (int i = tid; i < n; i += nthr) fl[i] |= F_IMP;
+    __syncthreads();
+  }
+
+  // 3. Stage II: sort X_rem by s ascending, pick positions 0, t, 2t, ...
+  if (need_s) {
+    // X_rem in ascending index order (the stable sort's tie order)
+    const int per = (n + nthr - 1) / nthr;
+    const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
+    int cnt = 0;
+    for (int i = i0; i < i1; ++i) cnt += !(fl[i] & F_IMP);
+    int m = 0;
+    int pos = block_exclusive_scan(cnt, &m);
+    for (int i = i0; i < i1; ++i) {
+      if (fl[i] & F_IMP) continue;
+      ia[pos++] = (uint16_t)i;
+      const float sv = (fl[i] & F_XS) ? exact_s_key(rec[i]) : key_s(st + (long long)i * TR_STATS_WORDS);
+      key[i] = ord32(sv);
+    }
+    __syncthreads();
+    const uint16_t *ord = radix_sort(key, ia, ib, m, hist);
+    const int t = max(1, m / k2);
+    for (int j = tid; j < k2; j += nthr) {
+      const int p = j * t;
+      const bool c0 = p == 0 || cert_s(key, ord, p, a.bounds);
+      const bool c1 = p + 1 >= m || cert_s(key, ord, p + 1, a.bounds);
+      if (c0 && c1) {
+        fl[ord[p]] |= F_DIV;
+      } else {
+        int lo = p;
+        while (lo > 0 && !cert_s(key, ord, lo, a.bounds)) --lo;
+        int hi = p + 1;
+        while (hi < m && !cert_s(key, ord, hi, a.bounds)) ++hi;
+        // Threads whose runs coincide write the same bits: the races are benign.
+        for (int q = lo; q < hi; ++q) {
+          const int r = ord[q];
+          fl[r] |= (uint8_t)(F_RUN | ((fl[r] & F_XS) ? 0 : F_NEEDS));
+        }
+      }
+    }
+    __syncthreads();
+    refine_pending(a, off, n, fl, rec);
+    __syncthreads();
+    for (int q = tid; q < m; q += nthr) {
+      const int r = ord[q];
+      if (!(fl[r] & F_RUN)) continue;
+      int lo = q;
+      while (lo > 0 && !cert_s(key, ord, lo, a.bounds)) --lo;
+      int hi = q + 1;
+      while (hi < m && !cert_s(key, ord, hi, a.bounds)) ++hi;
+      const bool ovf = rec[r].flags_s & kRecOverflowS;
+      int rank = 0;
+      for (int q2 = lo; q2 < hi; ++q2) {
+        if (q2 == q) continue;
+        const int r2 = ord[q2];
+        int c;
+        if (ovf || (rec[r2].flags_s & kRecOverflowS))
+          c = q2 < q ? -1 : 1;
+        else
+          c = cmp_s(rec[r2], rec[r]);
+        if (c < 0 || (c == 0 && r2 < r)) ++rank;
+      }
+      const int pp = lo + rank;
+      if (pp % t == 0 && pp / t < k2) fl[r] |= F_DIV;
+    }
+    __syncthreads();
+  }
+
+  // 4. X* = X_imp union X_div in ascending token order (Eq. 7), plus outputs.
+  const int per = (n + nthr - 1) / nthr;
+  const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
+  int cnt = 0;
+  for (int i = i0; i < i1; ++i) cnt += (fl[i] & (F_IMP | F_DIV)) != 0;
+  int kept_total = 0;
+  int pos = ko + block_exclusive_scan(cnt, &kept_total);
+  for (int i = i0; i < i1; ++i) {
+    const uint8_t f = fl[i];
+    if ((f & (F_IMP | F_DIV)) && pos < ko + k) {  // never write past this image's slots
+      a.idx[pos] = i;
+      ++pos;
+    }
+    if (a.role) a.role[off + i] = (f & F_IMP) ? 1 : ((f & F_DIV) ? 2 : 0);
+    int nonfinite = 0, overflow = 0;
+    if (f & F_XL) {
+      const ExactRec &r = rec[i];
+      nonfinite |= (r.flags_l & kRecNonFiniteX) != 0;
+      overflow |= (r.flags_l & kRecOverflowL) != 0;
+      if (a.h2 && !(r.flags_l & kRecOverflowL))
+        a.h2[off + i] = exact_h2(r);
+    }
+    if (f & F_XS) {
+      const ExactRec &r = rec[i];
+      nonfinite |= (r.flags_s & kRecNonFiniteS) != 0;
+      overflow |= (r.flags_s & kRecOverflowS) != 0;
+      if (a.s && !(r.flags_s & kRecOverflowS))
+        a.s[off + i] = (r.flags_s & kRecNonFiniteS) ? INFINITY : exact_s_key(r);
+    }
+    if (a.status) {
+      if (nonfinite) atomicAdd(&a.status[0], 1);
+      if (overflow) atomicAdd(&a.status[1], 1);
+    }
+  }
+  if (tid == 0 && kept_total != k && a.status) atomicAdd(&a.status[3], 1);
+}
+
+}  // namespace
+
+size_t select_smem_bytes(int max_n);
+
+}  // namespace tr
