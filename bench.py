@@ -50,7 +50,7 @@ BUDGETS = {
 def _args():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=1000)
+    ap.add_argument("--steps", type=int, default=4000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="llava576", choices=sorted(BUDGETS))
@@ -69,6 +69,26 @@ def _dist():
     rank = int(os.environ.get("RANK", "0"))
     local = int(os.environ.get("LOCAL_RANK", "0"))
     return world, rank, local
+
+
+def rank_seed(seed: int, rank: int) -> int:
+    """Seed of a rank's batch: every rank reduces its own images (weak scaling)."""
+    return seed + 1000 * rank
+
+
+def max_over_ranks(value: float, world: int, device=None) -> float:
+    """The slowest rank's time (the job finishes when it does)."""
+    if world <= 1:
+        return value
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_images_per_s(images_per_rank: int, world: int, ms_step_max: float) -> float:
+    """Whole-job throughput: all ranks' images over the slowest rank's step time."""
+    return images_per_rank * world / (ms_step_max * 1e-3)
 
 
 def _peaks():
@@ -213,7 +233,7 @@ def run_reference(args, world, rank):
 # ---------------------------------------------------------------- traffic from the committed ncu summary
 def _score_source_hash():
     h = hashlib.sha256()
-    for f in ("tr_score.cu", "tr_internal.cuh"):
+    for f in ("tr_score.cu", "tr_score_dev.cuh", "tr_df.cuh", "tr_internal.cuh"):
         h.update(open(os.path.join(ROOT, "paper_2607_13500_gb300", "csrc", f), "rb").read())
     return h.hexdigest()[:16]
 
@@ -246,7 +266,7 @@ def run_ours(args, world, rank, local):
 
     budget = BUDGETS[args.workload]
     over = {"batch": args.batch} if args.batch else {}
-    w = synth.make(args.workload, seed=args.seed + 1000 * rank, device=dev, **over)
+    w = synth.make(args.workload, seed=rank_seed(args.seed, rank), device=dev, **over)
     red = altr.Reducer(w.seqlens, w.d, w.x.dtype, dev, **budget)
     e = 2 if w.x.dtype == torch.bfloat16 else 4
     total_rows = w.total
@@ -278,13 +298,9 @@ def run_ours(args, world, rank, local):
     t_score = [ev[0].elapsed_time(ev[1]) for ev in evs]
     t_select = [ev[1].elapsed_time(ev[2]) for ev in evs]
     t_gather = [ev[2].elapsed_time(ev[3]) for ev in evs]
-    ms_step = total_ms / args.steps
-    if world > 1:
-        t = torch.tensor([ms_step], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms_step = float(t.item())
+    ms_step = max_over_ranks(total_ms / args.steps, world, dev)
     images = w.batch * world
-    value = images / (ms_step * 1e-3)
+    value = job_images_per_s(w.batch, world, ms_step)
 
     # end to end through the public API: pinned host inputs in, y and idx out
     pin = lambda t: t.cpu().pin_memory()
@@ -301,11 +317,7 @@ def run_ours(args, world, rank, local):
     for _ in range(e2e_steps):
         red.run_host(x_h, p_h, q_h, dev_in, y_h, idx_h)
         torch.cuda.synchronize()
-    e2e_s = (time.perf_counter() - t0) / e2e_steps
-    if world > 1:
-        t = torch.tensor([e2e_s], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        e2e_s = float(t.item())
+    e2e_s = max_over_ranks((time.perf_counter() - t0) / e2e_steps, world, dev)
     del dev_in
 
     peak, peak_kind = _peaks()

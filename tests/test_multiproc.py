@@ -1,0 +1,55 @@
+"""The multi-GPU host logic of bench.py on CPU: two gloo ranks, each with its
+own batch, the max over ranks and the whole-job aggregate.  The reduction
+itself has no collective (images are independent), so nothing else is
+exchanged between ranks."""
+import os
+import socket
+
+import pytest
+import torch
+import torch.distributed as dist
+import torch.multiprocessing as mp
+
+import bench
+import synth
+
+
+def _free_port():
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _worker(rank, world, port, out):
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank), WORLD_SIZE=str(world))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        w = synth.make("llava576", seed=bench.rank_seed(0, rank), batch=2, n=16, d=64)
+        local_ms = 1.0 + rank  # rank 1 is the slow one
+        ms = bench.max_over_ranks(local_ms, world)
+        value = bench.job_images_per_s(w.batch, world, ms)
+        first = w.x[0, :4].float()
+        gathered = [torch.zeros(4) for _ in range(world)]
+        dist.all_gather(gathered, first)
+        out[rank] = (ms, value, [g.tolist() for g in gathered])
+    finally:
+        dist.destroy_process_group()
+
+
+@pytest.mark.timeout(120)
+def test_two_gloo_ranks_max_and_aggregate():
+    world = 2
+    port = _free_port()
+    mgr = mp.Manager()
+    out = mgr.dict()
+    mp.spawn(_worker, args=(world, port, out), nprocs=world, join=True)
+    ms0, v0, g0 = out[0]
+    ms1, v1, g1 = out[1]
+    assert ms0 == ms1 == 2.0                      # the slowest rank's step time
+    assert v0 == v1 == pytest.approx(2 * 2 / 2e-3)  # all ranks' images / that time
+    assert g0[0] != g0[1]                          # each rank drew its own batch
+
+
+def test_single_rank_is_identity():
+    assert bench.max_over_ranks(3.5, 1) == 3.5
+    assert bench.job_images_per_s(64, 1, 0.25) == pytest.approx(256000.0)
