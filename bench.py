@@ -3,7 +3,8 @@
 
 One step = one pass of the whole path (per-token scores, per-image top-K1,
 sort of the rest by the consistency signal, stride pick, gather) over one
-batch of synthetic images already resident in HBM.  Prints one JSON line.
+batch of synthetic images already resident in HBM: two kernels, k_score and
+k_select_gather, timed with CUDA events around each.  Prints one JSON line.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload NAME]
 
@@ -283,7 +284,7 @@ def run_ours(args, world, rank, local):
     torch.cuda.synchronize()
     st = red.status.cpu().tolist()
     # timed region: K steps, per-kernel events inside every step
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier()
     torch.cuda.synchronize()
@@ -297,7 +298,6 @@ def run_ours(args, world, rank, local):
     total_ms = start.elapsed_time(end)
     t_score = [ev[0].elapsed_time(ev[1]) for ev in evs]
     t_select = [ev[1].elapsed_time(ev[2]) for ev in evs]
-    t_gather = [ev[2].elapsed_time(ev[3]) for ev in evs]
     ms_step = max_over_ranks(total_ms / args.steps, world, dev)
     images = w.batch * world
     value = job_images_per_s(w.batch, world, ms_step)
@@ -337,12 +337,11 @@ def run_ours(args, world, rank, local):
         "config": {**_workload_config(w, budget, args), "parallelism": f"replicas x{world} (images sharded)",
                    "l2": f"inputs {in_bytes / 2**20:.0f} MiB > L2 {L2_BYTES // 2**20} MiB, no flush"},
         "hbm_gbs": path_gbs, "frac_of_8tbs": path_gbs / NOMINAL_HBM_GBS, "frac_of_measured": path_gbs / peak,
-        "kernels_ms": {"k_score": score_ms, "k_select": statistics.mean(t_select),
-                       "k_gather": statistics.mean(t_gather)},
+        "kernels_ms": {"k_score": score_ms, "k_select_gather": statistics.mean(t_select)},
         "roofline": roofline,
         "e2e": {"value": images / e2e_s, "unit": "images/s", "h2d_bytes_per_step": in_bytes,
                 "d2h_bytes_per_step": red.total_k * (w.d * e + 4)},
-        "gpu_launches": 3 * args.steps,
+        "gpu_launches": 2 * args.steps,
         "clocks": clk,
         "status": st,
     }

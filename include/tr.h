@@ -158,8 +158,22 @@ tr_status tr_gather(const tr_tokens *in, const int32_t *d_cu_k, const int32_t *i
                     void *stream);
 
 /*
- * The whole path in one call: tr_score, tr_select and tr_gather on `stream`
- * (three kernel launches), with the statistics kept in the workspace.
+ * Selection and gather in one launch, from the statistics of tr_score: the
+ * result of tr_select (idx, optional H2 / s fix-ups, status) plus the kept
+ * rows y as tr_gather would copy them.  When there are fewer images than
+ * SMs, each image's selection is run by several CTAs at once and each copies
+ * its share of the kept rows (the selection is deterministic, so all reach
+ * the same indices; only one writes idx and the status words).
+ *   total_k:  host int, = cu_k[batch]; y: device [total_k, d], 16-byte aligned.
+ *   Other arguments as in tr_select (role is not produced).
+ */
+tr_status tr_select_gather(const tr_tokens *in, const float *stats, const int32_t *d_k, const int32_t *d_k1,
+                           const int32_t *d_cu_k, int32_t total_k, void *y, int32_t *idx, float *h2, float *s,
+                           void *ws, size_t ws_bytes, int32_t *d_status, void *stream);
+
+/*
+ * The whole path in one call: tr_score then tr_select_gather on `stream`
+ * (two kernel launches), with the statistics kept in the workspace.
  *   total_k:  host int, = cu_k[batch] (the number of output rows).
  *   y:        device [total_k, d] in the input dtype, 16-byte aligned.
  *   idx, h2, s, d_status: as in tr_select (role is not produced); h2 and s

@@ -62,6 +62,8 @@ def load() -> ctypes.CDLL:
     lib.tr_select.argtypes = [tok, VP, VP, VP, VP, VP, VP, VP, VP, VP, SZ, VP, VP]
     lib.tr_select.restype = I32
     lib.tr_gather.argtypes, lib.tr_gather.restype = [tok, VP, VP, I32, VP, VP], I32
+    lib.tr_select_gather.argtypes = [tok, VP, VP, VP, VP, I32, VP, VP, VP, VP, VP, SZ, VP, VP]
+    lib.tr_select_gather.restype = I32
     lib.tr_reduce.argtypes = [tok, VP, VP, VP, I32, VP, VP, VP, VP, VP, SZ, VP, VP]
     lib.tr_reduce.restype = I32
     _lib = lib

@@ -202,10 +202,10 @@ class Reducer:
                             self.status)
 
     def run_split(self, x, x_pre, x_post, events=None):
-        """The same three kernels as ``run`` through the three separate entry
-        points tr_score, tr_select and tr_gather, with ``events`` (four
-        torch.cuda.Event, or None) recorded before, between and after them on
-        the current stream, so each kernel can be timed inside a step."""
+        """The same two kernels as ``run`` through the entry points tr_score
+        and tr_select_gather, with ``events`` (three torch.cuda.Event, or
+        None) recorded before, between and after them on the current stream,
+        so that each kernel can be timed inside a step."""
         tok = self._bind(x, x_pre, x_post)
         st = _stream(self.device)
         lib = self.lib
@@ -215,14 +215,11 @@ class Reducer:
         check("tr_score", lib.tr_score(tok.ref(), _ptr(stats), _ptr(self.h2), _ptr(self.s), st))
         if events:
             events[1].record()
-        check("tr_select", lib.tr_select(tok.ref(), _ptr(stats), _ptr(self.d_k), _ptr(self.d_k1), _ptr(self.d_cu),
-                                         _ptr(self.idx), None, _ptr(self.h2), _ptr(self.s), _ptr(self._ws),
-                                         self._ws_bytes, _ptr(self.status), st))
+        check("tr_select_gather", lib.tr_select_gather(
+            tok.ref(), _ptr(stats), _ptr(self.d_k), _ptr(self.d_k1), _ptr(self.d_cu), self.total_k, _ptr(self.y),
+            _ptr(self.idx), _ptr(self.h2), _ptr(self.s), _ptr(self._ws), self._ws_bytes, _ptr(self.status), st))
         if events:
             events[2].record()
-        check("tr_gather", lib.tr_gather(tok.ref(), _ptr(self.d_cu), _ptr(self.idx), self.total_k, _ptr(self.y), st))
-        if events:
-            events[3].record()
         return ReduceResult(self.y[:self.total_k], self.idx[:self.total_k], self.cu_k, self.h2, self.s,
                             self.status)
 

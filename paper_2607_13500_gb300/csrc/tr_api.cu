@@ -1,5 +1,5 @@
 // Host side of the C ABI declared in include/tr.h: argument checks, budgets,
-// workspace carving and the launch sequence score -> select -> gather.
+// workspace carving and launches (tr_reduce: score, then select + gather).
 #include <climits>
 
 #include "tr_internal.cuh"
@@ -145,6 +145,21 @@ tr_status tr_select(const tr_tokens *in, const float *stats, const int32_t *d_k,
   return err == cudaSuccess ? TR_OK : TR_ERR_CUDA;
 }
 
+tr_status tr_select_gather(const tr_tokens *in, const float *stats, const int32_t *d_k, const int32_t *d_k1,
+                           const int32_t *d_cu_k, int32_t total_k, void *y, int32_t *idx, float *h2, float *s,
+                           void *ws, size_t ws_bytes, int32_t *d_status, void *stream) {
+  Shape sh;
+  tr_status rc = check_tokens(in, &sh);
+  if (rc != TR_OK) return rc;
+  if (total_k < 0 || total_k > sh.total) return TR_ERR_BUDGET;
+  if (in->batch > 0 && (!stats || !d_k || !d_k1 || !d_cu_k || !idx || (total_k > 0 && !y))) return TR_ERR_ARG;
+  if (misaligned(stats, 16) || misaligned(y, 16)) return TR_ERR_ALIGN;
+  if ((rc = check_ws(sh, ws, ws_bytes)) != TR_OK) return rc;
+  SelectArgs a = select_args(in, sh, stats, d_k, d_k1, d_cu_k, idx, nullptr, h2, s, ws, d_status);
+  cudaError_t err = launch_select_gather(a, y, static_cast<cudaStream_t>(stream));
+  return err == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+}
+
 tr_status tr_reduce(const tr_tokens *in, const int32_t *d_k, const int32_t *d_k1, const int32_t *d_cu_k,
                     int32_t total_k, void *y, int32_t *idx, float *h2, float *s, void *ws, size_t ws_bytes,
                     int32_t *d_status, void *stream) {
@@ -155,18 +170,10 @@ tr_status tr_reduce(const tr_tokens *in, const int32_t *d_k, const int32_t *d_k1
   if (in->batch > 0 && (!d_k || !d_k1 || !d_cu_k || !idx || (total_k > 0 && !y))) return TR_ERR_ARG;
   if (misaligned(y, 16)) return TR_ERR_ALIGN;
   if ((rc = check_ws(sh, ws, ws_bytes)) != TR_OK) return rc;
-  const WsLayout lay = ws_layout(sh.total);
-  char *w = static_cast<char *>(ws);
-  float *stats = reinterpret_cast<float *>(w + lay.stats);
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
-  cudaError_t err = launch_score(in->x, in->x_pre, in->x_post, in->dtype, in->d, sh.total, stats, h2, s, st);
-  if (err != cudaSuccess) return TR_ERR_CUDA;
-  SelectArgs a = select_args(in, sh, stats, d_k, d_k1, d_cu_k, idx, nullptr, h2, s, ws, d_status);
-  err = launch_select(a, st);
-  if (err != cudaSuccess) return TR_ERR_CUDA;
-  err = launch_gather(in->x, sh.total, in->dtype, in->d, in->batch, in->cu_seqlens ? 0 : in->n, in->cu_seqlens,
-                      d_cu_k, idx, total_k, y, st);
-  return err == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+  float *stats = reinterpret_cast<float *>(static_cast<char *>(ws) + ws_layout(sh.total).stats);
+  rc = tr_score(in, stats, h2, s, stream);
+  if (rc != TR_OK) return rc;
+  return tr_select_gather(in, stats, d_k, d_k1, d_cu_k, total_k, y, idx, h2, s, ws, ws_bytes, d_status, stream);
 }
 
 tr_status tr_gather(const tr_tokens *in, const int32_t *d_cu_k, const int32_t *idx, int32_t total_k, void *y,

@@ -1,5 +1,11 @@
-// The selection kernel: one CTA per image runs select_image (Algorithm 1,
+// The selection kernels: one CTA per image runs select_image (Algorithm 1,
 // see tr_select_dev.cuh) on statistics left by the scoring kernel.
+//
+// k_select_gather (tr_reduce) also copies the kept rows.  With fewer images
+// than SMs it runs R replica CTAs per image: each makes the same
+// deterministic selection (only replica 0 writes idx and the status words)
+// and copies its 1/R share of the image's kept rows, so the copies of one
+// image overlap the selections of the others on SMs that would be idle.
 #include "tr_select_dev.cuh"
 
 namespace tr {
@@ -10,7 +16,58 @@ __global__ void __launch_bounds__(kSelectThreads, 1) k_select(const SelectArgs a
   select_image(a, blockIdx.x, smem);
 }
 
-int g_smem_set[64];  // per device: dynamic shared memory limit already raised
+__device__ __forceinline__ uint4 ld_nc16(const uint4 *p) {
+  uint4 r;
+  asm("ld.global.nc.L1::no_allocate.v4.u32 {%0, %1, %2, %3}, [%4];"
+      : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+      : "l"(p));
+  return r;
+}
+
+__global__ void __launch_bounds__(kSelectThreads, 1)
+    k_select_gather(const SelectArgs a, const int replicas, const int nchunks, uint4 *__restrict__ y) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  const int b = blockIdx.x / replicas, r = blockIdx.x % replicas;
+  select_image(a, b, smem, r == 0);
+  long long off;
+  int n;
+  if (a.cu_seqlens) {
+    off = a.cu_seqlens[b];
+    n = a.cu_seqlens[b + 1] - a.cu_seqlens[b];
+  } else {
+    off = (long long)b * a.n_uniform;
+    n = a.n_uniform;
+  }
+  const int k = a.k[b], k1 = a.k1[b], ko = a.cu_k[b];
+  if (n <= 0 || n > a.max_n || k < 0 || k > n || k1 < 0 || k1 > k) return;  // counted by select_image
+  // this replica's share of the image's kept rows
+  const uint16_t *kept = kept_rows(a, smem);
+  const int j0 = (int)((long long)r * k / replicas), j1 = (int)((long long)(r + 1) * k / replicas);
+  const uint4 *x = static_cast<const uint4 *>(a.x);
+  // one warp per row, eight 16-byte loads in flight per lane, streaming stores
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  constexpr int kU = 8;
+  for (int j = j0 + warp; j < j1; j += kWarps) {
+    const uint4 *src = x + (off + kept[j]) * nchunks;
+    uint4 *dst = y + (long long)(ko + j) * nchunks;
+    for (int c0 = lane; c0 < nchunks; c0 += 32 * kU) {
+      uint4 v[kU];
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int c = c0 + 32 * u;
+        if (c < nchunks) v[u] = ld_nc16(src + c);
+      }
+#pragma unroll
+      for (int u = 0; u < kU; ++u) {
+        const int c = c0 + 32 * u;
+        if (c < nchunks) __stcs(dst + c, v[u]);
+      }
+    }
+  }
+}
+
+int g_smem_set[64];  // per device: dynamic shared memory limit already raised (bit 0 k_select, bit 1 k_select_gather)
+int g_sms[64];
 
 }  // namespace
 
@@ -19,24 +76,47 @@ size_t select_smem_bytes(int max_n) {
   return cap * (sizeof(uint32_t) + 2 * sizeof(uint16_t) + sizeof(uint8_t)) + kWarps * 256 * sizeof(uint32_t);
 }
 
+template <typename K>
+cudaError_t raise_smem_limit(K kernel, int dev) {
+  int optin = 0;
+  cudaError_t err = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+  if (err != cudaSuccess) return err;
+  cudaFuncAttributes fa;
+  err = cudaFuncGetAttributes(&fa, kernel);
+  if (err != cudaSuccess) return err;
+  return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, optin - (int)fa.sharedSizeBytes);
+}
+
 cudaError_t launch_select(const SelectArgs &a, cudaStream_t st) {
   if (a.batch == 0) return cudaSuccess;
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
   const size_t smem = select_smem_bytes(a.max_n);
-  if (!g_smem_set[dev & 63]) {
-    int optin = 0;
-    err = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-    if (err != cudaSuccess) return err;
-    cudaFuncAttributes fa;
-    err = cudaFuncGetAttributes(&fa, k_select);
-    if (err != cudaSuccess) return err;
-    err = cudaFuncSetAttribute(k_select, cudaFuncAttributeMaxDynamicSharedMemorySize, optin - (int)fa.sharedSizeBytes);
-    if (err != cudaSuccess) return err;
-    g_smem_set[dev & 63] = 1;
+  if (!(g_smem_set[dev & 63] & 1)) {
+    if ((err = raise_smem_limit(k_select, dev)) != cudaSuccess) return err;
+    g_smem_set[dev & 63] |= 1;
   }
   k_select<<<a.batch, kSelectThreads, smem, st>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_select_gather(const SelectArgs &a, void *y, cudaStream_t st) {
+  if (a.batch == 0) return cudaSuccess;
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err != cudaSuccess) return err;
+  if (!(g_smem_set[dev & 63] & 2)) {
+    if ((err = raise_smem_limit(k_select_gather, dev)) != cudaSuccess) return err;
+    int sms = 0;
+    if ((err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return err;
+    g_sms[dev & 63] = sms;
+    g_smem_set[dev & 63] |= 2;
+  }
+  const int replicas = max(1, min(16, g_sms[dev & 63] / a.batch));
+  const size_t smem = select_smem_bytes(a.max_n);
+  const int nchunks = a.d * elem_bytes(a.dtype) / 16;
+  k_select_gather<<<a.batch * replicas, kSelectThreads, smem, st>>>(a, replicas, nchunks, static_cast<uint4 *>(y));
   return cudaGetLastError();
 }
 

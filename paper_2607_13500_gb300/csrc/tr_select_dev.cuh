@@ -424,12 +424,31 @@ __device__ __forceinline__ __int128 part_sum(const Part128 &p, int which) {
   return v;
 }
 
-// Exact sums of one row computed by the whole CTA (one 16-byte chunk of each
-// stream per thread and pass), in three 128-bit windows; false (uniformly)
-// when a term does not fit its window.
+// A group of warps that works on one row: threads [first, first + size) of
+// the CTA, synchronised by named barrier `bar` (1..15; 0 is __syncthreads).
+struct Group {
+  int first, size, bar;
+  __device__ __forceinline__ int tid() const { return (int)threadIdx.x - first; }
+  __device__ __forceinline__ void sync() const {
+    asm volatile("bar.sync %0, %1;" ::"r"(bar), "r"(size) : "memory");
+  }
+  __device__ __forceinline__ bool all(bool v) const {
+    unsigned r;
+    asm volatile(
+        "{\n .reg .pred p, q;\n setp.ne.u32 p, %1, 0;\n bar.red.and.pred q, %2, %3, p;\n selp.u32 %0, 1, 0, q;\n}"
+        : "=r"(r)
+        : "r"((unsigned)v), "r"(bar), "r"(size)
+        : "memory");
+    return r != 0;
+  }
+};
+
+// Exact sums of one row computed by a group of warps (each thread takes
+// 16-byte chunks t, t + size, ...), in three 128-bit windows; false
+// (uniformly across the group) when a term does not fit its window.
 template <bool kBf16>
 __device__ bool exact_row_block(const SelectArgs &a, long long row, int mode, const float *st, ExactRec *rec,
-                                Part128 &part) {
+                                Part128 &part, const Group &g) {
   constexpr int kPer = kBf16 ? 8 : 4;  // elements per 16-byte chunk
   const int nchunks = a.d / kPer;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -442,7 +461,7 @@ __device__ bool exact_row_block(const SelectArgs &a, long long row, int mode, co
     b1 = window_bottom(__ldcg(st + 1));
     const uint4 *px = static_cast<const uint4 *>(a.x) + row * nchunks;
 #pragma unroll 4
-    for (int c = threadIdx.x; c < nchunks; c += blockDim.x) {
+    for (int c = g.tid(); c < nchunks; c += g.size) {
       unpack<kBf16>(__ldg(px + c), e0);
 #pragma unroll
       for (int i = 0; i < kPer; ++i) {
@@ -464,7 +483,7 @@ __device__ bool exact_row_block(const SelectArgs &a, long long row, int mode, co
     const uint4 *pp = static_cast<const uint4 *>(a.x_pre ? a.x_pre : a.x) + row * nchunks;
     const uint4 *pq = static_cast<const uint4 *>(a.x_post) + row * nchunks;
 #pragma unroll 4
-    for (int c = threadIdx.x; c < nchunks; c += blockDim.x) {
+    for (int c = g.tid(); c < nchunks; c += g.size) {
       unpack<kBf16>(__ldg(pp + c), e0);
       unpack<kBf16>(__ldg(pq + c), e1);
 #pragma unroll
@@ -487,7 +506,7 @@ __device__ bool exact_row_block(const SelectArgs &a, long long row, int mode, co
       }
     }
   }
-  if (!__syncthreads_and(fits)) return false;
+  if (!g.all(fits)) return false;
   s0 = warp_sum128(s0);
   s1 = warp_sum128(s1);
   s2 = warp_sum128(s2);
@@ -496,71 +515,89 @@ __device__ bool exact_row_block(const SelectArgs &a, long long row, int mode, co
     part_put(part, warp * 3 + 1, s1);
     part_put(part, warp * 3 + 2, s2);
   }
-  __syncthreads();
-  if (threadIdx.x == 0) {
+  g.sync();
+  // lanes 0..2 of the group's first warp reduce one sum each over the group's warps
+  const int w0 = g.first >> 5, nw = g.size >> 5;
+  if (g.tid() < 3) {
+    const int which = g.tid();
+    __int128 v = 0;
+    for (int w = w0; w < w0 + nw; ++w)
+      v += (__int128)(((unsigned __int128)part.hi[w * 3 + which] << 64) | part.lo[w * 3 + which]);
     if (mode == 0) {
-      int128_to_big(part_sum(part, 0), b0, rec->l1);
-      int128_to_big(part_sum(part, 1), b1, rec->s2);
-      rec->flags_l = 0u;
+      if (which == 0) int128_to_big(v, b0, rec->l1);
+      if (which == 1) int128_to_big(v, b1, rec->s2);
+      if (which == 0) rec->flags_l = 0u;
     } else {
-      int128_to_big(part_sum(part, 0), b0, rec->a);
-      int128_to_big(part_sum(part, 1), b1, rec->b);
-      int128_to_big(part_sum(part, 2), b2, rec->p);
-      rec->flags_s = 0u;
+      if (which == 0) int128_to_big(v, b0, rec->a);
+      if (which == 1) int128_to_big(v, b1, rec->b);
+      if (which == 2) int128_to_big(v, b2, rec->p);
+      if (which == 0) rec->flags_s = 0u;
     }
   }
-  __syncthreads();
+  g.sync();
   return true;
 }
 
-// Exact sums of one row by the whole CTA: the 128-bit windows when the row's
-// fp32 sums are trustworthy and its terms fit, else warp 0 runs the digit
-// accumulator (non-finite or extreme rows).
+// Exact sums of one row by a group: the 128-bit windows when the row's fp32
+// sums are trustworthy and its terms fit, else the group's first warp runs
+// the digit accumulator (non-finite or extreme rows).
 __device__ __forceinline__ void exact_row_any(const SelectArgs &a, long long row, int mode, const float *st,
-                                              ExactRec *rec, Part128 &part) {
+                                              ExactRec *rec, Part128 &part, const Group &g) {
   const bool trusted = mode == 0 ? !isnan(key_r(st)) : !isnan(key_s(st));
   bool ok = false;
   if (trusted)
-    ok = a.dtype == TR_BF16 ? exact_row_block<true>(a, row, mode, st, rec, part)
-                            : exact_row_block<false>(a, row, mode, st, rec, part);
+    ok = a.dtype == TR_BF16 ? exact_row_block<true>(a, row, mode, st, rec, part, g)
+                            : exact_row_block<false>(a, row, mode, st, rec, part, g);
   if (!ok) {
-    if ((threadIdx.x >> 5) == 0) exact_row(a, row, mode, rec, threadIdx.x & 31);
-    __syncthreads();
+    if (g.tid() < 32) exact_row(a, row, mode, rec, threadIdx.x & 31);
+    g.sync();
   }
 }
 
-// Recomputes, one row at a time with the whole CTA, the rows whose flags
-// request it; clears the request and records what is now exact.  A single
-// block-wide vote skips the scan when nothing is pending.
-__device__ void refine_pending(const SelectArgs &a, long long off, int n, uint8_t *fl, ExactRec *rec) {
-  __shared__ unsigned wmask[kWarps];
+// Recomputes the rows whose flags request it and records what is now exact.
+// The pending rows are listed first (a block-wide vote skips everything when
+// none is); then up to four rows at a time are handled by groups of warps.
+constexpr int kPendCap = 512;
+__device__ void refine_pending(const SelectArgs &a, long long off, int n, uint8_t *fl, ExactRec *rec,
+                               const bool primary) {
   __shared__ Part128 part;
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  __shared__ int plist[kPendCap];
+  __shared__ int pcount;
   bool any = false;
   for (int i = threadIdx.x; i < n; i += blockDim.x) any |= (fl[i] & (F_NEEDL | F_NEEDS)) != 0;
   if (!__syncthreads_or(any)) return;
-  for (int base = 0; base < n; base += blockDim.x) {
-    const int i = base + threadIdx.x;
-    const unsigned m = __ballot_sync(0xffffffffu, i < n && (fl[i] & (F_NEEDL | F_NEEDS)) != 0);
-    if (lane == 0) wmask[warp] = m;
+  for (;;) {
+    if (threadIdx.x == 0) pcount = 0;
     __syncthreads();
-    for (int w = 0; w < kWarps; ++w) {
-      unsigned mm = wmask[w];
-      while (mm) {
-        const int r = __ffs(mm) - 1;
-        mm &= mm - 1;
-        const int row = base + 32 * w + r;
-        const uint8_t fr = fl[row];
-        const float *st = a.stats + (off + row) * TR_STATS_WORDS;
-        if (fr & F_NEEDL) exact_row_any(a, off + row, 0, st, rec + row, part);
-        if (fr & F_NEEDS) exact_row_any(a, off + row, 1, st, rec + row, part);
-        if (threadIdx.x == 0) {
-          fl[row] = (uint8_t)((fr & ~(F_NEEDL | F_NEEDS)) | ((fr & F_NEEDL) ? F_XL : 0) | ((fr & F_NEEDS) ? F_XS : 0));
-          if (a.status) atomicAdd(&a.status[2], 1);
-        }
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+      if (fl[i] & (F_NEEDL | F_NEEDS)) {
+        const int slot = atomicAdd(&pcount, 1);
+        if (slot < kPendCap) plist[slot] = i;
       }
     }
     __syncthreads();
+    const int total = pcount;
+    if (total == 0) break;
+    const int cnt = min(total, kPendCap);
+    const int groups = cnt >= 4 ? 4 : (cnt >= 2 ? 2 : 1);
+    const int gsize = (int)blockDim.x / groups;
+    const int gi = (int)threadIdx.x / gsize;
+    const Group g{gi * gsize, gsize, 1 + gi};
+    for (int base = 0; base < cnt; base += groups) {
+      if (base + gi < cnt) {
+        const int row = plist[base + gi];
+        const uint8_t fr = fl[row];
+        const float *st = a.stats + (off + row) * TR_STATS_WORDS;
+        if (fr & F_NEEDL) exact_row_any(a, off + row, 0, st, rec + row, part, g);
+        if (fr & F_NEEDS) exact_row_any(a, off + row, 1, st, rec + row, part, g);
+        if (g.tid() == 0) {
+          fl[row] = (uint8_t)((fr & ~(F_NEEDL | F_NEEDS)) | ((fr & F_NEEDL) ? F_XL : 0) | ((fr & F_NEEDS) ? F_XS : 0));
+          if (a.status && primary) atomicAdd(&a.status[2], 1);
+        }
+      }
+      __syncthreads();
+    }
+    if (total <= kPendCap) break;  // otherwise list the rows still pending
   }
 }
 
@@ -794,13 +831,188 @@ __device__ uint16_t *radix_sort(const uint32_t *key, uint16_t *a, uint16_t *b, i
   return a;
 }
 
+// Ascending bitonic sort of kSelectThreads * E composite keys (sort key << 16
+// | row) held E per thread (thread t owns positions t E .. t E + E - 1).
+// Partners closer than E are in the same thread, closer than 32 E in the
+// same warp (register shuffles); only the remaining stages go through
+// shared memory (scratch: kSelectThreads * E words) with block barriers.
+template <int E>
+__device__ void bitonic_regs(unsigned long long (&v)[E], unsigned long long *scratch) {
+  constexpr int NP = kSelectThreads * E;
+  const int t = threadIdx.x, lane = t & 31;
+  for (int k = 2; k <= NP; k <<= 1) {
+    for (int j = k >> 1; j > 0; j >>= 1) {
+      if (j < E) {
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+          const int pe = e ^ j;
+          if (pe > e) {
+            const bool up = ((t * E + e) & k) == 0;
+            const unsigned long long x = v[e], y = v[pe];
+            if ((x > y) == up) {
+              v[e] = y;
+              v[pe] = x;
+            }
+          }
+        }
+      } else if (j < 32 * E) {
+        const int lm = j / E;
+        const bool lower = (lane & lm) == 0;
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+          const unsigned long long o = __shfl_xor_sync(0xffffffffu, v[e], lm);
+          const bool up = ((t * E + e) & k) == 0;
+          v[e] = (lower == up) ? min(v[e], o) : max(v[e], o);
+        }
+      } else {
+#pragma unroll
+        for (int e = 0; e < E; ++e) scratch[t * E + e] = v[e];
+        __syncthreads();
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+          const int i = t * E + e, pi = i ^ j;
+          const unsigned long long o = scratch[pi];
+          const bool up = (i & k) == 0;
+          v[e] = ((i < pi) == up) ? min(v[e], o) : max(v[e], o);
+        }
+        __syncthreads();
+      }
+    }
+  }
+}
+
+template <int E>
+__device__ void sort_small(const uint32_t *key, uint16_t *a, int m, unsigned long long *scratch) {
+  unsigned long long v[E];
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const int i = threadIdx.x * E + e;
+    v[e] = i < m ? (((unsigned long long)key[a[i]] << 16) | a[i]) : ~0ull;
+  }
+  __syncthreads();  // every thread has read its rows of a before they are overwritten
+  bitonic_regs<E>(v, scratch);
+#pragma unroll
+  for (int e = 0; e < E; ++e) {
+    const int i = threadIdx.x * E + e;
+    if (i < m) a[i] = (uint16_t)(v[e] & 0xffffu);
+  }
+  __syncthreads();
+}
+
+// Ascending order of the m rows listed in a by (key[row], row), by value
+// buckets: the float each key encodes (v = value, or -value for importance
+// keys, which are stored complemented) is mapped linearly from [vmin, vmax]
+// onto nb buckets -- a monotone map, so concatenated buckets are in order --
+// rows are scattered into their bucket with shared-memory atomics, and each
+// bucket (about one row on the workloads here) is insertion-sorted by
+// (key, row).  Returns nullptr, having changed nothing, when some bucket
+// would hold more than kBucketMax rows (ties, or keys crowded together) or
+// the keys span no usable range: the caller falls back to the radix sort.
+// hist: at least nb words.
+constexpr int kBucketMax = 32;
+constexpr int kBuckets = 4096;
+__device__ __forceinline__ float key_value(uint32_t k, bool complemented) {
+  return complemented ? -unord32(~k) : unord32(k);
+}
+__device__ uint16_t *bucket_sort(const uint32_t *key, uint16_t *a, uint16_t *b, int m, uint32_t *hist,
+                                 bool complemented) {
+  __shared__ float sh_min[kWarps], sh_max[kWarps];
+  __shared__ int sh_big;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  float vmin = INFINITY, vmax = -INFINITY;
+  for (int q = tid; q < m; q += blockDim.x) {
+    const float v = key_value(key[a[q]], complemented);
+    vmin = fminf(vmin, v);
+    vmax = fmaxf(vmax, v);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    vmin = fminf(vmin, __shfl_xor_sync(0xffffffffu, vmin, o));
+    vmax = fmaxf(vmax, __shfl_xor_sync(0xffffffffu, vmax, o));
+  }
+  if (lane == 0) {
+    sh_min[warp] = vmin;
+    sh_max[warp] = vmax;
+  }
+  int nb = 64;
+  while (nb < m && nb < kBuckets) nb <<= 1;
+  for (int c = tid; c < nb; c += blockDim.x) hist[c] = 0u;
+  if (tid == 0) sh_big = 0;
+  __syncthreads();
+  vmin = sh_min[0];
+  vmax = sh_max[0];
+  for (int w = 1; w < kWarps; ++w) {
+    vmin = fminf(vmin, sh_min[w]);
+    vmax = fmaxf(vmax, sh_max[w]);
+  }
+  const float span = vmax - vmin;
+  const float scale = (float)nb / span;
+  if (!(span > 0.f) || !isfinite(span) || !isfinite(scale)) return nullptr;  // uniform: all equal or no usable range
+  // bucket of a value: floor((v - vmin) * scale), monotone in v, clamped to the last bucket
+  auto bucket = [&](float v) { return min(nb - 1, (int)((v - vmin) * scale)); };
+  for (int q = tid; q < m; q += blockDim.x) atomicAdd(&hist[bucket(key_value(key[a[q]], complemented))], 1u);
+  __syncthreads();
+  // exclusive scan of the bucket counts (each thread a contiguous stretch) and the largest count
+  const int per = (nb + blockDim.x - 1) / blockDim.x;
+  const int c0 = min(nb, tid * per), c1 = min(nb, c0 + per);
+  int run = 0, big = 0;
+  for (int c = c0; c < c1; ++c) {
+    run += (int)hist[c];
+    big = max(big, (int)hist[c]);
+  }
+  if (big > kBucketMax) sh_big = 1;
+  int total = 0;
+  int base = block_exclusive_scan(run, &total);
+  if (sh_big) return nullptr;  // uniform: written before the scan's barriers
+  for (int c = c0; c < c1; ++c) {
+    const int cnt = (int)hist[c];
+    hist[c] = (uint32_t)base;
+    base += cnt;
+  }
+  __syncthreads();
+  for (int q = tid; q < m; q += blockDim.x) {
+    const uint16_t row = a[q];
+    b[atomicAdd(&hist[bucket(key_value(key[row], complemented))], 1u)] = row;
+  }
+  __syncthreads();
+  // hist[c] is now the end of bucket c, so bucket c spans [hist[c - 1], hist[c])
+  for (int c = tid; c < nb; c += blockDim.x) {
+    const int lo = c ? (int)hist[c - 1] : 0, hi = (int)hist[c];
+    for (int i = lo + 1; i < hi; ++i) {
+      const uint16_t row = b[i];
+      const unsigned long long kk = ((unsigned long long)key[row] << 16) | row;
+      int j = i - 1;
+      while (j >= lo && (((unsigned long long)key[b[j]] << 16) | b[j]) > kk) {
+        b[j + 1] = b[j];
+        --j;
+      }
+      b[j + 1] = row;
+    }
+  }
+  __syncthreads();
+  return b;
+}
+
+// Ascending order of the m rows listed in a by (key[row], row), a listed in
+// ascending row order: value buckets, or the stable radix sort when the keys
+// crowd into few buckets.  Returns the buffer holding the order.
+__device__ uint16_t *sort_rows(const uint32_t *key, uint16_t *a, uint16_t *b, int m, uint32_t *hist,
+                               bool complemented) {
+  if (m < 2) return a;
+  if (uint16_t *o = bucket_sort(key, a, b, m, hist, complemented)) return o;
+  return radix_sort(key, a, b, m, hist);
+}
+
 __host__ __device__ inline int row_capacity(int max_n) { return (max_n + 15) / 16 * 16; }
 
 // ---------------------------------------------------------------- one image
 // Algorithm 1 for image b, by the whole CTA (kSelectThreads threads);
 // smem holds select_smem_bytes(a.max_n) bytes.  Reads the statistics through
-// L2 so that rows scored by other CTAs of the same launch are seen.
-__device__ void select_image(const SelectArgs &a, const int b, unsigned char *smem) {
+// L2 so that rows scored by other CTAs of the same launch are seen.  Leaves
+// the K kept local indices, ascending, in the second order buffer of smem
+// (kept_rows); only a primary CTA writes idx, role, H2/s and the status words
+// (replicas that run the same deterministic selection write nothing).
+__device__ void select_image(const SelectArgs &a, const int b, unsigned char *smem, const bool primary = true) {
   __shared__ int sh_lo, sh_hi;
   const int tid = threadIdx.x, nthr = blockDim.x;
   long long off;
@@ -814,7 +1026,7 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
   }
   const int k = a.k[b], k1 = a.k1[b], k2 = k - k1, ko = a.cu_k[b];
   if (n < 0 || n > a.max_n || k < 0 || k > n || k1 < 0 || k1 > k) {
-    if (tid == 0 && a.status) atomicAdd(&a.status[3], 1);
+    if (tid == 0 && a.status && primary) atomicAdd(&a.status[3], 1);
     return;
   }
   if (n == 0) return;
@@ -839,7 +1051,7 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
     fl[i] = f;
   }
   __syncthreads();
-  refine_pending(a, off, n, fl, rec);
+  refine_pending(a, off, n, fl, rec, primary);
   __syncthreads();
 
   // 2. Stage I: top-K1 by R (equivalently H2), descending, lower index first.
@@ -850,7 +1062,7 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
       ia[i] = (uint16_t)i;
     }
     __syncthreads();
-    const uint16_t *ord = radix_sort(key, ia, ib, n, hist);
+    const uint16_t *ord = sort_rows(key, ia, ib, n, hist, true);
     if (tid == 0) {
       int lo = k1, hi = k1;
       if (!cert_r(key, ord, k1, a.bounds)) {
@@ -871,7 +1083,7 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
         if (!(fl[r] & F_XL)) fl[r] |= F_NEEDL;
       }
       __syncthreads();
-      refine_pending(a, off, n, fl, rec);
+      refine_pending(a, off, n, fl, rec, primary);
       __syncthreads();
       for (int q = lo + tid; q < hi; q += nthr) {
         const int r = ord[q];
@@ -912,7 +1124,7 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
       key[i] = ord32(sv);
     }
     __syncthreads();
-    const uint16_t *ord = radix_sort(key, ia, ib, m, hist);
+    const uint16_t *ord = sort_rows(key, ia, ib, m, hist, false);
     const int t = max(1, m / k2);
     for (int j = tid; j < k2; j += nthr) {
       const int p = j * t;
@@ -933,7 +1145,7 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
       }
     }
     __syncthreads();
-    refine_pending(a, off, n, fl, rec);
+    refine_pending(a, off, n, fl, rec, primary);
     __syncthreads();
     for (int q = tid; q < m; q += nthr) {
       const int r = ord[q];
@@ -970,9 +1182,11 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
   for (int i = i0; i < i1; ++i) {
     const uint8_t f = fl[i];
     if ((f & (F_IMP | F_DIV)) && pos < ko + k) {  // never write past this image's slots
-      a.idx[pos] = i;
+      if (primary) a.idx[pos] = i;
+      ia[pos - ko] = (uint16_t)i;
       ++pos;
     }
+    if (!primary) continue;
     if (a.role) a.role[off + i] = (f & F_IMP) ? 1 : ((f & F_DIV) ? 2 : 0);
     int nonfinite = 0, overflow = 0;
     if (f & F_XL) {
@@ -994,7 +1208,13 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
       if (overflow) atomicAdd(&a.status[1], 1);
     }
   }
-  if (tid == 0 && kept_total != k && a.status) atomicAdd(&a.status[3], 1);
+  if (tid == 0 && kept_total != k && a.status && primary) atomicAdd(&a.status[3], 1);
+  __syncthreads();
+}
+
+// Where select_image leaves the kept local indices.
+__device__ __forceinline__ const uint16_t *kept_rows(const SelectArgs &a, unsigned char *smem) {
+  return reinterpret_cast<const uint16_t *>(reinterpret_cast<uint32_t *>(smem) + row_capacity(a.max_n));
 }
 
 }  // namespace

@@ -17,7 +17,7 @@ def lib():
 
 def test_exports_every_declared_function(lib):
     names = _lib.declared_functions()
-    assert {"tr_budgets", "tr_score", "tr_select", "tr_gather", "tr_reduce", "tr_workspace_bytes",
+    assert {"tr_budgets", "tr_score", "tr_select", "tr_gather", "tr_select_gather", "tr_reduce", "tr_workspace_bytes",
             "tr_status_string", "tr_version"} <= set(names)
     for name in names:
         assert hasattr(lib, name), name

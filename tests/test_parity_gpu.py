@@ -121,6 +121,18 @@ def test_score_and_select_entry_points():
         assert set(np.nonzero(role[sl] == 1)[0].tolist()) == set(ref["imp"].tolist())
         assert set(np.nonzero(role[sl] == 2)[0].tolist()) == set(ref["div"].tolist())
         assert np.array_equal(idx[cu[b]:cu[b + 1]].cpu().numpy(), ref["kept"])
+    # tr_gather on the selection reproduces the rows tr_reduce gathers
+    from paper_2607_13500_gb300 import _lib
+    from paper_2607_13500_gb300.api import _Tokens, _ptr, _stream
+    tok = _Tokens(w.x, w.x_pre, w.x_post, w.seqlens)
+    y = torch.empty(cu[-1], w.d, dtype=w.x.dtype, device=w.x.device)
+    d_cu = torch.tensor(cu, dtype=torch.int32, device=w.x.device)
+    _lib.check("tr_gather", _lib.load().tr_gather(tok.ref(), _ptr(d_cu), _ptr(idx), cu[-1], _ptr(y),
+                                                  _stream(w.x.device)))
+    ref = altr.reduce(w.x, w.x_pre, w.x_post, seqlens=w.seqlens, budget=(ks, k1s, cu))
+    torch.cuda.synchronize()
+    assert torch.equal(y.view(torch.int16), ref.y.view(torch.int16))
+    assert torch.equal(idx, ref.idx)
     st = stats.cpu().numpy().astype(np.float64)
     xx = _f64(w.x)
     assert np.allclose(st[:, 0], np.abs(xx).sum(1), rtol=2e-6)
