@@ -12,7 +12,8 @@ namespace tr {
 
 // ---------------------------------------------------------------- launch shapes
 constexpr int kScoreWarps = 8;        // rows (one per warp) in flight per score CTA
-constexpr int kScoreBatch = 4;        // 16-byte chunks a lane loads per stream before it computes
+constexpr int kScoreBatchBf16 = 8;    // 16-byte chunks a lane loads per stream before it computes (bf16)
+constexpr int kScoreBatchF32 = 4;     // the same for fp32 inputs
 constexpr int kSelectThreads = 512;   // one select CTA per image
 constexpr int kGatherWarps = 8;
 
@@ -47,8 +48,10 @@ static_assert(sizeof(ExactRec) % 16 == 0, "ExactRec records keep 16-byte alignme
 // Rounding depth of the sums L1, S2, A, B in the score kernel: each term goes
 // through the depth-3 (bf16) or depth-2 (fp32, plus the rounding of the square
 // itself) tree of its 16-byte chunk; the chunk partials are accumulated
-// error-free into a double-float whose low part's own rounding is bounded
-// separately, and the keys are computed from the unrounded double-float.
+// error-free into double-floats (two per lane for bf16: even and odd chunks)
+// whose low parts' own rounding is bounded separately (at most lane_chunks
+// + 12 low-part additions on any path, folds and warp merges included), and
+// the keys are computed from the unrounded double-float.
 __host__ __device__ inline int elem_bytes(int dtype) { return dtype == TR_BF16 ? 2 : 4; }
 
 __host__ __device__ inline int score_depth(int d, int dtype) {

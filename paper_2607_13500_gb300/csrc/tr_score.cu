@@ -1,15 +1,5 @@
-// Scoring pass: per-token sums for the Renyi-2 entropy (Eq. 3-4) and the
-// consistency signal (Eq. 6) in one read of x, x', x''.
-//
-// One warp per row; lane l reads 16-byte chunks l, l+32, l+64, ... of each of
-// the three streams (fully coalesced 512-byte warp requests), kScoreBatch
-// chunks per stream in flight before any arithmetic.  Each chunk's partial
-// sums of |x|, x^2, x'^2, x''^2 come from a depth-3 fp32 tree; the partials
-// are accumulated error-free as double-floats (TwoSum), so every sum carries
-// at most score_depth() roundings whatever D is.  P = x'.x'' is accumulated
-// error-free term by term, since the ordering by s needs it to far better
-// than fp32.  The epilogue rounds the sums to fp32 and derives the fp32
-// selection keys, all without fp64 (GB300's fp64 rate would stall the warp).
+// Scoring pass (Eq. 3-4 and Eq. 6): one warp per row over a grid of resident
+// CTAs; the row arithmetic is in tr_score_dev.cuh.
 #include "tr_score_dev.cuh"
 
 namespace tr {
@@ -56,14 +46,18 @@ cudaError_t launch_score(const void *x, const void *x_pre, const void *x_post, i
     info.sms = sms;
     info.blocks_per_sm[which] = bps > 0 ? bps : 1;
   }
+  const int row_bytes = d * elem_bytes(dtype);
+  const unsigned char *bx = static_cast<const unsigned char *>(x);
+  const unsigned char *bp = static_cast<const unsigned char *>(x_pre ? x_pre : x);
+  const unsigned char *bq = static_cast<const unsigned char *>(x_post);
+  float4 *ps = reinterpret_cast<float4 *>(stats);
   const long long need = (total + kScoreWarps - 1) / kScoreWarps;
   const long long cap = (long long)info.sms * info.blocks_per_sm[which];
   const int grid = (int)(need < cap ? need : cap);
-  const int nchunks = d * elem_bytes(dtype) / 16;
-  const uint4 *px = static_cast<const uint4 *>(x);
-  const uint4 *pp = static_cast<const uint4 *>(x_pre ? x_pre : x);
-  const uint4 *pq = static_cast<const uint4 *>(x_post);
-  float4 *ps = reinterpret_cast<float4 *>(stats);
+  const int nchunks = row_bytes / 16;
+  const uint4 *px = reinterpret_cast<const uint4 *>(bx);
+  const uint4 *pp = reinterpret_cast<const uint4 *>(bp);
+  const uint4 *pq = reinterpret_cast<const uint4 *>(bq);
   if (which)
     k_score<true><<<grid, kScoreWarps * 32, 0, st>>>(px, pp, pq, nchunks, total, ps, h2, s);
   else

@@ -2,15 +2,19 @@
 // consistency signal (Eq. 6) in one read of x, x', x''.
 //
 // One warp per row; lane l reads 16-byte chunks l, l+32, l+64, ... of each of
-// the three streams (fully coalesced 512-byte warp requests), kScoreBatch
+// the three streams (fully coalesced 512-byte warp requests), a batch of
 // chunks per stream in flight before any arithmetic.  Each chunk's partial
 // sums of |x|, x^2, x'^2, x''^2 come from a depth-3 fp32 tree; the partials
 // are accumulated error-free as double-floats (TwoSum), so every sum carries
 // at most score_depth() roundings whatever D is.  P = x'.x'' is accumulated
 // error-free term by term, since the ordering by s needs it to far better
-// than fp32.  The epilogue derives the fp32 selection keys from the
-// unrounded double-float sums (double-float arithmetic, one final rounding),
-// all without fp64 (GB300's fp64 rate would stall the warp).
+// than fp32.  bf16 chunks are processed two at a time with the packed f32x2
+// instructions (half the issue slots; each half rounds exactly like the
+// scalar operation), so each lane carries two double-float accumulators per
+// sum, one for its even-numbered chunks and one for its odd ones.  The
+// epilogue derives the fp32 selection keys from the unrounded double-float
+// sums (double-float arithmetic, one final rounding), all without fp64
+// (GB300's fp64 rate would stall the warp).
 #pragma once
 
 #include <cmath>
@@ -61,30 +65,92 @@ struct Acc {
   DF l1, s2, a, b, p;
 };
 
-// Eight bf16 elements of each stream: depth-3 trees for |x|, x^2, x'^2, x''^2
-// (bf16 squares are exact in fp32, so only the additions round); the eight
-// exact products x'x'' go through TwoSum one by one.
-__device__ __forceinline__ void chunk_bf16(const uint4 &vx, const uint4 &vp, const uint4 &vq, Acc &acc) {
-  const uint32_t wx[4] = {vx.x, vx.y, vx.z, vx.w};
-  const uint32_t wp[4] = {vp.x, vp.y, vp.z, vp.w};
-  const uint32_t wq[4] = {vq.x, vq.y, vq.z, vq.w};
-  float l[4], s[4], a[4], b[4];
+// ---- packed pairs: two fp32 values in one 64-bit register pair, operated on
+// by the f32x2 instructions (one issue slot for both halves, each half
+// rounded to nearest exactly like its scalar counterpart).
+__device__ __forceinline__ uint64_t pk(uint32_t lo, uint32_t hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "r"(lo), "r"(hi));
+  return r;
+}
+__device__ __forceinline__ void unpk(uint64_t v, float &lo, float &hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ uint64_t sub2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ uint64_t mul2(uint64_t a, uint64_t b) {
+  uint64_t r;
+  asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+  return r;
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t r;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+  return r;
+}
+
+// A pair of double-float accumulators (one per half).
+struct DF2 {
+  uint64_t hi, lo;
+};
+__device__ __forceinline__ void df2_add(DF2 &a, uint64_t v) {  // TwoSum per half
+  const uint64_t t = add2(a.hi, v);
+  const uint64_t bb = sub2(t, a.hi);
+  const uint64_t aa = sub2(t, bb);
+  a.lo = add2(a.lo, add2(sub2(a.hi, aa), sub2(v, bb)));
+  a.hi = t;
+}
+// Folds the two halves into one double-float accumulator.
+__device__ __forceinline__ DF df2_fold(const DF2 &a) {
+  float h0, h1, l0, l1;
+  unpk(a.hi, h0, h1);
+  unpk(a.lo, l0, l1);
+  DF r{h0, l0};
+  df_merge(r, h1, l1);
+  return r;
+}
+
+struct Acc2 {
+  DF2 l1, s2, a, b, p;
+};
+
+// Two 16-byte chunks (u, v) of bf16 elements of each stream at once: half 0
+// of every packed value belongs to chunk u, half 1 to chunk v.  Per chunk:
+// depth-3 trees of |x|, x^2, x'^2, x''^2 (bf16 squares and products are exact
+// in fp32, so only the additions round; x^2 is taken as |x|^2, the same
+// value) and the eight exact products x'x'' through TwoSum one by one.
+// Chunk u's terms enter accumulator half 0, chunk v's half 1.
+__device__ __forceinline__ void chunk2_bf16(const uint4 &xu, const uint4 &xv, const uint4 &pu, const uint4 &pv,
+                                            const uint4 &qu, const uint4 &qv, Acc2 &acc) {
+  const uint32_t wxu[4] = {xu.x, xu.y, xu.z, xu.w}, wxv[4] = {xv.x, xv.y, xv.z, xv.w};
+  const uint32_t wpu[4] = {pu.x, pu.y, pu.z, pu.w}, wpv[4] = {pv.x, pv.y, pv.z, pv.w};
+  const uint32_t wqu[4] = {qu.x, qu.y, qu.z, qu.w}, wqv[4] = {qv.x, qv.y, qv.z, qv.w};
+  uint64_t l[4], s[4], a[4], b[4];
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    const float x0 = lo_bf16(wx[i]), x1 = hi_bf16(wx[i]);
-    const float p0 = lo_bf16(wp[i]), p1 = hi_bf16(wp[i]);
-    const float q0 = lo_bf16(wq[i]), q1 = hi_bf16(wq[i]);
-    l[i] = fabsf(x0) + fabsf(x1);
-    s[i] = fmaf(x0, x0, x1 * x1);
-    a[i] = fmaf(p0, p0, p1 * p1);
-    b[i] = fmaf(q0, q0, q1 * q1);
-    df_add(acc.p, p0 * q0);
-    df_add(acc.p, p1 * q1);
+    const uint32_t au = wxu[i] & 0x7fff7fffu, av = wxv[i] & 0x7fff7fffu;
+    const uint64_t x0 = pk(au << 16, av << 16), x1 = pk(au & 0xffff0000u, av & 0xffff0000u);
+    const uint64_t p0 = pk(wpu[i] << 16, wpv[i] << 16), p1 = pk(wpu[i] & 0xffff0000u, wpv[i] & 0xffff0000u);
+    const uint64_t q0 = pk(wqu[i] << 16, wqv[i] << 16), q1 = pk(wqu[i] & 0xffff0000u, wqv[i] & 0xffff0000u);
+    l[i] = add2(x0, x1);
+    s[i] = fma2(x0, x0, mul2(x1, x1));
+    a[i] = fma2(p0, p0, mul2(p1, p1));
+    b[i] = fma2(q0, q0, mul2(q1, q1));
+    df2_add(acc.p, mul2(p0, q0));
+    df2_add(acc.p, mul2(p1, q1));
   }
-  df_add(acc.l1, (l[0] + l[1]) + (l[2] + l[3]));
-  df_add(acc.s2, (s[0] + s[1]) + (s[2] + s[3]));
-  df_add(acc.a, (a[0] + a[1]) + (a[2] + a[3]));
-  df_add(acc.b, (b[0] + b[1]) + (b[2] + b[3]));
+  df2_add(acc.l1, add2(add2(l[0], l[1]), add2(l[2], l[3])));
+  df2_add(acc.s2, add2(add2(s[0], s[1]), add2(s[2], s[3])));
+  df2_add(acc.a, add2(add2(a[0], a[1]), add2(a[2], a[3])));
+  df2_add(acc.b, add2(add2(b[0], b[1]), add2(b[2], b[3])));
 }
 
 // Four fp32 elements of each stream: depth-2 trees (plus the rounding of each
@@ -115,38 +181,10 @@ __device__ __forceinline__ void df_warp_sum(DF &v) {
   }
 }
 
-// Scores one row (one warp): the five sums, the fp32 selection keys, and
-// optionally H2 and s.
-template <bool kBf16>
-__device__ __forceinline__ void score_row(const uint4 *__restrict__ x, const uint4 *__restrict__ xp,
-                                          const uint4 *__restrict__ xq, int nchunks, long long row,
-                                          float4 *__restrict__ stats, float *__restrict__ h2,
-                                          float *__restrict__ s_out, int lane) {
-  const uint4 *rx = x + row * nchunks;
-  const uint4 *rp = xp + row * nchunks;
-  const uint4 *rq = xq + row * nchunks;
-  Acc acc{{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
-  for (int c0 = lane; c0 < nchunks; c0 += 32 * kScoreBatch) {
-    uint4 vx[kScoreBatch], vp[kScoreBatch], vq[kScoreBatch];
-#pragma unroll
-    for (int u = 0; u < kScoreBatch; ++u) {
-      const int c = c0 + 32 * u;
-      if (c < nchunks) {
-        vx[u] = ld_stream(rx + c);
-        vp[u] = ld_stream(rp + c);
-        vq[u] = ld_stream(rq + c);
-      } else {
-        vx[u] = vp[u] = vq[u] = make_uint4(0u, 0u, 0u, 0u);
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kScoreBatch; ++u) {
-      if (kBf16)
-        chunk_bf16(vx[u], vp[u], vq[u], acc);
-      else
-        chunk_f32(vx[u], vp[u], vq[u], acc);
-    }
-  }
+// Warp-wide reduction of one row's partial sums and the row's outputs: the
+// five sums, the fp32 selection keys, and optionally H2 and s.  Lane 0 writes.
+__device__ __forceinline__ void finish_row(Acc &acc, long long row, float4 *__restrict__ stats,
+                                           float *__restrict__ h2, float *__restrict__ s_out, int lane) {
   df_warp_sum(acc.l1);
   df_warp_sum(acc.s2);
   df_warp_sum(acc.a);
@@ -175,6 +213,63 @@ __device__ __forceinline__ void score_row(const uint4 *__restrict__ x, const uin
     if (h2) h2[row] = l1 > 0.f ? logf(r) : 0.f;
     if (s_out) s_out[row] = (sa > 0.f && sb > 0.f) ? sv : 0.f;
   }
+}
+
+// Partial sums of chunks [c0, c1) of one row, read straight from global
+// memory: in each round lane l takes chunks base + l + 32u (u < the batch) of
+// each stream, all loads issued before any arithmetic; chunks past c1 are
+// zeros, which add nothing.
+template <bool kBf16>
+__device__ __forceinline__ void accumulate_global(const uint4 *__restrict__ rx, const uint4 *__restrict__ rp,
+                                                  const uint4 *__restrict__ rq, int c0, int c1, Acc &acc,
+                                                  int lane) {
+  constexpr int kB = kBf16 ? kScoreBatchBf16 : kScoreBatchF32;
+  static_assert(kB % 2 == 0, "bf16 chunks are summed in pairs");
+  Acc2 acc2{};
+  for (int base = c0; base < c1; base += 32 * kB) {
+    uint4 vx[kB], vp[kB], vq[kB];
+#pragma unroll
+    for (int u = 0; u < kB; ++u) {
+      const int c = base + lane + 32 * u;
+      if (c < c1) {
+        vx[u] = ld_stream(rx + c);
+        vp[u] = ld_stream(rp + c);
+        vq[u] = ld_stream(rq + c);
+      } else {
+        vx[u] = vp[u] = vq[u] = make_uint4(0u, 0u, 0u, 0u);
+      }
+    }
+    if (kBf16) {
+#pragma unroll
+      for (int u = 0; u < kB; u += 2)
+        chunk2_bf16(vx[u], vx[u + 1], vp[u], vp[u + 1], vq[u], vq[u + 1], acc2);
+    } else {
+#pragma unroll
+      for (int u = 0; u < kB; ++u)
+        chunk_f32(vx[u], vp[u], vq[u], acc);
+    }
+  }
+  if (kBf16) {
+    // Half 0 holds this lane's even-numbered chunks, half 1 its odd ones.
+    const DF l1 = df2_fold(acc2.l1), s2 = df2_fold(acc2.s2), a = df2_fold(acc2.a), b = df2_fold(acc2.b),
+             p = df2_fold(acc2.p);
+    df_merge(acc.l1, l1.hi, l1.lo);
+    df_merge(acc.s2, s2.hi, s2.lo);
+    df_merge(acc.a, a.hi, a.lo);
+    df_merge(acc.b, b.hi, b.lo);
+    df_merge(acc.p, p.hi, p.lo);
+  }
+}
+
+// Scores one row (one warp) straight from global memory.
+template <bool kBf16>
+__device__ __forceinline__ void score_row(const uint4 *__restrict__ x, const uint4 *__restrict__ xp,
+                                          const uint4 *__restrict__ xq, int nchunks, long long row,
+                                          float4 *__restrict__ stats, float *__restrict__ h2,
+                                          float *__restrict__ s_out, int lane) {
+  Acc acc{{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
+  accumulate_global<kBf16>(x + row * nchunks, xp + row * nchunks, xq + row * nchunks, 0, nchunks, acc, lane);
+  finish_row(acc, row, stats, h2, s_out, lane);
 }
 
 }  // namespace

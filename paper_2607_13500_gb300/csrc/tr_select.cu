@@ -73,7 +73,7 @@ int g_sms[64];
 
 size_t select_smem_bytes(int max_n) {
   const size_t cap = (size_t)row_capacity(max_n > 0 ? max_n : 1);
-  return cap * (sizeof(uint32_t) + 2 * sizeof(uint16_t) + sizeof(uint8_t)) + kWarps * 256 * sizeof(uint32_t);
+  return cap * (sizeof(uint32_t) + 3 * sizeof(uint16_t) + sizeof(uint8_t)) + kWarps * 256 * sizeof(uint32_t);
 }
 
 template <typename K>

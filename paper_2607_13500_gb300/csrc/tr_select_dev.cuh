@@ -150,8 +150,12 @@ __device__ __forceinline__ float s_of(const uint32_t *key, const uint16_t *ord, 
 // Cut between importance-sorted positions q-1 and q is certain when the
 // smallest R the bounds allow at q-1 exceeds the largest R they allow at q;
 // evaluated in fp32 with rounding toward the safe side.
+// Certain that a row with key R32 = ra ranks above one with R32 = rb.
+__device__ __forceinline__ bool cert_r_val(float ra, float rb, const Bounds &bd) {
+  return __fmul_rd(ra, bd.r_lo) > __fmul_ru(rb, bd.r_hi);
+}
 __device__ __forceinline__ bool cert_r(const uint32_t *key, const uint16_t *ord, int q, const Bounds &bd) {
-  return __fmul_rd(r_of(key, ord, q - 1), bd.r_lo) > __fmul_ru(r_of(key, ord, q), bd.r_hi);
+  return cert_r_val(r_of(key, ord, q - 1), r_of(key, ord, q), bd);
 }
 // Cut between consistency-sorted positions q-1 and q (ascending s32).
 __device__ __forceinline__ bool cert_s(const uint32_t *key, const uint16_t *ord, int q, const Bounds &bd) {
@@ -899,6 +903,127 @@ __device__ void sort_small(const uint32_t *key, uint16_t *a, int m, unsigned lon
   __syncthreads();
 }
 
+// ---------------------------------------------------------------- sorting
+// Every sort orders rows by the composite (key[row] << 16 | row): by key, ties
+// to the lower row (rows fit 16 bits), which is the order a stable sort of a
+// row-ascending list gives.
+__device__ __forceinline__ unsigned long long comp_key(const uint32_t *key, uint16_t row) {
+  return ((unsigned long long)key[row] << 16) | row;
+}
+
+// The 511 splitters are kept in breadth-first (Eytzinger) order: node e has
+// children 2e+1 and 2e+2, and an in-order walk visits them ascending.  The
+// nodes a search can reach at one level are contiguous, so the lanes of a
+// warp hit distinct banks (a sorted array searched by halving would send
+// them all to the same few banks at the middle levels).
+// In-order rank r (0..510) of the node at breadth-first index e:
+// level l = floor(log2(e + 1)), place p = e + 1 - 2^l, r = (2p + 1) 2^(8 - l) - 1;
+// inversely, with z the trailing zeros of r + 1: l = 8 - z, p = (r + 1) >> (z + 1).
+__device__ __forceinline__ int eytzinger_index(int r) {
+  const int z = __ffs(r + 1) - 1;
+  return (1 << (8 - z)) - 1 + ((r + 1) >> (z + 1));
+}
+// Number of splitters below c: nine comparisons down the tree; the leaf
+// reached, counted from the left, is that number.
+__device__ __forceinline__ int splitter_rank(const unsigned long long *sp, unsigned long long c) {
+  int e = 0;
+#pragma unroll
+  for (int l = 0; l < 9; ++l) e = 2 * e + 1 + (sp[e] < c ? 1 : 0);
+  return e - 511;
+}
+
+// Sample sort of the m rows listed in a (1024 < m <= 16384) by composite key.
+// kSelectThreads rows, one at a pseudo-random place inside each of
+// kSelectThreads equal stretches of a (stratified: evenly spread, yet not
+// aliased with periodic structure such as frames of equal length), are
+// sorted (bitonic); all but the smallest split the keys into kSelectThreads
+// buckets of about m / kSelectThreads rows each.  Each row finds its bucket
+// once (kept in bid), rows are counted per bucket, the counts scanned, the
+// rows scattered into their buckets (any order inside), and a row's place
+// inside its bucket is the number of bucket members with a smaller composite
+// key.  Returns the buffer holding the order, or nullptr, having changed
+// nothing, when the buckets are so uneven that the in-bucket counting would
+// cost more than kSampleWork comparisons per row on average, or hold more
+// than kSampleBucketMax rows in one bucket (the caller then falls back to
+// the radix sort).
+// hist: kWarps x 256 words (splitters and bucket counters); bid: m entries.
+constexpr int kSampleWork = 256;
+constexpr int kSampleBucketMax = 512;
+__device__ __forceinline__ uint32_t mix32(uint32_t x) {  // an integer hash (xorshift-multiply finaliser)
+  x ^= x >> 16;
+  x *= 0x7feb352du;
+  x ^= x >> 15;
+  x *= 0x846ca68bu;
+  x ^= x >> 16;
+  return x;
+}
+__device__ uint16_t *sample_sort(const uint32_t *key, uint16_t *a, uint16_t *b, uint16_t *bid, int m,
+                                 uint32_t *hist) {
+  static_assert(kSelectThreads == 512, "511 splitters, 512 buckets");
+  const int tid = threadIdx.x, nthr = blockDim.x, lane = tid & 31, warp = tid >> 5;
+  unsigned long long *sp = reinterpret_cast<unsigned long long *>(hist);  // [511] splitters (after the sample sort)
+  uint32_t *cnt = hist + 2 * kSelectThreads;                             // [512] bucket counters
+  unsigned long long v[1];
+  {
+    const int lo = (int)((long long)tid * m / kSelectThreads), hi = (int)((long long)(tid + 1) * m / kSelectThreads);
+    v[0] = comp_key(key, a[lo + (int)(mix32((uint32_t)tid + 0x9e3779b9u) % (uint32_t)(hi - lo))]);
+  }
+  __syncthreads();  // hist may still be read by the caller's previous step
+  bitonic_regs<1>(v, sp);
+  if (tid) sp[eytzinger_index(tid - 1)] = v[0];
+  cnt[tid] = 0u;
+  __syncthreads();
+  for (int q = tid; q < m; q += nthr) {
+    const int k = splitter_rank(sp, comp_key(key, a[q]));
+    bid[q] = (uint16_t)k;
+    atomicAdd(&cnt[k], 1u);
+  }
+  __syncthreads();
+  const int size = (int)cnt[tid];
+  if (__syncthreads_or(size > kSampleBucketMax)) return nullptr;
+  int total = 0;
+  const int start = block_exclusive_scan(size, &total);
+  int work = 0;  // sum of squared bucket sizes, at most m^2 <= 2^28
+  block_exclusive_scan(size * size, &work);
+  if ((long long)work > (long long)kSampleWork * m) return nullptr;  // uniform: work is block-wide
+  cnt[tid] = (uint32_t)start;
+  __syncthreads();
+  for (int q = tid; q < m; q += nthr) b[atomicAdd(&cnt[bid[q]], 1u)] = a[q];
+  __syncthreads();
+  // cnt[k] is now the end of bucket k, which spans [cnt[k - 1], cnt[k]).
+  // Warp w owns buckets 32w .. 32w + 31, contiguous in b; lane j holds the
+  // end of bucket 32w + j, and each lane takes one position of the warp's
+  // stretch per round: its bucket by a five-step shuffle search over the
+  // ends, its place by counting the bucket's members with a smaller key.
+  static_assert(kSelectThreads == 32 * kWarps, "one bucket per lane");
+  const int end_l = (int)cnt[warp * 32 + lane];
+  const int beg_w = warp ? (int)cnt[warp * 32 - 1] : 0;
+  const int end_w = __shfl_sync(0xffffffffu, end_l, 31);
+  for (int i0 = beg_w; i0 < end_w; i0 += 32) {
+    const int i = min(i0 + lane, end_w - 1);
+    int k = 0;  // number of this warp's buckets ending at or before i (at most 31)
+#pragma unroll
+    for (int step = 16; step >= 1; step >>= 1)
+      if (__shfl_sync(0xffffffffu, end_l, k + step - 1) <= i) k += step;
+    const int lo_s = __shfl_sync(0xffffffffu, end_l, max(k - 1, 0));
+    const int lo = k ? lo_s : beg_w, hi = __shfl_sync(0xffffffffu, end_l, k);
+    if (i0 + lane < end_w) {
+      const uint16_t row = b[i];
+      const unsigned long long c = comp_key(key, row);
+      int rank = 0, q = lo;
+      for (; q + 4 <= hi; q += 4) {  // four independent loads per step
+        const uint16_t r0 = b[q], r1 = b[q + 1], r2 = b[q + 2], r3 = b[q + 3];
+        rank += (comp_key(key, r0) < c ? 1 : 0) + (comp_key(key, r1) < c ? 1 : 0) +
+                (comp_key(key, r2) < c ? 1 : 0) + (comp_key(key, r3) < c ? 1 : 0);
+      }
+      for (; q < hi; ++q) rank += comp_key(key, b[q]) < c ? 1 : 0;
+      a[lo + rank] = row;
+    }
+  }
+  __syncthreads();
+  return a;
+}
+
 // Ascending order of the m rows listed in a by (key[row], row), by value
 // buckets: the float each key encodes (v = value, or -value for importance
 // keys, which are stored complemented) is mapped linearly from [vmin, vmax]
@@ -994,13 +1119,116 @@ __device__ uint16_t *bucket_sort(const uint32_t *key, uint16_t *a, uint16_t *b, 
 }
 
 // Ascending order of the m rows listed in a by (key[row], row), a listed in
-// ascending row order: value buckets, or the stable radix sort when the keys
-// crowd into few buckets.  Returns the buffer holding the order.
-__device__ uint16_t *sort_rows(const uint32_t *key, uint16_t *a, uint16_t *b, int m, uint32_t *hist,
-                               bool complemented) {
+// ascending row order: a register bitonic sort up to 1024 rows; above that
+// value buckets, the sample sort when the values crowd into few buckets,
+// and the stable radix sort when the sample sort declines too.  Returns the
+// buffer holding the order.
+__device__ uint16_t *sort_rows(const uint32_t *key, uint16_t *a, uint16_t *b, uint16_t *bid, int m,
+                               uint32_t *hist, bool complemented) {
   if (m < 2) return a;
+  unsigned long long *scratch = reinterpret_cast<unsigned long long *>(hist);
+  if (m <= kSelectThreads) {
+    __syncthreads();  // hist may still be read by the caller's previous step
+    sort_small<1>(key, a, m, scratch);
+    return a;
+  }
+  if (m <= 2 * kSelectThreads) {
+    __syncthreads();
+    sort_small<2>(key, a, m, scratch);
+    return a;
+  }
   if (uint16_t *o = bucket_sort(key, a, b, m, hist, complemented)) return o;
+  if (uint16_t *o = sample_sort(key, a, b, bid, m, hist)) return o;
   return radix_sort(key, a, b, m, hist);
+}
+
+// ---------------------------------------------------------------- selection
+// Relative half-width of the window of importance values around an uncertain
+// top-K1 cut whose rows are ordered first (about 2000 times the
+// certification band of the keys).
+constexpr float kCutWindow = 0x1p-11f;
+
+// Key at position r (0-based) of the ascending order of key[0..n), found
+// without sorting: four rounds of 8-bit digit histograms, most significant
+// digit first, each over the rows whose higher digits equal those found so
+// far.  *lt receives how many keys are smaller, *eq how many are equal.
+// hist: kWarps x 256 words.  Called by the whole block.
+__device__ uint32_t select_rank(const uint32_t *key, int n, int r, uint32_t *hist, int *lt, int *eq) {
+  __shared__ uint32_t sh_pre;
+  __shared__ int sh_r, sh_eq;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  uint32_t pre = 0u, mask = 0u;
+  int rr = r;
+  __syncthreads();  // hist may still be read by the caller's previous step
+  for (int shift = 24; shift >= 0; shift -= 8) {
+    uint32_t *h = hist + warp * 256;
+    for (int d = lane; d < 256; d += 32) h[d] = 0u;
+    __syncwarp();
+    for (int i = tid; i < n; i += blockDim.x) {
+      const uint32_t k = key[i];
+      if ((k & mask) == pre) atomicAdd(&h[(k >> shift) & 0xffu], 1u);
+    }
+    __syncthreads();
+    if (tid < 256) {  // column tid: only this thread reads or writes it here
+      uint32_t c = 0u;
+      for (int w = 0; w < kWarps; ++w) c += hist[w * 256 + tid];
+      hist[tid] = c;
+    }
+    __syncthreads();
+    if (warp == 0) {
+      uint32_t c[8], sum = 0u;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        c[j] = hist[lane * 8 + j];
+        sum += c[j];
+      }
+      uint32_t incl = sum;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+      }
+      uint32_t acc = incl - sum;
+      if (acc <= (uint32_t)rr && (uint32_t)rr < incl) {  // exactly one lane holds rank rr
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if ((uint32_t)rr < acc + c[j]) {
+            sh_pre = pre | ((uint32_t)(lane * 8 + j) << shift);
+            sh_r = rr - (int)acc;
+            sh_eq = (int)c[j];
+            break;
+          }
+          acc += c[j];
+        }
+      }
+    }
+    __syncthreads();
+    pre = sh_pre;
+    rr = sh_r;
+    mask |= 0xffu << shift;
+  }
+  *lt = r - rr;
+  *eq = sh_eq;
+  return pre;
+}
+
+// Smallest key[i] (i < n) above t, or 0xffffffff when there is none.
+__device__ uint32_t block_min_above(const uint32_t *key, int n, uint32_t t) {
+  __shared__ uint32_t wmin[32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+  uint32_t v = 0xffffffffu;
+  for (int i = threadIdx.x; i < n; i += blockDim.x) {
+    const uint32_t k = key[i];
+    if (k > t) v = min(v, k);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = min(v, __shfl_xor_sync(0xffffffffu, v, o));
+  __syncthreads();  // wmin may still be read by a previous call
+  if (lane == 0) wmin[warp] = v;
+  __syncthreads();
+  v = 0xffffffffu;
+  for (int w = 0; w < nwarps; ++w) v = min(v, wmin[w]);
+  return v;
 }
 
 __host__ __device__ inline int row_capacity(int max_n) { return (max_n + 15) / 16 * 16; }
@@ -1035,7 +1263,8 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
   uint16_t *ia = reinterpret_cast<uint16_t *>(key + cap);    // [cap] order buffers
   uint16_t *ib = ia + cap;                                   // [cap]
   uint32_t *hist = reinterpret_cast<uint32_t *>(ib + cap);   // [kWarps x 256]
-  uint8_t *fl = reinterpret_cast<uint8_t *>(hist + kWarps * 256);  // [cap] row flags
+  uint16_t *bid = reinterpret_cast<uint16_t *>(hist + kWarps * 256);  // [cap] sort scratch
+  uint8_t *fl = reinterpret_cast<uint8_t *>(bid + cap);             // [cap] row flags
   const float *st = a.stats + off * TR_STATS_WORDS;
   ExactRec *rec = a.exact + off;
   const bool need_r = k1 > 0 && k1 < n;  // the importance order decides something
@@ -1062,47 +1291,117 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
       ia[i] = (uint16_t)i;
     }
     __syncthreads();
-    const uint16_t *ord = sort_rows(key, ia, ib, n, hist, true);
-    if (tid == 0) {
-      int lo = k1, hi = k1;
-      if (!cert_r(key, ord, k1, a.bounds)) {
-        lo = k1 - 1;
-        while (lo > 0 && !cert_r(key, ord, lo, a.bounds)) --lo;
-        hi = k1 + 1;
-        while (hi < n && !cert_r(key, ord, hi, a.bounds)) ++hi;
-      }
-      sh_lo = lo;
-      sh_hi = hi;
+    // Fast path: the K1-th and (K1+1)-th keys by radix selection; when they
+    // differ and their order is certain, the top K1 are exactly the rows
+    // with a key up to the K1-th, and no order is needed.
+    int lt = 0, eq = 0;
+    const uint32_t t1 = select_rank(key, n, k1 - 1, hist, &lt, &eq);
+    bool settled = false;
+    if (lt + eq == k1) {
+      const uint32_t t2 = block_min_above(key, n, t1);
+      settled = cert_r_val(unord32(~t1), unord32(~t2), a.bounds);
     }
-    __syncthreads();
-    const int lo = sh_lo, hi = sh_hi;
-    for (int q = tid; q < lo; q += nthr) fl[ord[q]] |= F_IMP;
-    if (hi > lo) {
-      for (int q = lo + tid; q < hi; q += nthr) {
-        const int r = ord[q];
-        if (!(fl[r] & F_XL)) fl[r] |= F_NEEDL;
-      }
+    if (settled) {
+      for (int i = tid; i < n; i += nthr)
+        if (key[i] <= t1) fl[i] |= F_IMP;
       __syncthreads();
-      refine_pending(a, off, n, fl, rec, primary);
-      __syncthreads();
-      for (int q = lo + tid; q < hi; q += nthr) {
-        const int r = ord[q];
-        const bool ovf = rec[r].flags_l & kRecOverflowL;
-        int rank = 0;
-        for (int q2 = lo; q2 < hi; ++q2) {
-          if (q2 == q) continue;
-          const int r2 = ord[q2];
-          int c;
-          if (ovf || (rec[r2].flags_l & kRecOverflowL))
-            c = q2 < q ? 1 : -1;  // no exact value: keep the float order
-          else
-            c = cmp_r(rec[r2], rec[r]);
-          if (c > 0 || (c == 0 && r2 < r)) ++rank;
+    } else {
+      // Uncertain cut: only the order near it matters.  The rows whose R32
+      // lies within a relative kCutWindow of the K1-th one (far wider than
+      // the certification band) are listed and sorted; when the uncertain
+      // run around the cut ends inside that list, every row with a smaller
+      // key (larger R) precedes it in the full order and is certainly kept,
+      // every row with a larger key certainly not.  Otherwise (or when the
+      // window holds too many rows) all n rows are sorted.
+      const float r1 = unord32(~t1);
+      const uint32_t kw_lo = ~ord32(r1 * (1.f + kCutWindow)), kw_hi = ~ord32(r1 * (1.f - kCutWindow));
+      const bool windowed = isfinite(r1) && r1 > 0.f;  // uniform
+      const uint16_t *ord = nullptr;
+      int base = 0, len = 0;  // ord[q] sits at position base + q of the full order
+      if (windowed) {
+        const int per = (n + nthr - 1) / nthr;
+        const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
+        int c_in = 0, c_lt = 0;
+        for (int i = i0; i < i1; ++i) {
+          const uint32_t k = key[i];
+          c_in += k >= kw_lo && k <= kw_hi;
+          c_lt += k < kw_lo;
         }
-        if (lo + rank < k1) fl[r] |= F_IMP;
+        int n_in = 0, n_lt = 0;
+        int pos = block_exclusive_scan(c_in, &n_in);
+        block_exclusive_scan(c_lt, &n_lt);
+        if (n_in <= 2 * kSelectThreads) {  // uniform
+          for (int i = i0; i < i1; ++i) {
+            const uint32_t k = key[i];
+            if (k >= kw_lo && k <= kw_hi) ib[pos++] = (uint16_t)i;
+          }
+          __syncthreads();
+          unsigned long long *scratch = reinterpret_cast<unsigned long long *>(hist);
+          if (n_in <= kSelectThreads)
+            sort_small<1>(key, ib, n_in, scratch);
+          else
+            sort_small<2>(key, ib, n_in, scratch);
+          ord = ib;
+          base = n_lt;
+          len = n_in;
+        }
       }
+      for (int attempt = 0; attempt < 2; ++attempt) {
+        if (!ord) {
+          ord = sort_rows(key, ia, ib, bid, n, hist, true);
+          base = 0;
+          len = n;
+        }
+        const bool whole = base == 0 && len == n;
+        if (tid == 0) {
+          int lo = k1 - base, hi = k1 - base;
+          bool escaped = lo < 1 || lo >= len;
+          if (!escaped && !cert_r(key, ord, lo, a.bounds)) {
+            --lo;
+            while (lo > 0 && !cert_r(key, ord, lo, a.bounds)) --lo;
+            ++hi;
+            while (hi < len && !cert_r(key, ord, hi, a.bounds)) ++hi;
+            escaped = !whole && (lo == 0 || hi == len);  // the run may go on outside the list
+          }
+          sh_lo = escaped ? -1 : lo;
+          sh_hi = hi;
+        }
+        __syncthreads();
+        if (sh_lo >= 0) break;
+        ord = nullptr;  // the window was not enough: sort everything
+      }
+      const int lo = sh_lo, hi = sh_hi;
+      if (base > 0)
+        for (int i = tid; i < n; i += nthr)
+          if (key[i] < kw_lo) fl[i] |= F_IMP;
+      for (int q = tid; q < lo; q += nthr) fl[ord[q]] |= F_IMP;
+      if (hi > lo) {
+        for (int q = lo + tid; q < hi; q += nthr) {
+          const int r = ord[q];
+          if (!(fl[r] & F_XL)) fl[r] |= F_NEEDL;
+        }
+        __syncthreads();
+        refine_pending(a, off, n, fl, rec, primary);
+        __syncthreads();
+        for (int q = lo + tid; q < hi; q += nthr) {
+          const int r = ord[q];
+          const bool ovf = rec[r].flags_l & kRecOverflowL;
+          int rank = 0;
+          for (int q2 = lo; q2 < hi; ++q2) {
+            if (q2 == q) continue;
+            const int r2 = ord[q2];
+            int c;
+            if (ovf || (rec[r2].flags_l & kRecOverflowL))
+              c = q2 < q ? 1 : -1;  // no exact value: keep the float order
+            else
+              c = cmp_r(rec[r2], rec[r]);
+            if (c > 0 || (c == 0 && r2 < r)) ++rank;
+          }
+          if (base + lo + rank < k1) fl[r] |= F_IMP;
+        }
+      }
+      __syncthreads();
     }
-    __syncthreads();
   } else if (k1 == n) {
     for (int i = tid; i < n; i += nthr) fl[i] |= F_IMP;
     __syncthreads();
@@ -1124,7 +1423,7 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
       key[i] = ord32(sv);
     }
     __syncthreads();
-    const uint16_t *ord = sort_rows(key, ia, ib, m, hist, false);
+    const uint16_t *ord = sort_rows(key, ia, ib, bid, m, hist, false);
     const int t = max(1, m / k2);
     for (int j = tid; j < k2; j += nthr) {
       const int p = j * t;

@@ -186,6 +186,54 @@ def test_exact_ties_and_degenerate_rows():
     check_reduce(xe, xp, xq, [n], ([40], [13], [0, 40]))
 
 
+def test_sort_paths_uneven_and_tied_keys():
+    # 512 distinct rows at every 4th position and 1536 copies of one row
+    # whose R = 1 (one-hot) is the smallest of all: the importance cut falls
+    # inside the copies (an exact tie), so the full importance order is
+    # needed (value buckets crowd, the sample sort orders them); the rows
+    # left for the consistency order tie in s.
+    n, d = 2048, 64
+    x, xp, xq = _rows(n, d, 11)
+    tied = [i for i in range(n) if i % 4]
+    x[tied] = 0
+    x[tied, 5] = 1.0
+    xp[tied] = xp[1].clone()
+    xq[tied] = xq[1].clone()
+    for k, k1 in [(900, 600), (700, 256), (1024, 0)]:
+        check_reduce(x, xp, xq, [n], ([k], [k1], [0, k]))
+
+
+def _mix32(v):
+    v &= 0xFFFFFFFF
+    v ^= v >> 16
+    v = (v * 0x7FEB352D) & 0xFFFFFFFF
+    v ^= v >> 15
+    v = (v * 0x846CA68B) & 0xFFFFFFFF
+    return v ^ (v >> 16)
+
+
+def test_sort_fallback_when_samples_are_adversarial():
+    # Above 1024 rows the sort first tries value buckets, then draws 512
+    # samples, one at a hashed place in each equal stretch of the row list
+    # (the places below repeat that scheme).  Here exactly the sampled rows
+    # are distinct and every other row is a copy of one row with the
+    # smallest R and the largest s: the copies crowd one value bucket and
+    # one sample bucket, so both sorts decline and the radix sort orders the
+    # rows, for the importance cut (which falls inside the copies) and for
+    # the consistency order over all rows.
+    n, d, S = 4096, 64, 512
+    picked = [t * n // S + _mix32(t + 0x9E3779B9) % ((t + 1) * n // S - t * n // S) for t in range(S)]
+    assert len(set(picked)) == S
+    x, xp, xq = _rows(n, d, 12)
+    rest = sorted(set(range(n)) - set(picked))
+    x[rest] = 0
+    x[rest, 9] = 1.0
+    xp[rest] = 1.0
+    xq[rest] = 1.0  # s = 1, the largest
+    for k, k1 in [(900, 600), (3000, 0)]:
+        check_reduce(x, xp, xq, [n], ([k], [k1], [0, k]))
+
+
 def test_nonfinite_huge_and_tiny_rows():
     n, d = 64, 256
     x, xp, xq = _rows(n, d, 4)
