@@ -3,8 +3,12 @@
 
 One step = one pass of the whole path (per-token scores, per-image top-K1,
 sort of the rest by the consistency signal, stride pick, gather) over one
-batch of synthetic images already resident in HBM: two kernels, k_score and
-k_select_gather, timed with CUDA events around each.  Prints one JSON line.
+batch of synthetic images already resident in HBM: three kernels, k_score,
+k_select and k_gather.  Steps go through the library's two-stream pipeline
+(tr_pipeline): step i's selection and gather run on a high-priority stream
+while step i + 1 is scored.  The timed region spans all K steps; the score
+kernel is bracketed by CUDA events on its stream in every step.  Prints one
+JSON line.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference] [--workload NAME]
 
@@ -269,6 +273,7 @@ def run_ours(args, world, rank, local):
     over = {"batch": args.batch} if args.batch else {}
     w = synth.make(args.workload, seed=rank_seed(args.seed, rank), device=dev, **over)
     red = altr.Reducer(w.seqlens, w.d, w.x.dtype, dev, **budget)
+    pipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, slots=2, **budget)
     e = 2 if w.x.dtype == torch.bfloat16 else 4
     total_rows = w.total
     in_bytes = 3 * total_rows * w.d * e
@@ -278,29 +283,40 @@ def run_ours(args, world, rank, local):
         if world > 1:
             torch.distributed.barrier()
 
+    # each kernel alone (one stream, back to back), outside the timed region
+    alone_evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(max(3, args.warmup))]
+    for ev in alone_evs:
+        red.run_separate(w.x, w.x_pre, w.x_post, ev)
+    torch.cuda.synchronize()
+    alone = {name: statistics.median(ev[j].elapsed_time(ev[j + 1]) for ev in alone_evs[1:])
+             for j, name in enumerate(["k_score", "k_select", "k_gather"])}
+
     clocks = ClockSampler(dev)
     for _ in range(args.warmup):
-        red.run_split(w.x, w.x_pre, w.x_post)
-    torch.cuda.synchronize()
-    st = red.status.cpu().tolist()
-    # timed region: K steps, per-kernel events inside every step
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+        pipe.submit(w.x, w.x_pre, w.x_post)
+    pipe.synchronize()
+    st = pipe.outs[(pipe.submitted - 1) % pipe.slots]["status"].cpu().tolist()
+    # timed region: K steps through the two-stream pipeline (the selection
+    # and gather of step i overlap the scoring of step i + 1), the score
+    # kernel bracketed by events on its stream in every step
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     barrier()
     torch.cuda.synchronize()
-    start.record()
+    start.record(pipe.score_stream)
     for i in range(args.steps):
-        red.run_split(w.x, w.x_pre, w.x_post, evs[i])
-    end.record()
+        pipe.submit(w.x, w.x_pre, w.x_post, score_events=evs[i])
+    pipe.wait(pipe.score_stream)
+    end.record(pipe.score_stream)
     torch.cuda.synchronize()
     barrier()
     clk = clocks.stop()
     total_ms = start.elapsed_time(end)
     t_score = [ev[0].elapsed_time(ev[1]) for ev in evs]
-    t_select = [ev[1].elapsed_time(ev[2]) for ev in evs]
     ms_step = max_over_ranks(total_ms / args.steps, world, dev)
     images = w.batch * world
     value = job_images_per_s(w.batch, world, ms_step)
+    pipe.close()
 
     # end to end through the public API: pinned host inputs in, y and idx out
     pin = lambda t: t.cpu().pin_memory()
@@ -337,11 +353,12 @@ def run_ours(args, world, rank, local):
         "config": {**_workload_config(w, budget, args), "parallelism": f"replicas x{world} (images sharded)",
                    "l2": f"inputs {in_bytes / 2**20:.0f} MiB > L2 {L2_BYTES // 2**20} MiB, no flush"},
         "hbm_gbs": path_gbs, "frac_of_8tbs": path_gbs / NOMINAL_HBM_GBS, "frac_of_measured": path_gbs / peak,
-        "kernels_ms": {"k_score": score_ms, "k_select_gather": statistics.mean(t_select)},
+        "kernels_ms": {"k_score_in_pipeline": score_ms, **{f"{k}_alone": v for k, v in alone.items()}},
+        "pipeline": "2 slots: step i's k_select + k_gather (high-priority stream) overlap step i+1's k_score",
         "roofline": roofline,
         "e2e": {"value": images / e2e_s, "unit": "images/s", "h2d_bytes_per_step": in_bytes,
                 "d2h_bytes_per_step": red.total_k * (w.d * e + 4)},
-        "gpu_launches": 2 * args.steps,
+        "gpu_launches": 3 * args.steps,
         "clocks": clk,
         "status": st,
     }

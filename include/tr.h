@@ -9,9 +9,10 @@
  * Eq. 5-6), returned as X* = X_imp union X_div (Eq. 7, Algorithm 1).
  *
  * Conventions shared by every entry point:
- *  - Device pointers are owned by the caller; the library never allocates,
- *    frees or synchronises.  Every call enqueues work on `stream` (a
- *    cudaStream_t; NULL is the legacy default stream) and returns at once.
+ *  - Device pointers are owned by the caller; the library never allocates
+ *    device memory, frees it or synchronises.  Every call enqueues work on
+ *    `stream` (a cudaStream_t; NULL is the legacy default stream) and returns
+ *    at once.  (A tr_pipeline owns host-side CUDA events, see below.)
  *  - Host-detectable errors (null or misaligned pointers, bad sizes, too small
  *    a workspace) are returned before anything is launched; outputs are left
  *    untouched.  A launch failure returns TR_ERR_CUDA.
@@ -205,6 +206,44 @@ tr_status tr_reduce(const tr_tokens *in, const int32_t *d_k, const int32_t *d_k1
 tr_status tr_reduce_noalloc(const tr_tokens *in, const int32_t *d_k, const int32_t *d_k1, const int32_t *d_cu_k,
                             int32_t total_k, void *y, int32_t *idx, float *h2, float *s, int32_t *d_status,
                             void *stream);
+
+/*
+ * Overlapped reduction of successive batches, a two-stream pipeline.  A
+ * submission scores its batch on `score_stream` (tr_score), then selects
+ * (tr_select) and gathers (tr_gather) it on `select_stream`, which waits for
+ * that scoring only; so the selection and gather of one batch run while the
+ * next batch is scored.  Give `select_stream` the higher priority: the score
+ * kernel's CTAs retire one by one, and a higher-priority kernel takes the
+ * SMs they free.  Submission i uses workspace ws[i mod slots] (each of
+ * ws_bytes >= tr_workspace_bytes bytes, 256-byte aligned, owned by the
+ * caller) and waits, on score_stream, until the submission that used that
+ * workspace last has been gathered.
+ *
+ * Ordering the caller keeps: the inputs of a submission (x, x', x'') stay
+ * unchanged, and its outputs (y, idx, h2, s, d_status) untouched by other
+ * work, until select_stream has passed the submission -- give each
+ * submission still in flight its own output buffers (one set per slot).
+ * Work that consumes a submission's outputs orders itself after it on
+ * select_stream (or tr_pipeline_wait).
+ *
+ * The pipeline owns 2 x slots CUDA events, created on the current device by
+ * tr_pipeline_create (make it the device of both streams) and destroyed by
+ * tr_pipeline_destroy; it allocates no device memory and never synchronises.
+ *   tr_pipeline_submit: arguments as in tr_reduce; score_begin / score_end
+ *     are optional cudaEvent_t (or NULL) recorded on score_stream right
+ *     before and after the score kernel, to time it.  Host-detectable errors
+ *     are returned before anything is enqueued.
+ *   tr_pipeline_wait: makes `stream` wait for every submission so far.
+ */
+#define TR_PIPELINE_MAX_SLOTS 8
+typedef struct tr_pipeline tr_pipeline;
+tr_status tr_pipeline_create(void *score_stream, void *select_stream, int32_t slots, void *const *ws,
+                             size_t ws_bytes, tr_pipeline **out);
+tr_status tr_pipeline_submit(tr_pipeline *p, const tr_tokens *in, const int32_t *d_k, const int32_t *d_k1,
+                             const int32_t *d_cu_k, int32_t total_k, void *y, int32_t *idx, float *h2, float *s,
+                             int32_t *d_status, void *score_begin, void *score_end);
+tr_status tr_pipeline_wait(tr_pipeline *p, void *stream);
+tr_status tr_pipeline_destroy(tr_pipeline *p);
 
 #ifdef __cplusplus
 }

@@ -9,6 +9,6 @@ by consistency (Algorithm 1), gathered into a compact [sum K, D] tensor.
 The work runs in libtr.so (hand-written CUDA for sm_103a, C ABI in
 include/tr.h); this package is its Python binding.
 """
-from .api import Reducer, ReduceResult, budgets, reduce, score, select, workspace_bytes
+from .api import Pipeline, Reducer, ReduceResult, budgets, reduce, score, select, workspace_bytes
 
-__all__ = ["Reducer", "ReduceResult", "budgets", "reduce", "score", "select", "workspace_bytes"]
+__all__ = ["Pipeline", "Reducer", "ReduceResult", "budgets", "reduce", "score", "select", "workspace_bytes"]

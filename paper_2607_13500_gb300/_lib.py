@@ -64,6 +64,12 @@ def load() -> ctypes.CDLL:
     lib.tr_gather.argtypes, lib.tr_gather.restype = [tok, VP, VP, I32, VP, VP], I32
     lib.tr_select_gather.argtypes = [tok, VP, VP, VP, VP, I32, VP, VP, VP, VP, VP, SZ, VP, VP]
     lib.tr_select_gather.restype = I32
+    lib.tr_pipeline_create.argtypes = [VP, VP, I32, P(VP), SZ, P(VP)]
+    lib.tr_pipeline_create.restype = I32
+    lib.tr_pipeline_submit.argtypes = [VP, tok, VP, VP, VP, I32, VP, VP, VP, VP, VP, VP, VP]
+    lib.tr_pipeline_submit.restype = I32
+    lib.tr_pipeline_wait.argtypes, lib.tr_pipeline_wait.restype = [VP, VP], I32
+    lib.tr_pipeline_destroy.argtypes, lib.tr_pipeline_destroy.restype = [VP], I32
     lib.tr_reduce.argtypes = [tok, VP, VP, VP, I32, VP, VP, VP, VP, VP, SZ, VP, VP]
     lib.tr_reduce.restype = I32
     _lib = lib

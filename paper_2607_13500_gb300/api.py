@@ -223,6 +223,30 @@ class Reducer:
         return ReduceResult(self.y[:self.total_k], self.idx[:self.total_k], self.cu_k, self.h2, self.s,
                             self.status)
 
+    def run_separate(self, x, x_pre, x_post, events=None):
+        """The three kernels the pipeline launches, tr_score, tr_select and
+        tr_gather, on the current stream, with ``events`` (four
+        torch.cuda.Event, or None) recorded before, between and after them."""
+        tok = self._bind(x, x_pre, x_post)
+        st = _stream(self.device)
+        lib = self.lib
+        stats = self._stats_view()
+        if events:
+            events[0].record()
+        check("tr_score", lib.tr_score(tok.ref(), _ptr(stats), _ptr(self.h2), _ptr(self.s), st))
+        if events:
+            events[1].record()
+        check("tr_select", lib.tr_select(
+            tok.ref(), _ptr(stats), _ptr(self.d_k), _ptr(self.d_k1), _ptr(self.d_cu), _ptr(self.idx), None,
+            _ptr(self.h2), _ptr(self.s), _ptr(self._ws), self._ws_bytes, _ptr(self.status), st))
+        if events:
+            events[2].record()
+        check("tr_gather", lib.tr_gather(tok.ref(), _ptr(self.d_cu), _ptr(self.idx), self.total_k, _ptr(self.y), st))
+        if events:
+            events[3].record()
+        return ReduceResult(self.y[:self.total_k], self.idx[:self.total_k], self.cu_k, self.h2, self.s,
+                            self.status)
+
     def _stats_view(self):
         # tr_reduce keeps the statistics at the start of the workspace; the
         # split path uses the same bytes.
@@ -245,6 +269,107 @@ class Reducer:
         y_h.copy_(r.y, non_blocking=True)
         idx_h.copy_(r.idx, non_blocking=True)
         return r
+
+
+class Pipeline:
+    """tr_pipeline: successive batches of one shape, each scored on
+    ``score_stream`` and then selected and gathered on ``select_stream``
+    (higher priority), so that the selection and gather of one batch overlap
+    the scoring of the next.  Submission i uses workspace and output set
+    i mod ``slots``; its ReduceResult holds that set's tensors, valid once
+    ``select_stream`` has passed the submission (``wait`` or
+    ``synchronize``) and until submission i + ``slots`` is made.
+    """
+
+    def __init__(self, seqlens, d, dtype, device, k=None, ratio=None, lam=(1, 3), alias_pre=False, scores=False,
+                 budget=None, slots=2):
+        self.lib = load()
+        self.seqlens = [int(v) for v in seqlens]
+        self.device = torch.device(device)
+        self.d, self.dtype, self.alias_pre, self.slots = d, dtype, alias_pre, int(slots)
+        self.ks, self.k1s, self.cu_k = budget if budget is not None else budgets(self.seqlens, k, ratio, lam)
+        self.total_k = self.cu_k[-1]
+        t = sum(self.seqlens)
+        dev = self.device
+        self.d_k = torch.tensor(self.ks, dtype=torch.int32, device=dev)
+        self.d_k1 = torch.tensor(self.k1s, dtype=torch.int32, device=dev)
+        self.d_cu = torch.tensor(self.cu_k, dtype=torch.int32, device=dev)
+        mk = lambda *shape, dt: torch.empty(*shape, dtype=dt, device=dev)
+        self.outs = [dict(y=mk(max(self.total_k, 1), d, dt=dtype), idx=mk(max(self.total_k, 1), dt=torch.int32),
+                          h2=mk(t, dt=torch.float32) if scores else None, s=mk(t, dt=torch.float32) if scores else None,
+                          status=torch.zeros(TR_STATUS_WORDS, dtype=torch.int32, device=dev))
+                     for _ in range(self.slots)]
+        self.score_stream = torch.cuda.Stream(dev, priority=0)
+        self.select_stream = torch.cuda.Stream(dev, priority=-100)  # the device's highest priority
+        self._ws = None
+        self._handle = None
+        self._tok = None
+        self._in = None
+        self.submitted = 0
+
+    def _bind(self, x, x_pre, x_post):
+        x, x_pre, x_post, _ = _flatten(x, x_pre, x_post, self.seqlens)
+        key = (x.data_ptr(), None if x_pre is None else x_pre.data_ptr(), x_post.data_ptr())
+        if self._tok is None or self._in != key:
+            self._tok = _Tokens(x, x_pre, x_post, self.seqlens)
+            self._in = key
+        if self._handle is None:
+            nbytes = self.lib.tr_workspace_bytes(self._tok.ref())
+            if nbytes == 0:
+                raise ValueError("invalid token tensors for tr_pipeline")
+            self._ws = [torch.empty(nbytes, dtype=torch.uint8, device=self.device) for _ in range(self.slots)]
+            assert all(w.data_ptr() % 256 == 0 for w in self._ws)
+            ptrs = (ctypes.c_void_p * self.slots)(*[w.data_ptr() for w in self._ws])
+            handle = ctypes.c_void_p()
+            with torch.cuda.device(self.device):
+                check("tr_pipeline_create", self.lib.tr_pipeline_create(
+                    ctypes.c_void_p(self.score_stream.cuda_stream), ctypes.c_void_p(self.select_stream.cuda_stream),
+                    self.slots, ptrs, nbytes, ctypes.byref(handle)))
+            self._handle = handle
+        return self._tok
+
+    def submit(self, x, x_pre, x_post, score_events=None) -> ReduceResult:
+        """Enqueues one batch; ``score_events`` (two torch.cuda.Event, or
+        None) are recorded on score_stream around the score kernel."""
+        tok = self._bind(x, x_pre, x_post)
+        o = self.outs[self.submitted % self.slots]
+        # the inputs come from the caller's stream; the status words start at zero
+        self.score_stream.wait_stream(torch.cuda.current_stream(self.device))
+        with torch.cuda.stream(self.select_stream):
+            o["status"].zero_()
+        ev = [None, None]
+        if score_events is not None:
+            for e in score_events:
+                if not e.cuda_event:  # torch creates its events lazily, at the first record
+                    e.record(self.score_stream)
+            ev = [ctypes.c_void_p(e.cuda_event) for e in score_events]
+        check("tr_pipeline_submit", self.lib.tr_pipeline_submit(
+            self._handle, tok.ref(), _ptr(self.d_k), _ptr(self.d_k1), _ptr(self.d_cu), self.total_k, _ptr(o["y"]),
+            _ptr(o["idx"]), _ptr(o["h2"]), _ptr(o["s"]), _ptr(o["status"]), ev[0], ev[1]))
+        self.submitted += 1
+        return ReduceResult(o["y"][:self.total_k], o["idx"][:self.total_k], self.cu_k, o["h2"], o["s"], o["status"])
+
+    def wait(self, stream=None):
+        """Makes ``stream`` (default: the current stream) wait for every submission."""
+        st = stream if stream is not None else torch.cuda.current_stream(self.device)
+        if self._handle is not None:
+            check("tr_pipeline_wait", self.lib.tr_pipeline_wait(self._handle, ctypes.c_void_p(st.cuda_stream)))
+
+    def synchronize(self):
+        self.select_stream.synchronize()
+        self.score_stream.synchronize()
+
+    def close(self):
+        if self._handle is not None:
+            self.synchronize()
+            self.lib.tr_pipeline_destroy(self._handle)
+            self._handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
 
 
 def reduce(x, x_pre, x_post, k=None, ratio=None, lam=(1, 3), seqlens=None, scores=False, budget=None):

@@ -2,6 +2,8 @@
 // workspace carving and launches (tr_reduce: score, then select + gather).
 #include <climits>
 
+#include <new>
+
 #include "tr_internal.cuh"
 
 using namespace tr;
@@ -187,6 +189,91 @@ tr_status tr_gather(const tr_tokens *in, const int32_t *d_cu_k, const int32_t *i
   cudaError_t err = launch_gather(in->x, sh.total, in->dtype, in->d, in->batch, in->cu_seqlens ? 0 : in->n,
                                   in->cu_seqlens, d_cu_k, idx, total_k, y, static_cast<cudaStream_t>(stream));
   return err == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+}
+
+// ---------------------------------------------------------------- pipeline
+struct tr_pipeline {
+  cudaStream_t score_stream = nullptr, select_stream = nullptr;
+  int slots = 0;
+  void *ws[TR_PIPELINE_MAX_SLOTS] = {};
+  size_t ws_bytes = 0;
+  cudaEvent_t scored[TR_PIPELINE_MAX_SLOTS] = {};
+  cudaEvent_t done[TR_PIPELINE_MAX_SLOTS] = {};
+  long long submitted = 0;
+};
+
+tr_status tr_pipeline_create(void *score_stream, void *select_stream, int32_t slots, void *const *ws,
+                             size_t ws_bytes, tr_pipeline **out) {
+  if (!out) return TR_ERR_ARG;
+  *out = nullptr;
+  if (slots < 1 || slots > TR_PIPELINE_MAX_SLOTS || !ws) return TR_ERR_ARG;
+  for (int i = 0; i < slots; ++i)
+    if (!ws[i] || misaligned(ws[i], 256)) return TR_ERR_WORKSPACE;
+  tr_pipeline *p = new (std::nothrow) tr_pipeline;
+  if (!p) return TR_ERR_ARG;
+  p->score_stream = static_cast<cudaStream_t>(score_stream);
+  p->select_stream = static_cast<cudaStream_t>(select_stream);
+  p->slots = slots;
+  p->ws_bytes = ws_bytes;
+  for (int i = 0; i < slots; ++i) {
+    p->ws[i] = ws[i];
+    if (cudaEventCreateWithFlags(&p->scored[i], cudaEventDisableTiming) != cudaSuccess ||
+        cudaEventCreateWithFlags(&p->done[i], cudaEventDisableTiming) != cudaSuccess) {
+      tr_pipeline_destroy(p);
+      return TR_ERR_CUDA;
+    }
+  }
+  *out = p;
+  return TR_OK;
+}
+
+tr_status tr_pipeline_submit(tr_pipeline *p, const tr_tokens *in, const int32_t *d_k, const int32_t *d_k1,
+                             const int32_t *d_cu_k, int32_t total_k, void *y, int32_t *idx, float *h2, float *s,
+                             int32_t *d_status, void *score_begin, void *score_end) {
+  if (!p) return TR_ERR_ARG;
+  Shape sh;
+  tr_status rc = check_tokens(in, &sh);
+  if (rc != TR_OK) return rc;
+  if (total_k < 0 || total_k > sh.total) return TR_ERR_BUDGET;
+  if (in->batch > 0 && (!d_k || !d_k1 || !d_cu_k || !idx || (total_k > 0 && !y))) return TR_ERR_ARG;
+  if (misaligned(y, 16) || misaligned(h2, 4) || misaligned(s, 4)) return TR_ERR_ALIGN;
+  const int slot = (int)(p->submitted % p->slots);
+  void *ws = p->ws[slot];
+  if ((rc = check_ws(sh, ws, p->ws_bytes)) != TR_OK) return rc;
+  float *stats = reinterpret_cast<float *>(static_cast<char *>(ws) + ws_layout(sh.total).stats);
+  cudaStream_t a = p->score_stream, b = p->select_stream;
+  // The slot's workspace is free once the submission that used it last has
+  // been selected and gathered.
+  if (p->submitted >= p->slots && cudaStreamWaitEvent(a, p->done[slot], 0) != cudaSuccess) return TR_ERR_CUDA;
+  if (score_begin && cudaEventRecord(static_cast<cudaEvent_t>(score_begin), a) != cudaSuccess) return TR_ERR_CUDA;
+  if ((rc = tr_score(in, stats, h2, s, a)) != TR_OK) return rc;
+  if (score_end && cudaEventRecord(static_cast<cudaEvent_t>(score_end), a) != cudaSuccess) return TR_ERR_CUDA;
+  if (cudaEventRecord(p->scored[slot], a) != cudaSuccess || cudaStreamWaitEvent(b, p->scored[slot], 0) != cudaSuccess)
+    return TR_ERR_CUDA;
+  if ((rc = tr_select(in, stats, d_k, d_k1, d_cu_k, idx, nullptr, h2, s, ws, p->ws_bytes, d_status, b)) != TR_OK)
+    return rc;
+  if ((rc = tr_gather(in, d_cu_k, idx, total_k, y, b)) != TR_OK) return rc;
+  if (cudaEventRecord(p->done[slot], b) != cudaSuccess) return TR_ERR_CUDA;
+  ++p->submitted;
+  return TR_OK;
+}
+
+tr_status tr_pipeline_wait(tr_pipeline *p, void *stream) {
+  if (!p) return TR_ERR_ARG;
+  const long long used = p->submitted < p->slots ? p->submitted : p->slots;
+  for (long long i = 0; i < used; ++i)
+    if (cudaStreamWaitEvent(static_cast<cudaStream_t>(stream), p->done[i], 0) != cudaSuccess) return TR_ERR_CUDA;
+  return TR_OK;
+}
+
+tr_status tr_pipeline_destroy(tr_pipeline *p) {
+  if (!p) return TR_OK;
+  for (int i = 0; i < TR_PIPELINE_MAX_SLOTS; ++i) {
+    if (p->scored[i]) cudaEventDestroy(p->scored[i]);
+    if (p->done[i]) cudaEventDestroy(p->done[i]);
+  }
+  delete p;
+  return TR_OK;
 }
 
 }  // extern "C"

@@ -47,6 +47,11 @@ def check_reduce(x, x_pre, x_post, seqlens, budget, images=None, alias=False, ex
     dp = None if alias else x_pre.to(dev)
     r = altr.reduce(dx, dp, dq, seqlens=seqlens, budget=budget, scores=True)
     torch.cuda.synchronize()
+    return compare_result(r, x, x_pre, x_post, seqlens, budget, images, alias, expect_nonfinite)
+
+
+def compare_result(r, x, x_pre, x_post, seqlens, budget, images=None, alias=False, expect_nonfinite=False):
+    """A ReduceResult (already complete) against the oracle, image by image."""
     ks, k1s, cu = budget
     status = r.status.cpu().tolist()
     assert status[1] == 0, f"unresolved rows: {status}"
@@ -140,6 +145,31 @@ def test_score_and_select_entry_points():
     p = (_f64(w.x_pre) * _f64(w.x_post)).sum(1)
     scale = np.sqrt((_f64(w.x_pre) ** 2).sum(1) * (_f64(w.x_post) ** 2).sum(1))
     assert np.all(np.abs(st[:, 4] + st[:, 5] - p) <= 1e-9 * scale)
+
+
+def test_pipeline_overlapped_batches():
+    # Three different batches of one shape through a two-slot pipeline: the
+    # selection of one overlaps the scoring of the next, slot 0 is reused
+    # (its workspace and outputs wait for the earlier gather), and a run of
+    # submissions without a host sync in between ends with the right results.
+    altr = _alt()
+    ws = [synth.make("multitile2880", seed=s, device="cuda", batch=3, n=700, d=1024) for s in range(3)]
+    budget = _budget(ws[0], k=120)
+    pipe = altr.Pipeline(ws[0].seqlens, ws[0].d, ws[0].x.dtype, "cuda", budget=budget, scores=True, slots=2)
+    cpu = [(w.x.cpu(), w.x_pre.cpu(), w.x_post.cpu()) for w in ws]
+    try:
+        r0 = pipe.submit(ws[0].x, ws[0].x_pre, ws[0].x_post)
+        r1 = pipe.submit(ws[1].x, ws[1].x_pre, ws[1].x_post)
+        pipe.synchronize()
+        compare_result(r0, *cpu[0], ws[0].seqlens, budget)
+        compare_result(r1, *cpu[1], ws[1].seqlens, budget)
+        order = [2, 0, 1, 2, 2, 1, 0, 2, 1]
+        rs = [pipe.submit(ws[i].x, ws[i].x_pre, ws[i].x_post) for i in order]
+        pipe.synchronize()
+        compare_result(rs[-2], *cpu[order[-2]], ws[0].seqlens, budget)
+        compare_result(rs[-1], *cpu[order[-1]], ws[0].seqlens, budget)
+    finally:
+        pipe.close()
 
 
 # ---------------------------------------------------------------- edge cases
