@@ -304,8 +304,8 @@ def run_ours(args, world, rank, local):
     barrier()
     torch.cuda.synchronize()
     start.record(pipe.score_stream)
-    for i in range(args.steps):
-        pipe.submit(w.x, w.x_pre, w.x_post, score_events=evs[i])
+    for i in range(args.steps):  # the inputs stay resident and unchanged
+        pipe.submit(w.x, w.x_pre, w.x_post, score_events=evs[i], after_current=False)
     pipe.wait(pipe.score_stream)
     end.record(pipe.score_stream)
     torch.cuda.synchronize()
@@ -340,10 +340,13 @@ def run_ours(args, world, rank, local):
     score_ms = statistics.mean(t_score)
     achieved = in_bytes / (score_ms * 1e-3) / 1e9
     tpr = _traffic_per_row(args.workload)
+    alone_gbs = in_bytes / (alone["k_score"] * 1e-3) / 1e9
     roofline = {"bound": "hbm", "kernel": "k_score", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "peak_source": f"{peak_kind} copy bandwidth",
                 "traffic": None if tpr is None else tpr * total_rows,
-                "algorithmic_bytes": in_bytes}
+                "algorithmic_bytes": in_bytes,
+                "note": "in the timed region k_score shares HBM with the previous step's k_gather (pipeline)",
+                "alone": {"achieved": alone_gbs, "frac": alone_gbs / peak}}
     path_gbs = alg_bytes / (ms_step * 1e-3) / 1e9  # per GPU: every rank moves its own batch
 
     line = {

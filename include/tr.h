@@ -229,10 +229,11 @@ tr_status tr_reduce_noalloc(const tr_tokens *in, const int32_t *d_k, const int32
  * The pipeline owns 2 x slots CUDA events, created on the current device by
  * tr_pipeline_create (make it the device of both streams) and destroyed by
  * tr_pipeline_destroy; it allocates no device memory and never synchronises.
- *   tr_pipeline_submit: arguments as in tr_reduce; score_begin / score_end
- *     are optional cudaEvent_t (or NULL) recorded on score_stream right
- *     before and after the score kernel, to time it.  Host-detectable errors
- *     are returned before anything is enqueued.
+ *   tr_pipeline_submit: arguments as in tr_reduce, except that d_status is
+ *     zeroed by the call itself (on select_stream, before the selection);
+ *     score_begin / score_end are optional cudaEvent_t (or NULL) recorded on
+ *     score_stream right before and after the score kernel, to time it.
+ *     Host-detectable errors are returned before anything is enqueued.
  *   tr_pipeline_wait: makes `stream` wait for every submission so far.
  */
 #define TR_PIPELINE_MAX_SLOTS 8

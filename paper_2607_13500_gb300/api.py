@@ -328,15 +328,16 @@ class Pipeline:
             self._handle = handle
         return self._tok
 
-    def submit(self, x, x_pre, x_post, score_events=None) -> ReduceResult:
+    def submit(self, x, x_pre, x_post, score_events=None, after_current=True) -> ReduceResult:
         """Enqueues one batch; ``score_events`` (two torch.cuda.Event, or
-        None) are recorded on score_stream around the score kernel."""
+        None) are recorded on score_stream around the score kernel.  With
+        ``after_current`` the scoring waits for the work already queued on
+        the caller's current stream (where the inputs were written); pass
+        False when the inputs are known to be ready."""
         tok = self._bind(x, x_pre, x_post)
         o = self.outs[self.submitted % self.slots]
-        # the inputs come from the caller's stream; the status words start at zero
-        self.score_stream.wait_stream(torch.cuda.current_stream(self.device))
-        with torch.cuda.stream(self.select_stream):
-            o["status"].zero_()
+        if after_current:
+            self.score_stream.wait_stream(torch.cuda.current_stream(self.device))
         ev = [None, None]
         if score_events is not None:
             for e in score_events:

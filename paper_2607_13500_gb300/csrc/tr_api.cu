@@ -250,6 +250,8 @@ tr_status tr_pipeline_submit(tr_pipeline *p, const tr_tokens *in, const int32_t 
   if (score_end && cudaEventRecord(static_cast<cudaEvent_t>(score_end), a) != cudaSuccess) return TR_ERR_CUDA;
   if (cudaEventRecord(p->scored[slot], a) != cudaSuccess || cudaStreamWaitEvent(b, p->scored[slot], 0) != cudaSuccess)
     return TR_ERR_CUDA;
+  if (d_status && cudaMemsetAsync(d_status, 0, TR_STATUS_WORDS * sizeof(int32_t), b) != cudaSuccess)
+    return TR_ERR_CUDA;
   if ((rc = tr_select(in, stats, d_k, d_k1, d_cu_k, idx, nullptr, h2, s, ws, p->ws_bytes, d_status, b)) != TR_OK)
     return rc;
   if ((rc = tr_gather(in, d_cu_k, idx, total_k, y, b)) != TR_OK) return rc;
