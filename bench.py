@@ -61,6 +61,10 @@ def _args():
     ap.add_argument("--workload", default="llava576", choices=sorted(BUDGETS))
     ap.add_argument("--batch", type=int, default=None, help="override the workload's batch")
     ap.add_argument("--seed", type=int, default=0)
+    ap.add_argument("--per-frame", action="store_true",
+                    help="video6272: select per 196-token frame instead of per 32-frame clip")
+    ap.add_argument("--stride", choices=["alg1", "interval"], default="alg1",
+                    help="diversity pick positions: Algorithm 1's integer stride or Section IV-B's real interval")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     a = ap.parse_args()
@@ -109,11 +113,14 @@ def _workload_config(w, budget, args):
     ks_desc = f"K={budget['k']}" if "k" in budget else f"ratio={budget['ratio'][0]}/{budget['ratio'][1]}"
     n = f"{min(w.seqlens)}-{max(w.seqlens)}" if len(set(w.seqlens)) > 1 else str(w.seqlens[0])
     dt = "bf16" if w.x.dtype == torch.bfloat16 else "f32"
+    extra = "".join([", per-frame budgets" if getattr(args, "per_frame", False) else "",
+                     ", interval stride" if getattr(args, "stride", "alg1") == "interval" else ""])
     return {
-        "workload": f"{w.name}: B={w.batch}, N={n}, D={w.d}, {dt}, {ks_desc}, lambda=1/3",
+        "workload": f"{w.name}: B={w.batch}, N={n}, D={w.d}, {dt}, {ks_desc}, lambda=1/3{extra}",
         "batch": w.batch, "n": n, "d": w.d, "input_dtype": dt, **({"k": budget["k"]} if "k" in budget else
                                                                  {"ratio": list(budget["ratio"])}),
-        "lambda": "1/3",
+        "lambda": "1/3", "stride": getattr(args, "stride", "alg1"),
+        "budget_unit": "frame" if getattr(args, "per_frame", False) else "image",
     }
 
 
@@ -272,8 +279,10 @@ def run_ours(args, world, rank, local):
     budget = BUDGETS[args.workload]
     over = {"batch": args.batch} if args.batch else {}
     w = synth.make(args.workload, seed=rank_seed(args.seed, rank), device=dev, **over)
-    red = altr.Reducer(w.seqlens, w.d, w.x.dtype, dev, **budget)
-    pipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, slots=2, **budget)
+    if args.per_frame:
+        w = w.frames()
+    red = altr.Reducer(w.seqlens, w.d, w.x.dtype, dev, stride=args.stride, **budget)
+    pipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, slots=2, stride=args.stride, **budget)
     e = 2 if w.x.dtype == torch.bfloat16 else 4
     total_rows = w.total
     in_bytes = 3 * total_rows * w.d * e

@@ -75,7 +75,19 @@ typedef struct {
   const int32_t *cu_seqlens;  /* device int32[batch+1] row offsets, or NULL                         */
   int32_t total;              /* total rows T (ragged: must equal cu_seqlens[batch])                */
   int32_t max_n;              /* ragged: max_b N_b (host-known); ignored when uniform              */
+  int32_t flags;              /* selection options, 0 or TR_STRIDE_INTERVAL                         */
 } tr_tokens;
+
+/*
+ * Positions of the diversity picks along X_rem sorted by s (M = |X_rem|):
+ *   flags = 0:                  Algorithm 1, the integer stride
+ *                               t = max(1, floor(M / K2)): 0, t, ..., (K2-1) t;
+ *   flags = TR_STRIDE_INTERVAL: the fixed interval (N - |X_imp|) / K2 = M / K2
+ *                               of Section IV-B taken as a real number:
+ *                               floor(j M / K2) for j < K2.
+ * Both pick K2 distinct positions; they agree whenever K2 divides M.
+ */
+#define TR_STRIDE_INTERVAL 1
 
 /* Name of a status code (static string). */
 const char *tr_status_string(int32_t status);

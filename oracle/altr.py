@@ -17,7 +17,9 @@ What it computes, step by step in the order of Algorithm 1:
 6. s_i = x'_i . x''_i / (||x'_i|| ||x''_i||)                 (Eq. 6)
 7. sort X_rem by s ascending                                 (Section IV-B, Alg. 1)
 8. t = max(1, floor(|X_rem| / K2)); take sorted positions
-   0, t, 2t, ... up to K2 tokens (the 1-based 1, 1+t, ... of Alg. 1)
+   0, t, 2t, ... up to K2 tokens (the 1-based 1, 1+t, ... of Alg. 1);
+   or, as the text of Section IV-B states it, a fixed real interval
+   |X_rem| / K2: positions floor(j |X_rem| / K2), j < K2
 9. X* = X_imp union X_div, returned in ascending token order (Eq. 7)
 
 Readings of points the paper leaves open (each is listed in the design doc):
@@ -75,6 +77,24 @@ def budget_from_ratio(n: int, ratio):
 def stride(n_rem: int, k2: int) -> int:
     """t = max(1, floor(|X_rem| / K2)) (Algorithm 1)."""
     return max(1, n_rem // k2)
+
+
+def pick_positions(n_rem: int, k2: int, mode: str = "alg1") -> np.ndarray:
+    """0-based positions of X_div along X_rem sorted by s.
+
+    ``"alg1"``: Algorithm 1's integer stride, 0, t, 2t, ..., (K2 - 1) t.
+    ``"interval"``: the fixed interval (N - |X_imp|) / K2 = |X_rem| / K2 of
+    Section IV-B taken as a real number: sample j sits at the real position
+    j |X_rem| / K2 and takes the sorted token at its floor, j < K2.
+    """
+    if k2 == 0:
+        return np.zeros(0, dtype=np.int64)
+    j = np.arange(k2, dtype=np.int64)
+    if mode == "alg1":
+        return j * stride(n_rem, k2)
+    if mode == "interval":
+        return (j * n_rem) // k2
+    raise ValueError(f"unknown stride mode {mode!r}")
 
 
 # --------------------------------------------------------------------------
@@ -187,12 +207,13 @@ def _order(values: np.ndarray, exact_key, descending: bool) -> np.ndarray:
 # --------------------------------------------------------------------------
 # Steps 4-9: one image (Algorithm 1)
 # --------------------------------------------------------------------------
-def select_image(x, x_pre, x_post, k: int, k1: int) -> dict:
+def select_image(x, x_pre, x_post, k: int, k1: int, stride_mode: str = "alg1") -> dict:
     """Run Algorithm 1 on one image: x, x', x'' are [N, D] arrays.
 
     Returns a dict with ``imp`` (importance tokens, in H2 order), ``div``
     (diversity tokens, in pick order), ``kept`` (ascending token indices),
-    ``h2``, ``s`` and the stride ``t``.
+    ``h2``, ``s`` and the stride ``t``.  ``stride_mode`` chooses the
+    positions of X_div (see ``pick_positions``).
     """
     x = np.asarray(x, dtype=np.float64)
     n = x.shape[0]
@@ -209,7 +230,7 @@ def select_image(x, x_pre, x_post, k: int, k1: int) -> dict:
     rem_sorted = rem[_order(s[rem], lambda j: exact_sigma(xp[rem[j]], xq[rem[j]]), descending=False)]
     if k2 > 0:
         t = stride(len(rem), k2)
-        div = rem_sorted[np.arange(k2) * t]
+        div = rem_sorted[pick_positions(len(rem), k2, stride_mode)]
     else:
         t = 0
         div = np.zeros(0, dtype=np.int64)
@@ -217,7 +238,7 @@ def select_image(x, x_pre, x_post, k: int, k1: int) -> dict:
     return dict(imp=imp, div=div, kept=kept, h2=h2, s=s, t=t, rem_sorted=rem_sorted)
 
 
-def reduce_batch(x, x_pre, x_post, seqlens, ks, k1s):
+def reduce_batch(x, x_pre, x_post, seqlens, ks, k1s, stride_mode="alg1"):
     """Algorithm 1 per image over a packed [T, D] batch.
 
     Returns (idx, cu_k, rows): ``idx`` int32 local kept indices ascending per
@@ -227,7 +248,7 @@ def reduce_batch(x, x_pre, x_post, seqlens, ks, k1s):
     idx, rows, cu_k = [], [], [0]
     off = 0
     for n, k, k1 in zip(seqlens, ks, k1s):
-        r = select_image(x[off:off + n], x_pre[off:off + n], x_post[off:off + n], k, k1)
+        r = select_image(x[off:off + n], x_pre[off:off + n], x_post[off:off + n], k, k1, stride_mode)
         idx.append(r["kept"].astype(np.int32))
         rows.append(r["kept"].astype(np.int64) + off)
         cu_k.append(cu_k[-1] + k)

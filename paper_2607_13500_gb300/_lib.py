@@ -10,6 +10,8 @@ LIB_PATH = os.path.join(_HERE, "libtr.so")
 HEADER = os.path.join(os.path.dirname(_HERE), "include", "tr.h")
 
 TR_F32, TR_BF16 = 0, 1
+TR_STRIDE_INTERVAL = 1
+STRIDE_MODES = {"alg1": 0, "interval": TR_STRIDE_INTERVAL}
 TR_STATS_WORDS = 8
 TR_STATUS_WORDS = 4
 TR_MAX_N = 16384
@@ -30,6 +32,7 @@ class TrTokens(ctypes.Structure):
         ("cu_seqlens", ctypes.c_void_p),
         ("total", ctypes.c_int32),
         ("max_n", ctypes.c_int32),
+        ("flags", ctypes.c_int32),
     ]
 
 

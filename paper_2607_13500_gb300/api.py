@@ -12,7 +12,7 @@ from dataclasses import dataclass
 import torch
 
 from . import _lib
-from ._lib import TR_BF16, TR_F32, TR_STATS_WORDS, TR_STATUS_WORDS, TrTokens, check, load
+from ._lib import STRIDE_MODES, TR_BF16, TR_F32, TR_STATS_WORDS, TR_STATUS_WORDS, TrTokens, check, load
 
 _I32 = ctypes.c_int32
 
@@ -64,8 +64,10 @@ def _flatten(x, x_pre, x_post, seqlens):
 class _Tokens:
     """A TrTokens struct plus the device tensors it points into."""
 
-    def __init__(self, x, x_pre, x_post, seqlens):
+    def __init__(self, x, x_pre, x_post, seqlens, stride="alg1"):
         self.x, self.x_pre, self.x_post, self.seqlens = x, x_pre, x_post, seqlens
+        if stride not in STRIDE_MODES:
+            raise ValueError(f"stride must be one of {sorted(STRIDE_MODES)}")
         uniform = len(set(seqlens)) <= 1
         self.cu = None
         if not uniform:
@@ -78,7 +80,7 @@ class _Tokens:
             dtype=_dtype_code(x), d=x.shape[1], batch=len(seqlens),
             n=seqlens[0] if (uniform and seqlens) else 0,
             cu_seqlens=None if self.cu is None else self.cu.data_ptr(),
-            total=x.shape[0], max_n=max(seqlens) if seqlens else 0)
+            total=x.shape[0], max_n=max(seqlens) if seqlens else 0, flags=STRIDE_MODES[stride])
 
     def ref(self):
         return ctypes.byref(self.s)
@@ -121,13 +123,16 @@ def _workspace(lib, tok, device):
     return ws, nbytes
 
 
-def select(x, x_pre, x_post, stats, k=None, ratio=None, lam=(1, 3), seqlens=None, h2=None, s=None, budget=None):
+def select(x, x_pre, x_post, stats, k=None, ratio=None, lam=(1, 3), seqlens=None, h2=None, s=None, budget=None,
+           stride="alg1"):
     """tr_select: returns (idx int32 [sum K], role uint8 [T], cu_k list, status int32 [4]).
 
-    ``budget`` may pass explicit (ks, k1s, cu_k) lists instead of k/ratio/lam."""
+    ``budget`` may pass explicit (ks, k1s, cu_k) lists instead of k/ratio/lam;
+    ``stride`` is "alg1" (Algorithm 1) or "interval" (Section IV-B's real
+    interval, TR_STRIDE_INTERVAL)."""
     lib = load()
     x, x_pre, x_post, seqlens = _flatten(x, x_pre, x_post, seqlens)
-    tok = _Tokens(x, x_pre, x_post, seqlens)
+    tok = _Tokens(x, x_pre, x_post, seqlens, stride)
     ks, k1s, cu_k = budget if budget is not None else budgets(seqlens, k, ratio, lam)
     dev = x.device
     d_k = torch.tensor(ks, dtype=torch.int32, device=dev)
@@ -161,11 +166,11 @@ class Reducer:
     """
 
     def __init__(self, seqlens, d, dtype, device, k=None, ratio=None, lam=(1, 3), alias_pre=False, scores=False,
-                 budget=None):
+                 budget=None, stride="alg1"):
         self.lib = load()
         self.seqlens = [int(v) for v in seqlens]
         self.device = torch.device(device)
-        self.d, self.dtype, self.alias_pre = d, dtype, alias_pre
+        self.d, self.dtype, self.alias_pre, self.stride = d, dtype, alias_pre, stride
         self.ks, self.k1s, self.cu_k = budget if budget is not None else budgets(self.seqlens, k, ratio, lam)
         self.total_k = self.cu_k[-1]
         t = sum(self.seqlens)
@@ -186,7 +191,7 @@ class Reducer:
         x, x_pre, x_post, _ = _flatten(x, x_pre, x_post, self.seqlens)
         key = (x.data_ptr(), None if x_pre is None else x_pre.data_ptr(), x_post.data_ptr())
         if self._tok is None or self._in != key:
-            self._tok = _Tokens(x, x_pre, x_post, self.seqlens)
+            self._tok = _Tokens(x, x_pre, x_post, self.seqlens, self.stride)
             self._in = key
             if self._ws is None:
                 self._ws, self._ws_bytes = _workspace(self.lib, self._tok, self.device)
@@ -282,11 +287,11 @@ class Pipeline:
     """
 
     def __init__(self, seqlens, d, dtype, device, k=None, ratio=None, lam=(1, 3), alias_pre=False, scores=False,
-                 budget=None, slots=2):
+                 budget=None, slots=2, stride="alg1"):
         self.lib = load()
         self.seqlens = [int(v) for v in seqlens]
         self.device = torch.device(device)
-        self.d, self.dtype, self.alias_pre, self.slots = d, dtype, alias_pre, int(slots)
+        self.d, self.dtype, self.alias_pre, self.slots, self.stride = d, dtype, alias_pre, int(slots), stride
         self.ks, self.k1s, self.cu_k = budget if budget is not None else budgets(self.seqlens, k, ratio, lam)
         self.total_k = self.cu_k[-1]
         t = sum(self.seqlens)
@@ -311,7 +316,7 @@ class Pipeline:
         x, x_pre, x_post, _ = _flatten(x, x_pre, x_post, self.seqlens)
         key = (x.data_ptr(), None if x_pre is None else x_pre.data_ptr(), x_post.data_ptr())
         if self._tok is None or self._in != key:
-            self._tok = _Tokens(x, x_pre, x_post, self.seqlens)
+            self._tok = _Tokens(x, x_pre, x_post, self.seqlens, self.stride)
             self._in = key
         if self._handle is None:
             nbytes = self.lib.tr_workspace_bytes(self._tok.ref())
@@ -373,10 +378,12 @@ class Pipeline:
             pass
 
 
-def reduce(x, x_pre, x_post, k=None, ratio=None, lam=(1, 3), seqlens=None, scores=False, budget=None):
-    """tr_reduce in one call: returns a ReduceResult (device tensors)."""
+def reduce(x, x_pre, x_post, k=None, ratio=None, lam=(1, 3), seqlens=None, scores=False, budget=None,
+           stride="alg1"):
+    """tr_reduce in one call: returns a ReduceResult (device tensors).
+    ``stride`` is "alg1" (Algorithm 1) or "interval" (Section IV-B)."""
     x2, p2, q2, seqlens = _flatten(x, x_pre, x_post, seqlens)
     r = Reducer(seqlens, x2.shape[1], x2.dtype, x2.device, k=k, ratio=ratio, lam=lam, alias_pre=p2 is None,
-                scores=scores, budget=budget)
+                scores=scores, budget=budget, stride=stride)
     out = r.run(x2, p2, q2)
     return out

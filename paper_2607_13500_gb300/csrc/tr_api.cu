@@ -20,6 +20,7 @@ struct Shape {
 tr_status check_tokens(const tr_tokens *in, Shape *sh) {
   if (!in || !in->x || !in->x_post) return TR_ERR_ARG;
   if (in->dtype != TR_F32 && in->dtype != TR_BF16) return TR_ERR_DTYPE;
+  if (in->flags & ~TR_STRIDE_INTERVAL) return TR_ERR_ARG;
   if (in->d <= 0 || in->batch < 0) return TR_ERR_ARG;
   if (in->d > TR_MAX_D) return TR_ERR_UNSUPPORTED;
   if ((in->d * elem_bytes(in->dtype)) % 16 != 0) return TR_ERR_ALIGN;
@@ -68,6 +69,7 @@ SelectArgs select_args(const tr_tokens *in, const Shape &sh, const float *stats,
   a.status = d_status;
   a.bounds = certification_bounds(in->d, in->dtype);
   a.max_n = sh.max_n;
+  a.stride_interval = (in->flags & TR_STRIDE_INTERVAL) != 0;
   return a;
 }
 

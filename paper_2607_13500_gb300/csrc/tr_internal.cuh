@@ -143,6 +143,7 @@ struct SelectArgs {
   int32_t *status;    // or NULL
   Bounds bounds;
   int max_n;
+  bool stride_interval;  // diversity picks at floor(j M / K2) instead of j t
 };
 
 size_t select_smem_bytes(int max_n);  // dynamic shared memory of one select CTA

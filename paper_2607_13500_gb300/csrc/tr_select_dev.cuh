@@ -1235,6 +1235,20 @@ __host__ __device__ inline int row_capacity(int max_n) { return (max_n + 15) / 1
 
 // ---------------------------------------------------------------- one image
 // Algorithm 1 for image b, by the whole CTA (kSelectThreads threads);
+// Sorted position of diversity pick j < K2 among the M rows of X_rem:
+// Algorithm 1's integer stride j t, or the real interval M / K2 of
+// Section IV-B, floor(j M / K2).
+__device__ __forceinline__ int pick_position(int j, int m, int k2, int t, bool interval) {
+  return interval ? (int)((long long)j * m / k2) : j * t;
+}
+// Whether sorted position q of X_rem is one of the K2 picks.  For the
+// interval the first pick at or after q is j = ceil(q K2 / M).
+__device__ __forceinline__ bool is_pick(int q, int m, int k2, int t, bool interval) {
+  if (!interval) return q % t == 0 && q / t < k2;
+  const long long j = ((long long)q * k2 + m - 1) / m;
+  return j < k2 && (j * m) / k2 == q;
+}
+
 // smem holds select_smem_bytes(a.max_n) bytes.  Reads the statistics through
 // L2 so that rows scored by other CTAs of the same launch are seen.  Leaves
 // the K kept local indices, ascending, in the second order buffer of smem
@@ -1426,7 +1440,7 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
     const uint16_t *ord = sort_rows(key, ia, ib, bid, m, hist, false);
     const int t = max(1, m / k2);
     for (int j = tid; j < k2; j += nthr) {
-      const int p = j * t;
+      const int p = pick_position(j, m, k2, t, a.stride_interval);
       const bool c0 = p == 0 || cert_s(key, ord, p, a.bounds);
       const bool c1 = p + 1 >= m || cert_s(key, ord, p + 1, a.bounds);
       if (c0 && c1) {
@@ -1465,8 +1479,7 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
           c = cmp_s(rec[r2], rec[r]);
         if (c < 0 || (c == 0 && r2 < r)) ++rank;
       }
-      const int pp = lo + rank;
-      if (pp % t == 0 && pp / t < k2) fl[r] |= F_DIV;
+      if (is_pick(lo + rank, m, k2, t, a.stride_interval)) fl[r] |= F_DIV;
     }
     __syncthreads();
   }

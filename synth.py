@@ -84,6 +84,16 @@ class Workload:
             cu.append(cu[-1] + n)
         return torch.tensor(cu, dtype=torch.int32, device=device or self.x.device)
 
+    def frames(self) -> "Workload":
+        """The same tokens with every frame of a video workload as its own
+        image (per-frame budgets instead of per-clip ones)."""
+        ft = self.meta["spec"].get("frame_tokens")
+        if not ft or any(n % ft for n in self.seqlens):
+            raise ValueError(f"{self.name} has no frames")
+        seqlens = [ft] * (sum(self.seqlens) // ft)
+        return Workload(name=self.name, x=self.x, x_pre=self.x_pre, x_post=self.x_post, seqlens=seqlens,
+                        k=self.k, ratio=self.ratio, lam=self.lam, meta=dict(self.meta, per_frame=True))
+
     def image(self, b: int):
         """Rows of image ``b`` as (x, x_pre, x_post) views."""
         off = sum(self.seqlens[:b])

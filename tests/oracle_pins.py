@@ -156,8 +156,38 @@ def pin_budgets_floor_and_stride():
         [12, 4, 1, 1, 12]
 
 
+def pin_interval_positions():
+    """The text's fixed interval |X_rem| / K2 (Section IV-B) as a real step:
+    K2 distinct positions inside X_rem starting at 0; below every cut x of
+    the sorted list sit exactly ceil(x K2 / |X_rem|) picks (uniform sampling
+    along the list, counted here one position at a time); it is Algorithm 1's
+    integer stride whenever K2 divides |X_rem|; hand values for the shapes of
+    the configs."""
+    rng = _rng(29)
+    pairs = [(555, 43), (512, 128), (6011, 523), (2827, 107), (3, 3), (7, 1), (1, 1)]
+    pairs += [(int(m), int(rng.integers(1, m + 1))) for m in rng.integers(1, 400, 40)]
+    for m, k2 in pairs:
+        pos = oracle.pick_positions(m, k2, "interval").tolist()
+        assert len(pos) == k2 and pos[0] == 0 and pos[-1] < m, (m, k2)
+        assert all(b > a for a, b in zip(pos, pos[1:])), (m, k2)
+        picked = set(pos)
+        below = 0
+        for x in range(m + 1):
+            assert below == -(-x * k2 // m), (m, k2, x)
+            if x < m and x in picked:
+                below += 1
+        if m % k2 == 0:
+            assert pos == oracle.pick_positions(m, k2, "alg1").tolist(), (m, k2)
+    # K = 64 on N = 576: K1 = 21, |X_rem| = 555, K2 = 43 (interval 12.9 vs stride 12);
+    # video clips: N = 6272, K = 784: |X_rem| = 6011, K2 = 523 (interval 11.49 vs stride 11)
+    assert oracle.pick_positions(555, 43, "interval")[-1] == 542
+    assert oracle.pick_positions(555, 43, "alg1")[-1] == 504
+    assert oracle.pick_positions(6011, 523, "interval")[-1] == 5999
+    assert oracle.pick_positions(6011, 523, "alg1")[-1] == 5742
+
+
 # ---------------------------------------------------------------- Algorithm 1, brute force
-def _brute_select(x, xp, xq, k, lam):
+def _brute_select(x, xp, xq, k, lam, mode="alg1"):
     """Independent O(N^2) rank-count implementation with exact rationals.
 
     Importance: token i is in X_imp when fewer than K1 tokens beat it
@@ -186,10 +216,15 @@ def _brute_select(x, xp, xq, k, lam):
         sig[i] = Fraction(0) if aa == 0 or bb == 0 else (1 if p > 0 else -1) * p * p / (aa * bb)
     div = set()
     if k2:
-        t = max(1, len(rem) // k2)
+        m = len(rem)
+        t = max(1, m // k2)
         for i in rem:
             pos = sum(1 for j in rem if sig[j] < sig[i] or (sig[j] == sig[i] and j < i))
-            if pos % t == 0 and pos // t < k2:
+            if mode == "alg1":
+                hit = pos % t == 0 and pos // t < k2
+            else:  # a sample of the interval m / k2 falls in [pos, pos + 1)
+                hit = Fraction((pos + 1) * k2, m).__ceil__() > Fraction(pos * k2, m).__ceil__()
+            if hit:
                 div.add(i)
     return imp, div
 
@@ -213,11 +248,12 @@ def pin_select_brute_force_tiny():
         k = int(rng.integers(0, n + 1))
         lam = [(1, 3), (1, 2), (0, 1), (1, 1), (2, 3)][trial % 5]
         k1, _ = oracle.budget_split(k, lam)
-        got = oracle.select_image(x, xp, xq, k, k1)
-        imp, div = _brute_select(x, xp, xq, k, lam)
-        assert set(got["imp"].tolist()) == imp, (trial, got["imp"], imp)
-        assert set(got["div"].tolist()) == div, (trial, got["div"], div)
-        assert got["kept"].tolist() == sorted(imp | div)
+        for mode in ("alg1", "interval"):
+            got = oracle.select_image(x, xp, xq, k, k1, mode)
+            imp, div = _brute_select(x, xp, xq, k, lam, mode)
+            assert set(got["imp"].tolist()) == imp, (trial, mode, got["imp"], imp)
+            assert set(got["div"].tolist()) == div, (trial, mode, got["div"], div)
+            assert got["kept"].tolist() == sorted(imp | div)
 
 
 # ---------------------------------------------------------------- Algorithm 1, properties

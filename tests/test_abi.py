@@ -73,6 +73,8 @@ def test_host_argument_checks(lib):
     assert r(_tok(d=20000)) == 7
     assert r(_tok(n=20000)) == 7
     assert r(_tok(n=-1)) == 1
+    assert r(_tok(flags=2)) == 1           # unknown selection option
+    assert r(_tok(flags=-1)) == 1
     assert lib.tr_score(ctypes.byref(_tok()), None, None, None, None) == 1
     assert lib.tr_score(ctypes.byref(_tok()), ctypes.c_void_p(0x30004), None, None, None) == 4
     # workspace checks of tr_select / tr_reduce come before any launch

@@ -25,8 +25,9 @@ MUTANTS = {
                              "imp_order = _order(h2, lambda i: exact_r(x[i]), descending=False)"),
     "consistency_sorted_descending": ("exact_sigma(xp[rem[j]], xq[rem[j]]), descending=False)",
                                       "exact_sigma(xp[rem[j]], xq[rem[j]]), descending=True)"),
-    "stride_picks_interval_ends": ("div = rem_sorted[np.arange(k2) * t]",
-                                   "div = rem_sorted[np.arange(1, k2 + 1) * t - 1]"),
+    "stride_picks_interval_ends": ("return j * stride(n_rem, k2)", "return (j + 1) * stride(n_rem, k2) - 1"),
+    "interval_ceil_not_floor": ("return (j * n_rem) // k2", "return -((-j * n_rem) // k2)"),
+    "interval_rounded": ("return (j * n_rem) // k2", "return np.round(j * n_rem / k2).astype(np.int64)"),
     "stride_rounded": ("return max(1, n_rem // k2)", "return max(1, round(n_rem / k2))"),
     "k1_rounded_up": ("k1 = (k * num) // den", "k1 = -((-k * num) // den)"),
     "ratio_rounded": ("return max(1, (n * num) // den)", "return max(1, round(n * num / den))"),

@@ -39,18 +39,20 @@ def _bits(t):
     return t.view(torch.int16) if t.dtype == torch.bfloat16 else t.view(torch.int32)
 
 
-def check_reduce(x, x_pre, x_post, seqlens, budget, images=None, alias=False, expect_nonfinite=False):
+def check_reduce(x, x_pre, x_post, seqlens, budget, images=None, alias=False, expect_nonfinite=False,
+                 stride="alg1"):
     """Runs tr_reduce on the device and compares sampled images with the oracle."""
     altr = _alt()
     dev = torch.device("cuda")
     dx, dq = x.to(dev), x_post.to(dev)
     dp = None if alias else x_pre.to(dev)
-    r = altr.reduce(dx, dp, dq, seqlens=seqlens, budget=budget, scores=True)
+    r = altr.reduce(dx, dp, dq, seqlens=seqlens, budget=budget, scores=True, stride=stride)
     torch.cuda.synchronize()
-    return compare_result(r, x, x_pre, x_post, seqlens, budget, images, alias, expect_nonfinite)
+    return compare_result(r, x, x_pre, x_post, seqlens, budget, images, alias, expect_nonfinite, stride)
 
 
-def compare_result(r, x, x_pre, x_post, seqlens, budget, images=None, alias=False, expect_nonfinite=False):
+def compare_result(r, x, x_pre, x_post, seqlens, budget, images=None, alias=False, expect_nonfinite=False,
+                   stride="alg1"):
     """A ReduceResult (already complete) against the oracle, image by image."""
     ks, k1s, cu = budget
     status = r.status.cpu().tolist()
@@ -68,7 +70,7 @@ def compare_result(r, x, x_pre, x_post, seqlens, budget, images=None, alias=Fals
     for b in images:
         o0, o1 = int(offs[b]), int(offs[b + 1])
         xb, pb, qb = _f64(x[o0:o1]), _f64(pre[o0:o1]), _f64(x_post[o0:o1])
-        ref = oracle.select_image(xb, pb, qb, ks[b], k1s[b])
+        ref = oracle.select_image(xb, pb, qb, ks[b], k1s[b], stride)
         got = idx[cu[b]:cu[b + 1]]
         assert np.array_equal(got, ref["kept"]), (b, np.setdiff1d(got, ref["kept"]), np.setdiff1d(ref["kept"], got))
         want_rows = x[o0:o1][torch.from_numpy(ref["kept"].astype(np.int64))]
@@ -102,6 +104,37 @@ def test_workloads_small(name, over, budgets):
     x, xp, xq = w.x.cpu(), w.x_pre.cpu(), w.x_post.cpu()
     for bk in budgets:
         check_reduce(x, xp, xq, w.seqlens, _budget(w, **bk))
+
+
+@pytest.mark.parametrize("name,over,bud", [
+    ("llava576", dict(batch=4), dict(k=64)),            # |X_rem| = 555, K2 = 43: interval 12.9
+    ("multitile2880", dict(batch=2), dict(k=160)),      # 2827 / 107: interval 26.4
+    ("ragged_dynres", dict(batch=5, n=(256, 3000)), dict(ratio=(1, 9))),
+    ("video6272", dict(batch=2), dict(ratio=(1, 8))),    # 6011 / 523: interval 11.49
+], ids=["llava576", "multitile2880", "ragged_dynres", "video6272"])
+def test_interval_stride(name, over, bud):
+    # Section IV-B's real interval |X_rem| / K2 (TR_STRIDE_INTERVAL), through
+    # the single call and through the pipeline.
+    w = synth.make(name, seed=5, **over)
+    budget = _budget(w, **bud)
+    check_reduce(w.x, w.x_pre, w.x_post, w.seqlens, budget, stride="interval")
+    altr = _alt()
+    dev = torch.device("cuda")
+    pipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, budget=budget, scores=True, stride="interval")
+    try:
+        r = pipe.submit(w.x.to(dev), w.x_pre.to(dev), w.x_post.to(dev))
+        pipe.synchronize()
+        compare_result(r, w.x, w.x_pre, w.x_post, w.seqlens, budget, stride="interval")
+    finally:
+        pipe.close()
+
+
+def test_video_per_frame_budgets():
+    # Every 196-token frame of a clip selected on its own (ratio 1/8: 24 of
+    # 196 tokens per frame) instead of once per 6272-token clip.
+    w = synth.make("video6272", seed=6, batch=1, frames=8).frames()
+    assert w.seqlens == [196] * 8
+    check_reduce(w.x, w.x_pre, w.x_post, w.seqlens, _budget(w, ratio=(1, 8)))
 
 
 def test_lambda_extremes_and_alias():

@@ -1,4 +1,5 @@
 """The seeded input generator: shapes, determinism and recipe features."""
+import pytest
 import torch
 
 import synth
@@ -31,3 +32,11 @@ def test_outliers_and_residual():
     chans = list(synth.OUTLIER_CHANNELS)
     others = [c for c in range(1024) if c not in chans]
     assert w.x_pre[:, chans].abs().max() > 4 * w.x_pre[:, others].abs().max()
+
+
+def test_video_frames_view():
+    w = synth.make("video6272", seed=1, batch=2, frames=4)
+    f = w.frames()
+    assert f.seqlens == [196] * 8 and f.x is w.x and f.total == w.total
+    with pytest.raises(ValueError):
+        synth.make("llava576", batch=1, d=64).frames()
