@@ -299,6 +299,16 @@ def run_ours(args, world, rank, local):
     torch.cuda.synchronize()
     alone = {name: statistics.median(ev[j].elapsed_time(ev[j + 1]) for ev in alone_evs[1:])
              for j, name in enumerate(["k_score", "k_select", "k_gather"])}
+    # latency of one reduction: tr_reduce captured in a CUDA graph, replayed
+    graph = red.graph(w.x, w.x_pre, w.x_post)
+    lat_evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(max(5, args.warmup))]
+    for ev in lat_evs:
+        ev[0].record()
+        graph.replay()
+        ev[1].record()
+    torch.cuda.synchronize()
+    latency_us = 1e3 * statistics.median(ev[0].elapsed_time(ev[1]) for ev in lat_evs[1:])
+    del graph
 
     clocks = ClockSampler(dev)
     for _ in range(args.warmup):
@@ -367,6 +377,7 @@ def run_ours(args, world, rank, local):
         "hbm_gbs": path_gbs, "frac_of_8tbs": path_gbs / NOMINAL_HBM_GBS, "frac_of_measured": path_gbs / peak,
         "kernels_ms": {"k_score_in_pipeline": score_ms, **{f"{k}_alone": v for k, v in alone.items()}},
         "pipeline": "2 slots: step i's k_select + k_gather (high-priority stream) overlap step i+1's k_score",
+        "latency_us": {"tr_reduce_graph_replay": latency_us},
         "roofline": roofline,
         "e2e": {"value": images / e2e_s, "unit": "images/s", "h2d_bytes_per_step": in_bytes,
                 "d2h_bytes_per_step": red.total_k * (w.d * e + 4)},

@@ -30,6 +30,10 @@
  *  - The library keeps no global state besides a per-device "shared memory
  *    limit already raised" flag; calls on different streams may run
  *    concurrently when they use different workspaces.
+ *  - The single-call entry points only enqueue kernels (no allocation,
+ *    synchronisation or copies), so they can be captured into a CUDA graph
+ *    and replayed; make one call on the device outside the capture first
+ *    (it raises the kernels' shared-memory limit once).
  */
 #ifndef TR_H
 #define TR_H

@@ -206,6 +206,18 @@ class Reducer:
         return ReduceResult(self.y[:self.total_k], self.idx[:self.total_k], self.cu_k, self.h2, self.s,
                             self.status)
 
+    def graph(self, x, x_pre, x_post) -> "torch.cuda.CUDAGraph":
+        """``run`` (with the status words zeroed first) captured into a CUDA
+        graph for these input tensors; ``replay()`` repeats it with one
+        launch.  Outputs land in this Reducer's buffers (``y``, ``idx``, ...)."""
+        self.run(x, x_pre, x_post)  # outside the capture first: sets the kernels' shared-memory limit once
+        torch.cuda.synchronize(self.device)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.status.zero_()
+            self.run(x, x_pre, x_post)
+        return g
+
     def run_split(self, x, x_pre, x_post, events=None):
         """The same two kernels as ``run`` through the entry points tr_score
         and tr_select_gather, with ``events`` (three torch.cuda.Event, or

@@ -837,29 +837,18 @@ __device__ uint16_t *radix_sort(const uint32_t *key, uint16_t *a, uint16_t *b, i
 
 // Ascending bitonic sort of kSelectThreads * E composite keys (sort key << 16
 // | row) held E per thread (thread t owns positions t E .. t E + E - 1).
-// Partners closer than E are in the same thread, closer than 32 E in the
-// same warp (register shuffles); only the remaining stages go through
-// shared memory (scratch: kSelectThreads * E words) with block barriers.
+// For each merge size k the stages run with partner distance j = k/2, k/4,
+// ..., 1: distances of at least 32 E go through shared memory (scratch:
+// kSelectThreads * E words) between block barriers, distances of at least E
+// through register shuffles inside a warp, and the last ones (j < E) inside
+// the thread, with compile-time j so that v[] stays in registers.
 template <int E>
 __device__ void bitonic_regs(unsigned long long (&v)[E], unsigned long long *scratch) {
   constexpr int NP = kSelectThreads * E;
   const int t = threadIdx.x, lane = t & 31;
   for (int k = 2; k <= NP; k <<= 1) {
-    for (int j = k >> 1; j > 0; j >>= 1) {
-      if (j < E) {
-#pragma unroll
-        for (int e = 0; e < E; ++e) {
-          const int pe = e ^ j;
-          if (pe > e) {
-            const bool up = ((t * E + e) & k) == 0;
-            const unsigned long long x = v[e], y = v[pe];
-            if ((x > y) == up) {
-              v[e] = y;
-              v[pe] = x;
-            }
-          }
-        }
-      } else if (j < 32 * E) {
+    for (int j = k >> 1; j >= E; j >>= 1) {
+      if (j < 32 * E) {
         const int lm = j / E;
         const bool lower = (lane & lm) == 0;
 #pragma unroll
@@ -880,6 +869,23 @@ __device__ void bitonic_regs(unsigned long long (&v)[E], unsigned long long *scr
           v[e] = ((i < pi) == up) ? min(v[e], o) : max(v[e], o);
         }
         __syncthreads();
+      }
+    }
+#pragma unroll
+    for (int j = E >> 1; j > 0; j >>= 1) {
+      if (j < k) {
+#pragma unroll
+        for (int e = 0; e < E; ++e) {
+          const int pe = e ^ j;
+          if (pe > e) {
+            const bool up = ((t * E + e) & k) == 0;
+            const unsigned long long x = v[e], y = v[pe];
+            if ((x > y) == up) {
+              v[e] = y;
+              v[pe] = x;
+            }
+          }
+        }
       }
     }
   }
@@ -1119,7 +1125,7 @@ __device__ uint16_t *bucket_sort(const uint32_t *key, uint16_t *a, uint16_t *b, 
 }
 
 // Ascending order of the m rows listed in a by (key[row], row), a listed in
-// ascending row order: a register bitonic sort up to 1024 rows; above that
+// ascending row order: a register bitonic sort up to 2048 rows; above that
 // value buckets, the sample sort when the values crowd into few buckets,
 // and the stable radix sort when the sample sort declines too.  Returns the
 // buffer holding the order.
@@ -1135,6 +1141,11 @@ __device__ uint16_t *sort_rows(const uint32_t *key, uint16_t *a, uint16_t *b, ui
   if (m <= 2 * kSelectThreads) {
     __syncthreads();
     sort_small<2>(key, a, m, scratch);
+    return a;
+  }
+  if (m <= 4 * kSelectThreads) {
+    __syncthreads();
+    sort_small<4>(key, a, m, scratch);
     return a;
   }
   if (uint16_t *o = bucket_sort(key, a, b, m, hist, complemented)) return o;

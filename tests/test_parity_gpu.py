@@ -205,6 +205,57 @@ def test_pipeline_overlapped_batches():
         pipe.close()
 
 
+def test_graph_replay_and_limits():
+    # tr_reduce captured in a CUDA graph and replayed; one image at the
+    # largest N (16384 tokens), and rows at the largest D (16384 channels).
+    altr = _alt()
+    dev = torch.device("cuda")
+    w = synth.make("llava576", seed=8, batch=3, d=512)
+    budget = _budget(w, k=100)
+    red = altr.Reducer(w.seqlens, w.d, w.x.dtype, dev, budget=budget, scores=True)
+    dx, dp, dq = w.x.to(dev), w.x_pre.to(dev), w.x_post.to(dev)
+    g = red.graph(dx, dp, dq)
+    red.y.zero_()
+    red.idx.zero_()
+    for _ in range(3):
+        g.replay()
+    torch.cuda.synchronize()
+    res = altr.ReduceResult(red.y[:red.total_k], red.idx[:red.total_k], red.cu_k, red.h2, red.s, red.status)
+    compare_result(res, w.x, w.x_pre, w.x_post, w.seqlens, budget)
+    x, xp, xq = _rows(16384, 32, 21)
+    check_reduce(x, xp, xq, [16384], _alt().budgets([16384], k=1500))
+    x, xp, xq = _rows(40, 16384, 22, dtype=torch.float32)
+    check_reduce(x, xp, xq, [40], _alt().budgets([40], k=12))
+    x, xp, xq = _rows(40, 16384, 23)
+    check_reduce(x, xp, xq, [25, 15], _alt().budgets([25, 15], k=10))
+
+
+def test_pipeline_edge_cases():
+    # one slot and three slots, an empty image and K = 0 images in a ragged
+    # batch, fp32 inputs, and a batch that keeps nothing at all
+    altr = _alt()
+    dev = torch.device("cuda")
+    x, xp, xq = _rows(300, 256, 31, dtype=torch.float32)
+    seqlens = [120, 0, 100, 80]
+    for slots in (1, 3):
+        budget = altr.budgets(seqlens, k=None, ratio=(1, 5))
+        pipe = altr.Pipeline(seqlens, 256, torch.float32, dev, budget=budget, scores=True, slots=slots)
+        try:
+            rs = [pipe.submit(x.to(dev), xp.to(dev), xq.to(dev)) for _ in range(slots + 1)]
+            pipe.synchronize()
+            compare_result(rs[-1], x, xp, xq, seqlens, budget)
+        finally:
+            pipe.close()
+    budget = ([0, 0, 0, 0], [0, 0, 0, 0], [0, 0, 0, 0, 0])
+    pipe = altr.Pipeline(seqlens, 256, torch.float32, dev, budget=budget, scores=True)
+    try:
+        r = pipe.submit(x.to(dev), xp.to(dev), xq.to(dev))
+        pipe.synchronize()
+        assert r.idx.numel() == 0 and r.status.cpu().tolist() == [0, 0, 0, 0]
+    finally:
+        pipe.close()
+
+
 # ---------------------------------------------------------------- edge cases
 def _rows(n, d, seed, dtype=torch.bfloat16):
     g = torch.Generator().manual_seed(seed)
@@ -250,19 +301,21 @@ def test_exact_ties_and_degenerate_rows():
 
 
 def test_sort_paths_uneven_and_tied_keys():
-    # 512 distinct rows at every 4th position and 1536 copies of one row
-    # whose R = 1 (one-hot) is the smallest of all: the importance cut falls
-    # inside the copies (an exact tie), so the full importance order is
-    # needed (value buckets crowd, the sample sort orders them); the rows
-    # left for the consistency order tie in s.
-    n, d = 2048, 64
+    # 750 distinct rows at every 4th position and 2250 copies of one row
+    # whose R = 1 (one-hot) is the smallest of all.  With K1 = 800 the
+    # importance cut falls inside the copies (an exact tie) and the window
+    # around it is too full, so all 3000 rows are ordered: the copies crowd
+    # one value bucket and the stratified sample sort orders them.  The rows
+    # left for the consistency order tie in s (sample sort again); with
+    # K1 = 256 the cut is certain without any order.
+    n, d = 3000, 64
     x, xp, xq = _rows(n, d, 11)
     tied = [i for i in range(n) if i % 4]
     x[tied] = 0
     x[tied, 5] = 1.0
     xp[tied] = xp[1].clone()
     xq[tied] = xq[1].clone()
-    for k, k1 in [(900, 600), (700, 256), (1024, 0)]:
+    for k, k1 in [(1200, 800), (700, 256), (1024, 0)]:
         check_reduce(x, xp, xq, [n], ([k], [k1], [0, k]))
 
 
