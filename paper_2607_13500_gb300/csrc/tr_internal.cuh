@@ -11,7 +11,7 @@
 namespace tr {
 
 // ---------------------------------------------------------------- launch shapes
-constexpr int kScoreWarps = 8;        // rows (one per warp) in flight per score CTA
+constexpr int kScoreWarps = 2;        // rows (one per warp) in flight per score CTA
 constexpr int kScoreBatchBf16 = 8;    // 16-byte chunks a lane loads per stream before it computes (bf16)
 constexpr int kScoreBatchF32 = 8;     // the same for fp32 inputs
 constexpr int kSelectThreads = 512;   // one select CTA per image

@@ -28,10 +28,12 @@ cudaError_t launch_score(const void *x, const void *x_pre, const void *x_post, i
   const unsigned char *bp = static_cast<const unsigned char *>(x_pre ? x_pre : x);
   const unsigned char *bq = static_cast<const unsigned char *>(x_post);
   float4 *ps = reinterpret_cast<float4 *>(stats);
-  // One row per warp and no more: CTAs retire as they finish, so kernels on
-  // other streams (the selection of an earlier batch) can take SMs while
-  // this one still runs.  (A persistent grid of resident CTAs is no faster
-  // alone and would hold every SM to the end.)
+  // One row per warp and no more, in small CTAs: CTAs retire as they
+  // finish, so kernels on other streams (the selection of an earlier batch)
+  // can take SMs while this one still runs, and an SM's slots refill row by
+  // row.  (Measured on GB300: 2-warp CTAs beat 1-, 4-, 8- and 16-warp ones
+  // and 2 or 4 rows per warp; a persistent grid is no faster alone and would
+  // hold every SM to the end.)
   const long long need = (total + kScoreWarps - 1) / kScoreWarps;
   const int grid = (int)(need < INT_MAX ? need : INT_MAX);
   const int nchunks = row_bytes / 16;
