@@ -54,16 +54,23 @@ def check_reduce(x, x_pre, x_post, seqlens, budget, images=None, alias=False, ex
 def compare_result(r, x, x_pre, x_post, seqlens, budget, images=None, alias=False, expect_nonfinite=False,
                    stride="alg1"):
     """A ReduceResult (already complete) against the oracle, image by image."""
+    return compare_results([r], x, x_pre, x_post, seqlens, budget, images, alias, expect_nonfinite, stride)[0]
+
+
+def compare_results(rs, x, x_pre, x_post, seqlens, budget, images=None, alias=False, expect_nonfinite=False,
+                    stride="alg1"):
+    """Several ReduceResults of the same batch against one oracle run per image."""
     ks, k1s, cu = budget
-    status = r.status.cpu().tolist()
-    assert status[1] == 0, f"unresolved rows: {status}"
-    assert status[3] == 0, f"invalid budget or kept-count mismatch: {status}"
-    if expect_nonfinite:
-        assert status[0] > 0
-    idx = r.idx.cpu().numpy()
-    y = r.y.cpu()
-    h2 = r.h2.cpu().numpy().astype(np.float64)
-    s = r.s.cpu().numpy().astype(np.float64)
+    statuses, host = [], []
+    for r in rs:
+        status = r.status.cpu().tolist()
+        assert status[1] == 0, f"unresolved rows: {status}"
+        assert status[3] == 0, f"invalid budget or kept-count mismatch: {status}"
+        if expect_nonfinite:
+            assert status[0] > 0
+        statuses.append(status)
+        host.append((r.idx.cpu().numpy(), r.y.cpu(), r.h2.cpu().numpy().astype(np.float64),
+                     r.s.cpu().numpy().astype(np.float64)))
     offs = np.concatenate([[0], np.cumsum(seqlens)]).astype(np.int64)
     images = range(len(seqlens)) if images is None else images
     pre = x if alias else x_pre
@@ -71,17 +78,19 @@ def compare_result(r, x, x_pre, x_post, seqlens, budget, images=None, alias=Fals
         o0, o1 = int(offs[b]), int(offs[b + 1])
         xb, pb, qb = _f64(x[o0:o1]), _f64(pre[o0:o1]), _f64(x_post[o0:o1])
         ref = oracle.select_image(xb, pb, qb, ks[b], k1s[b], stride)
-        got = idx[cu[b]:cu[b + 1]]
-        assert np.array_equal(got, ref["kept"]), (b, np.setdiff1d(got, ref["kept"]), np.setdiff1d(ref["kept"], got))
         want_rows = x[o0:o1][torch.from_numpy(ref["kept"].astype(np.int64))]
-        assert torch.equal(_bits(y[cu[b]:cu[b + 1]]), _bits(want_rows)), b
         fin = np.isfinite(ref["h2"])
-        rt = H2_RTOL[x.dtype]
-        assert np.all(np.abs(h2[o0:o1][fin] - ref["h2"][fin]) <= rt * np.abs(ref["h2"][fin]) + 1e-6), b
-        assert np.array_equal(np.isneginf(h2[o0:o1][~fin]), np.ones((~fin).sum(), bool))
         sf = np.isfinite(ref["s"])
-        assert np.all(np.abs(s[o0:o1][sf] - ref["s"][sf]) <= S_ATOL), b
-    return status
+        rt = H2_RTOL[x.dtype]
+        for j, (idx, y, h2, s) in enumerate(host):
+            got = idx[cu[b]:cu[b + 1]]
+            assert np.array_equal(got, ref["kept"]), (j, b, np.setdiff1d(got, ref["kept"]),
+                                                      np.setdiff1d(ref["kept"], got))
+            assert torch.equal(_bits(y[cu[b]:cu[b + 1]]), _bits(want_rows)), (j, b)
+            assert np.all(np.abs(h2[o0:o1][fin] - ref["h2"][fin]) <= rt * np.abs(ref["h2"][fin]) + 1e-6), (j, b)
+            assert np.array_equal(np.isneginf(h2[o0:o1][~fin]), np.ones((~fin).sum(), bool)), (j, b)
+            assert np.all(np.abs(s[o0:o1][sf] - ref["s"][sf]) <= S_ATOL), (j, b)
+    return statuses
 
 
 def _budget(w, k=None, ratio=None, lam=(1, 3)):
@@ -387,10 +396,20 @@ FULL = [
 
 @pytest.mark.parametrize("name,bk,sample", FULL, ids=[f[0] for f in FULL])
 def test_workloads_full_size(name, bk, sample):
+    # The full-size batch through tr_reduce and through the two-slot
+    # pipeline bench.py times (three submissions: both slots, then slot 0
+    # again), each checked image by image on the sampled images.
+    altr = _alt()
     w = synth.make(name, seed=0, device="cuda")
     if sample == "largest3":
         sample = sorted(range(w.batch), key=lambda b: -w.seqlens[b])[:2] + [0]
-    x, xp, xq = w.x.cpu(), w.x_pre.cpu(), w.x_post.cpu()
-    del w.x, w.x_pre, w.x_post
-    torch.cuda.empty_cache()
-    check_reduce(x, xp, xq, w.seqlens, _alt().budgets(w.seqlens, **bk), images=sample)
+    budget = altr.budgets(w.seqlens, **bk)
+    single = altr.reduce(w.x, w.x_pre, w.x_post, seqlens=w.seqlens, budget=budget, scores=True)
+    pipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, w.x.device, budget=budget, scores=True, slots=2)
+    try:
+        piped = [pipe.submit(w.x, w.x_pre, w.x_post) for _ in range(3)][-1]
+        pipe.synchronize()
+        x, xp, xq = w.x.cpu(), w.x_pre.cpu(), w.x_post.cpu()
+        compare_results([single, piped], x, xp, xq, w.seqlens, budget, images=sample)
+    finally:
+        pipe.close()
