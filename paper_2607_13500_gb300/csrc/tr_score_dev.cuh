@@ -215,10 +215,38 @@ __device__ __forceinline__ void finish_row(Acc &acc, long long row, float4 *__re
   }
 }
 
+// One round: lane l takes chunks base + l + 32u (u < kB) of each stream,
+// all loads issued before any arithmetic; with kGuard, chunks at or past c1
+// are zeros (which add nothing).
+template <bool kBf16, int kB, bool kGuard>
+__device__ __forceinline__ void accumulate_round(const uint4 *__restrict__ rx, const uint4 *__restrict__ rp,
+                                                 const uint4 *__restrict__ rq, int base, int c1, Acc &acc,
+                                                 Acc2 &acc2, int lane) {
+  uint4 vx[kB], vp[kB], vq[kB];
+#pragma unroll
+  for (int u = 0; u < kB; ++u) {
+    const int c = base + lane + 32 * u;
+    if (!kGuard || c < c1) {
+      vx[u] = ld_stream(rx + c);
+      vp[u] = ld_stream(rp + c);
+      vq[u] = ld_stream(rq + c);
+    } else {
+      vx[u] = vp[u] = vq[u] = make_uint4(0u, 0u, 0u, 0u);
+    }
+  }
+  if (kBf16) {
+#pragma unroll
+    for (int u = 0; u < kB; u += 2) chunk2_bf16(vx[u], vx[u + 1], vp[u], vp[u + 1], vq[u], vq[u + 1], acc2);
+  } else {
+#pragma unroll
+    for (int u = 0; u < kB; ++u) chunk_f32(vx[u], vp[u], vq[u], acc);
+  }
+}
+
 // Partial sums of chunks [c0, c1) of one row, read straight from global
-// memory: in each round lane l takes chunks base + l + 32u (u < the batch) of
-// each stream, all loads issued before any arithmetic; chunks past c1 are
-// zeros, which add nothing.
+// memory in rounds of kB chunks per lane and stream.  When the row's chunks
+// are a multiple of 32 (every lane has the same count) the last round is cut
+// to the chunks that remain (6, 4 or 2 per lane), so no lane works on padding.
 template <bool kBf16>
 __device__ __forceinline__ void accumulate_global(const uint4 *__restrict__ rx, const uint4 *__restrict__ rp,
                                                   const uint4 *__restrict__ rq, int c0, int c1, Acc &acc,
@@ -226,28 +254,18 @@ __device__ __forceinline__ void accumulate_global(const uint4 *__restrict__ rx, 
   constexpr int kB = kBf16 ? kScoreBatchBf16 : kScoreBatchF32;
   static_assert(kB % 2 == 0, "bf16 chunks are summed in pairs");
   Acc2 acc2{};
-  for (int base = c0; base < c1; base += 32 * kB) {
-    uint4 vx[kB], vp[kB], vq[kB];
-#pragma unroll
-    for (int u = 0; u < kB; ++u) {
-      const int c = base + lane + 32 * u;
-      if (c < c1) {
-        vx[u] = ld_stream(rx + c);
-        vp[u] = ld_stream(rp + c);
-        vq[u] = ld_stream(rq + c);
-      } else {
-        vx[u] = vp[u] = vq[u] = make_uint4(0u, 0u, 0u, 0u);
-      }
-    }
-    if (kBf16) {
-#pragma unroll
-      for (int u = 0; u < kB; u += 2)
-        chunk2_bf16(vx[u], vx[u + 1], vp[u], vp[u + 1], vq[u], vq[u + 1], acc2);
-    } else {
-#pragma unroll
-      for (int u = 0; u < kB; ++u)
-        chunk_f32(vx[u], vp[u], vq[u], acc);
-    }
+  int base = c0;
+  for (; base + 32 * kB <= c1; base += 32 * kB) accumulate_round<kBf16, kB, false>(rx, rp, rq, base, c1, acc, acc2, lane);
+  const int rest = c1 - base;
+  if (rest > 0) {
+    if (kB == 8 && rest == 32 * 6)
+      accumulate_round<kBf16, 6, false>(rx, rp, rq, base, c1, acc, acc2, lane);
+    else if (kB == 8 && rest == 32 * 4)
+      accumulate_round<kBf16, 4, false>(rx, rp, rq, base, c1, acc, acc2, lane);
+    else if (rest == 32 * 2)
+      accumulate_round<kBf16, 2, false>(rx, rp, rq, base, c1, acc, acc2, lane);
+    else
+      accumulate_round<kBf16, kB, true>(rx, rp, rq, base, c1, acc, acc2, lane);
   }
   if (kBf16) {
     // Half 0 holds this lane's even-numbered chunks, half 1 its odd ones.
