@@ -189,8 +189,9 @@ tr_status tr_select_gather(const tr_tokens *in, const float *stats, const int32_
                            void *ws, size_t ws_bytes, int32_t *d_status, void *stream);
 
 /*
- * The whole path in one call: tr_score then tr_select_gather on `stream`
- * (two kernel launches), with the statistics kept in the workspace.
+ * The whole path in one call on `stream`, with the statistics kept in the
+ * workspace: tr_score then tr_select_gather for a uniform batch (two kernel
+ * launches); tr_score, tr_select and tr_gather for a ragged one (three).
  *   total_k:  host int, = cu_k[batch] (the number of output rows).
  *   y:        device [total_k, d] in the input dtype, 16-byte aligned.
  *   idx, h2, s, d_status: as in tr_select (role is not produced); h2 and s

@@ -149,7 +149,9 @@ struct SelectArgs {
 size_t select_smem_bytes(int max_n);  // dynamic shared memory of one select CTA
 cudaError_t launch_score(const void *x, const void *x_pre, const void *x_post, int dtype, int d, long long total,
                          float *stats, float *h2, float *s, cudaStream_t st);
-cudaError_t launch_select(const SelectArgs &a, cudaStream_t st);
+// max_ctas > 0 caps the grid (each CTA then selects several images in turn).
+cudaError_t launch_select(const SelectArgs &a, cudaStream_t st, int max_ctas = 0);
+int sm_count();  // SMs of the current device (cached), 0 on error
 cudaError_t launch_select_gather(const SelectArgs &a, void *y, cudaStream_t st);
 cudaError_t launch_gather(const void *x, long long total_rows, int dtype, int d, int batch, int n_uniform,
                           const int32_t *cu_seqlens, const int32_t *cu_k, const int32_t *idx, int total_k, void *y,

@@ -11,9 +11,11 @@
 namespace tr {
 namespace {
 
+// CTA c selects images c, c + gridDim.x, ... (one image per CTA unless the
+// launch caps the grid below the batch).
 __global__ void __launch_bounds__(kSelectThreads, 1) k_select(const SelectArgs a) {
   extern __shared__ __align__(16) unsigned char smem[];
-  select_image(a, blockIdx.x, smem);
+  for (int b = blockIdx.x; b < a.batch; b += gridDim.x) select_image(a, b, smem);
 }
 
 __device__ __forceinline__ uint4 ld_nc16(const uint4 *p) {
@@ -87,7 +89,7 @@ cudaError_t raise_smem_limit(K kernel, int dev) {
   return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, optin - (int)fa.sharedSizeBytes);
 }
 
-cudaError_t launch_select(const SelectArgs &a, cudaStream_t st) {
+cudaError_t launch_select(const SelectArgs &a, cudaStream_t st, int max_ctas) {
   if (a.batch == 0) return cudaSuccess;
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
@@ -97,8 +99,19 @@ cudaError_t launch_select(const SelectArgs &a, cudaStream_t st) {
     if ((err = raise_smem_limit(k_select, dev)) != cudaSuccess) return err;
     g_smem_set[dev & 63] |= 1;
   }
-  k_select<<<a.batch, kSelectThreads, smem, st>>>(a);
+  const int grid = max_ctas > 0 && max_ctas < a.batch ? max_ctas : a.batch;
+  k_select<<<grid, kSelectThreads, smem, st>>>(a);
   return cudaGetLastError();
+}
+
+int sm_count() {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (!g_sms[dev & 63]) {
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+    g_sms[dev & 63] = sms;
+  }
+  return g_sms[dev & 63];
 }
 
 cudaError_t launch_select_gather(const SelectArgs &a, void *y, cudaStream_t st) {
