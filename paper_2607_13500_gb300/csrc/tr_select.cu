@@ -1,11 +1,13 @@
-// The selection kernels: one CTA per image runs select_image (Algorithm 1,
-// see tr_select_dev.cuh) on statistics left by the scoring kernel.
+// The selection kernels: a CTA runs select_image (Algorithm 1, see
+// tr_select_dev.cuh) on statistics left by the scoring kernel, one image at
+// a time (k_select: one image per CTA, or several in turn when the launch
+// caps the grid, as the pipeline does).
 //
-// k_select_gather (tr_reduce) also copies the kept rows.  With fewer images
-// than SMs it runs R replica CTAs per image: each makes the same
-// deterministic selection (only replica 0 writes idx and the status words)
-// and copies its 1/R share of the image's kept rows, so the copies of one
-// image overlap the selections of the others on SMs that would be idle.
+// k_select_gather (tr_reduce on uniform batches) also copies the kept rows.
+// With fewer images than SMs it runs R replica CTAs per image: each makes
+// the same deterministic selection (only replica 0 writes idx and the status
+// words) and copies its 1/R share of the image's kept rows, so the copies of
+// one image overlap the selections of the others on SMs that would be idle.
 #include "tr_select_dev.cuh"
 
 namespace tr {
