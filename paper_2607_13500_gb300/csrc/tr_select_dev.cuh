@@ -53,6 +53,9 @@ __device__ __forceinline__ float unord32(uint32_t o) {
 // fp32 keys from the statistics record; NaN = outside the fp32 error model.
 __device__ __forceinline__ float key_r(const float *st) { return __ldcg(st + 6); }
 __device__ __forceinline__ float key_s(const float *st) { return __ldcg(st + 7); }
+// Both keys in one 8-byte load (records are 32-byte aligned).
+__device__ __forceinline__ float2 key_rs(const float *st) { return __ldcg(reinterpret_cast<const float2 *>(st + 6)); }
+constexpr int kKeyIlp = 4;  // rows whose keys a thread loads before it uses any
 
 // ---- a Big truncated to a 64-bit mantissa: value in [m 2^e, (m + 1) 2^e) ----
 // Integer-only (the GPU's fp64 rate is far too low for this path).
@@ -1299,13 +1302,27 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
   const bool need_s = k2 > 0;
 
   // 1. Rows whose fp32 sums left the error model are settled exactly first
-  //    (also when only their H2 / s outputs need it).
-  for (int i = tid; i < n; i += nthr) {
-    const float *r = st + (long long)i * TR_STATS_WORDS;
-    uint8_t f = 0;
-    if ((need_r || a.h2) && isnan(key_r(r))) f |= F_NEEDL;
-    if ((need_s || a.s) && isnan(key_s(r))) f |= F_NEEDS;
-    fl[i] = f;
+  //    (also when only their H2 / s outputs need it).  The same pass lays
+  //    out the importance keys ~ord32(R32) and the identity order.
+  for (int i0 = tid; i0 < n; i0 += kKeyIlp * nthr) {
+    float2 kk[kKeyIlp];
+#pragma unroll
+    for (int u = 0; u < kKeyIlp; ++u) {
+      const int i = i0 + u * nthr;
+      kk[u] = i < n ? key_rs(st + (long long)i * TR_STATS_WORDS) : make_float2(0.f, 0.f);
+    }
+#pragma unroll
+    for (int u = 0; u < kKeyIlp; ++u) {
+      const int i = i0 + u * nthr;
+      if (i < n) {
+        uint8_t f = 0;
+        if ((need_r || a.h2) && isnan(kk[u].x)) f |= F_NEEDL;
+        if ((need_s || a.s) && isnan(kk[u].y)) f |= F_NEEDS;
+        fl[i] = f;
+        key[i] = ~ord32(kk[u].x);
+        ia[i] = (uint16_t)i;
+      }
+    }
   }
   __syncthreads();
   refine_pending(a, off, n, fl, rec, primary);
@@ -1313,11 +1330,8 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
 
   // 2. Stage I: top-K1 by R (equivalently H2), descending, lower index first.
   if (need_r) {
-    for (int i = tid; i < n; i += nthr) {
-      const float r = (fl[i] & F_XL) ? exact_r_key(rec[i]) : key_r(st + (long long)i * TR_STATS_WORDS);
-      key[i] = ~ord32(r);
-      ia[i] = (uint16_t)i;
-    }
+    for (int i = tid; i < n; i += nthr)  // rows settled exactly carry their exact key
+      if (fl[i] & F_XL) key[i] = ~ord32(exact_r_key(rec[i]));
     __syncthreads();
     // Fast path: the K1-th and (K1+1)-th keys by radix selection; when they
     // differ and their order is certain, the top K1 are exactly the rows
@@ -1437,6 +1451,21 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
 
   // 3. Stage II: sort X_rem by s ascending, pick positions 0, t, 2t, ...
   if (need_s) {
+    // consistency keys ord32(s32) of every row (stage I's keys are no longer
+    // needed; X_imp rows' keys are never read), exact ones for settled rows
+    for (int i0 = tid; i0 < n; i0 += kKeyIlp * nthr) {
+      float sv[kKeyIlp];
+#pragma unroll
+      for (int u = 0; u < kKeyIlp; ++u) {
+        const int i = i0 + u * nthr;
+        sv[u] = i < n ? key_s(st + (long long)i * TR_STATS_WORDS) : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < kKeyIlp; ++u) {
+        const int i = i0 + u * nthr;
+        if (i < n) key[i] = ord32((fl[i] & F_XS) ? exact_s_key(rec[i]) : sv[u]);
+      }
+    }
     // X_rem in ascending index order (the stable sort's tie order)
     const int per = (n + nthr - 1) / nthr;
     const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
@@ -1444,12 +1473,8 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
     for (int i = i0; i < i1; ++i) cnt += !(fl[i] & F_IMP);
     int m = 0;
     int pos = block_exclusive_scan(cnt, &m);
-    for (int i = i0; i < i1; ++i) {
-      if (fl[i] & F_IMP) continue;
-      ia[pos++] = (uint16_t)i;
-      const float sv = (fl[i] & F_XS) ? exact_s_key(rec[i]) : key_s(st + (long long)i * TR_STATS_WORDS);
-      key[i] = ord32(sv);
-    }
+    for (int i = i0; i < i1; ++i)
+      if (!(fl[i] & F_IMP)) ia[pos++] = (uint16_t)i;
     __syncthreads();
     const uint16_t *ord = sort_rows(key, ia, ib, bid, m, hist, false);
     const int t = max(1, m / k2);
