@@ -337,23 +337,26 @@ def run_ours(args, world, rank, local):
     value = job_images_per_s(w.batch, world, ms_step)
     pipe.close()
 
-    # end to end through the public API: pinned host inputs in, y and idx out
+    # end to end through the public API: every step copies its inputs in from
+    # pinned host memory and its y and idx back out (Pipeline.submit_host:
+    # the next step's upload overlaps this step's work and download)
     pin = lambda t: t.cpu().pin_memory()
     x_h, p_h, q_h = pin(w.x), pin(w.x_pre), pin(w.x_post)
     y_h = torch.empty(red.total_k, w.d, dtype=w.x.dtype).pin_memory()
     idx_h = torch.empty(red.total_k, dtype=torch.int32).pin_memory()
-    dev_in = red.alloc_device_inputs()
+    epipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, slots=2, stride=args.stride, **budget)
     for _ in range(3):
-        red.run_host(x_h, p_h, q_h, dev_in, y_h, idx_h)
-    torch.cuda.synchronize()
+        epipe.submit_host(x_h, p_h, q_h, y_h, idx_h)
+    epipe.synchronize()
     e2e_steps = max(3, min(args.steps, args.e2e_steps))
     barrier()
     t0 = time.perf_counter()
     for _ in range(e2e_steps):
-        red.run_host(x_h, p_h, q_h, dev_in, y_h, idx_h)
-        torch.cuda.synchronize()
+        epipe.submit_host(x_h, p_h, q_h, y_h, idx_h)
+    epipe.synchronize()
     e2e_s = max_over_ranks((time.perf_counter() - t0) / e2e_steps, world, dev)
-    del dev_in
+    epipe.close()
+    del epipe
 
     peak, peak_kind = _peaks()
     score_ms = statistics.mean(t_score)

@@ -318,6 +318,7 @@ class Pipeline:
                      for _ in range(self.slots)]
         self.score_stream = torch.cuda.Stream(dev, priority=0)
         self.select_stream = torch.cuda.Stream(dev, priority=-100)  # the device's highest priority
+        self._host = None  # submit_host: per-slot device inputs, copy streams and reuse events
         self._ws = None
         self._handle = None
         self._tok = None
@@ -367,6 +368,44 @@ class Pipeline:
         self.submitted += 1
         return ReduceResult(o["y"][:self.total_k], o["idx"][:self.total_k], self.cu_k, o["h2"], o["s"], o["status"])
 
+    def submit_host(self, x_h, x_pre_h, x_post_h, y_h, idx_h) -> ReduceResult:
+        """End to end from pinned host memory: copies this batch's inputs into
+        the slot's device buffers on a copy-in stream, submits it, and copies
+        y and idx back into the pinned ``y_h`` / ``idx_h`` on a copy-out
+        stream.  The next batch's upload overlaps this batch's work and
+        download.  ``y_h`` and ``idx_h`` are complete after ``synchronize``."""
+        slot = self.submitted % self.slots
+        if self._host is None:
+            t = sum(self.seqlens)
+            mk = lambda: torch.empty(t, self.d, dtype=self.dtype, device=self.device)
+            self._host = dict(
+                bufs=[(mk(), None if self.alias_pre else mk(), mk()) for _ in range(self.slots)],
+                cin=torch.cuda.Stream(self.device), cout=torch.cuda.Stream(self.device),
+                in_free=[None] * self.slots, out_free=[None] * self.slots)
+        h = self._host
+        dx, dp, dq = h["bufs"][slot]
+        if h["in_free"][slot] is not None:  # the slot's last batch has been gathered
+            h["cin"].wait_event(h["in_free"][slot])
+        if h["out_free"][slot] is not None:  # and its results copied out
+            self.select_stream.wait_event(h["out_free"][slot])
+        with torch.cuda.stream(h["cin"]):
+            dx.copy_(x_h, non_blocking=True)
+            if dp is not None:
+                dp.copy_(x_pre_h, non_blocking=True)
+            dq.copy_(x_post_h, non_blocking=True)
+            r = self.submit(dx, dp, dq)  # scoring waits for the copies (the current stream)
+        done = torch.cuda.Event()
+        done.record(self.select_stream)
+        h["in_free"][slot] = done
+        h["cout"].wait_event(done)
+        with torch.cuda.stream(h["cout"]):
+            y_h.copy_(r.y, non_blocking=True)
+            idx_h.copy_(r.idx, non_blocking=True)
+            out = torch.cuda.Event()
+            out.record(h["cout"])
+        h["out_free"][slot] = out
+        return r
+
     def wait(self, stream=None):
         """Makes ``stream`` (default: the current stream) wait for every submission."""
         st = stream if stream is not None else torch.cuda.current_stream(self.device)
@@ -376,6 +415,9 @@ class Pipeline:
     def synchronize(self):
         self.select_stream.synchronize()
         self.score_stream.synchronize()
+        if self._host is not None:
+            self._host["cin"].synchronize()
+            self._host["cout"].synchronize()
 
     def close(self):
         if self._handle is not None:

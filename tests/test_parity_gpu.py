@@ -239,6 +239,36 @@ def test_graph_replay_and_limits():
     check_reduce(x, xp, xq, [25, 15], _alt().budgets([25, 15], k=10))
 
 
+def test_pipeline_from_host():
+    # Pinned host batches in, y and idx back to pinned host buffers, three
+    # different batches through two slots (uploads overlap the work).
+    altr = _alt()
+    ws = [synth.make("llava576", seed=40 + s, batch=3, d=256) for s in range(3)]
+    budget = _budget(ws[0], k=96)
+    pipe = altr.Pipeline(ws[0].seqlens, 256, torch.bfloat16, "cuda", budget=budget, scores=True)
+    try:
+        pin = lambda t: t.pin_memory()
+        outs = []
+        for w in ws:
+            y_h = torch.empty(budget[2][-1], 256, dtype=torch.bfloat16).pin_memory()
+            idx_h = torch.empty(budget[2][-1], dtype=torch.int32).pin_memory()
+            r = pipe.submit_host(pin(w.x), pin(w.x_pre), pin(w.x_post), y_h, idx_h)
+            outs.append((y_h, idx_h, r))
+        pipe.synchronize()
+        w, (y_h, idx_h, r) = ws[-1], outs[-1]
+        compare_result(r, w.x, w.x_pre, w.x_post, w.seqlens, budget)
+        for w, (y_h, idx_h, _) in zip(ws, outs):
+            ks, k1s, cu = budget
+            for b in range(w.batch):
+                xb, pb, qb = (_f64(t[b * 576:(b + 1) * 576]) for t in (w.x, w.x_pre, w.x_post))
+                ref = oracle.select_image(xb, pb, qb, ks[b], k1s[b])
+                assert np.array_equal(idx_h[cu[b]:cu[b + 1]].numpy(), ref["kept"]), b
+                rows = w.x[b * 576:(b + 1) * 576][torch.from_numpy(ref["kept"].astype(np.int64))]
+                assert torch.equal(_bits(y_h[cu[b]:cu[b + 1]]), _bits(rows)), b
+    finally:
+        pipe.close()
+
+
 def test_pipeline_edge_cases():
     # one slot and three slots, an empty image and K = 0 images in a ragged
     # batch, fp32 inputs, and a batch that keeps nothing at all
