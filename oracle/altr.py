@@ -22,7 +22,7 @@ What it computes, step by step in the order of Algorithm 1:
    |X_rem| / K2: positions floor(j |X_rem| / K2), j < K2
 9. X* = X_imp union X_div, returned in ascending token order (Eq. 7)
 
-Readings of points the paper leaves open (each is listed in the design doc):
+Readings of points the paper leaves open:
 
 * ties (top-K and sort) go to the lower token index;
 * an all-zero row has H2 = 0 (p is undefined; 0 is the one-hot value);
