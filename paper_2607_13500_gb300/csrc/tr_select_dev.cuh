@@ -568,14 +568,11 @@ __device__ __forceinline__ void exact_row_any(const SelectArgs &a, long long row
 // The pending rows are listed first (a block-wide vote skips everything when
 // none is); then up to four rows at a time are handled by groups of warps.
 constexpr int kPendCap = 512;
-__device__ void refine_pending(const SelectArgs &a, long long off, int n, uint8_t *fl, ExactRec *rec,
-                               const bool primary) {
+__device__ __noinline__ void refine_listed(const SelectArgs &a, long long off, int n, uint8_t *fl, ExactRec *rec,
+                                           const bool primary) {
   __shared__ Part128 part;
   __shared__ int plist[kPendCap];
   __shared__ int pcount;
-  bool any = false;
-  for (int i = threadIdx.x; i < n; i += blockDim.x) any |= (fl[i] & (F_NEEDL | F_NEEDS)) != 0;
-  if (!__syncthreads_or(any)) return;
   for (;;) {
     if (threadIdx.x == 0) pcount = 0;
     __syncthreads();
@@ -609,6 +606,14 @@ __device__ void refine_pending(const SelectArgs &a, long long off, int n, uint8_
     }
     if (total <= kPendCap) break;  // otherwise list the rows still pending
   }
+}
+// The common case -- nothing pending -- costs one pass over the flags and a
+// block vote; the work itself stays out of line.
+__device__ __forceinline__ void refine_pending(const SelectArgs &a, long long off, int n, uint8_t *fl,
+                                               ExactRec *rec, const bool primary) {
+  bool any = false;
+  for (int i = threadIdx.x; i < n; i += blockDim.x) any |= (fl[i] & (F_NEEDL | F_NEEDS)) != 0;
+  if (__syncthreads_or(any)) refine_listed(a, off, n, fl, rec, primary);
 }
 
 // ---------------------------------------------------------------- exact comparisons
@@ -776,7 +781,7 @@ __device__ int block_exclusive_scan(int v, int *total) {
 // warp scatters its stretch in order, ranking equal digits within 32 lanes
 // with match-any, which keeps the sort stable.  A pass whose digit is the
 // same for every row is skipped.  Returns the buffer holding the order.
-__device__ uint16_t *radix_sort(const uint32_t *key, uint16_t *a, uint16_t *b, int m, uint32_t *hist) {
+__device__ __noinline__ uint16_t *radix_sort(const uint32_t *key, uint16_t *a, uint16_t *b, int m, uint32_t *hist) {
   __shared__ int skip;
   __shared__ uint32_t dsum[8];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -969,7 +974,7 @@ __device__ __forceinline__ uint32_t mix32(uint32_t x) {  // an integer hash (xor
   x ^= x >> 16;
   return x;
 }
-__device__ uint16_t *sample_sort(const uint32_t *key, uint16_t *a, uint16_t *b, uint16_t *bid, int m,
+__device__ __noinline__ uint16_t *sample_sort(const uint32_t *key, uint16_t *a, uint16_t *b, uint16_t *bid, int m,
                                  uint32_t *hist) {
   static_assert(kSelectThreads == 512, "511 splitters, 512 buckets");
   const int tid = threadIdx.x, nthr = blockDim.x, lane = tid & 31, warp = tid >> 5;
