@@ -63,6 +63,7 @@ def _args():
     ap.add_argument("--seed", type=int, default=0)
     ap.add_argument("--per-frame", action="store_true",
                     help="video6272: select per 196-token frame instead of per 32-frame clip")
+    ap.add_argument("--lam", default="1/3", help="balance lambda = K1 / K as a rational num/den (Algorithm 1)")
     ap.add_argument("--stride", choices=["alg1", "interval"], default="alg1",
                     help="diversity pick positions: Algorithm 1's integer stride or Section IV-B's real interval")
     ap.add_argument("--e2e-steps", type=int, default=20)
@@ -71,6 +72,11 @@ def _args():
     if a.warmup < 3:
         ap.error("--warmup must be at least 3")
     return a
+
+
+def _lam(args):
+    num, den = (int(v) for v in args.lam.split("/"))
+    return num, den
 
 
 def _dist():
@@ -116,10 +122,10 @@ def _workload_config(w, budget, args):
     extra = "".join([", per-frame budgets" if getattr(args, "per_frame", False) else "",
                      ", interval stride" if getattr(args, "stride", "alg1") == "interval" else ""])
     return {
-        "workload": f"{w.name}: B={w.batch}, N={n}, D={w.d}, {dt}, {ks_desc}, lambda=1/3{extra}",
+        "workload": f"{w.name}: B={w.batch}, N={n}, D={w.d}, {dt}, {ks_desc}, lambda={args.lam}{extra}",
         "batch": w.batch, "n": n, "d": w.d, "input_dtype": dt, **({"k": budget["k"]} if "k" in budget else
                                                                  {"ratio": list(budget["ratio"])}),
-        "lambda": "1/3", "stride": getattr(args, "stride", "alg1"),
+        "lambda": args.lam, "stride": getattr(args, "stride", "alg1"),
         "budget_unit": "frame" if getattr(args, "per_frame", False) else "image",
     }
 
@@ -183,14 +189,14 @@ def _oracle_images(w, count):
     return out
 
 
-def cpu_baseline(w, ks, k1s, seconds):
+def cpu_baseline(w, ks, k1s, seconds, stride="alg1"):
     """The CPU oracle, as it stands, on a bounded sample of the same workload."""
     import oracle
     imgs = _oracle_images(w, 8)
     done, t0 = 0, time.perf_counter()
     while True:
         b = done % len(imgs)
-        oracle.select_image(*imgs[b], ks[b], k1s[b])
+        oracle.select_image(*imgs[b], ks[b], k1s[b], stride)
         done += 1
         el = time.perf_counter() - t0
         if el >= seconds and done >= 1:
@@ -210,13 +216,13 @@ def run_reference(args, world, rank):
     w = synth.make(args.workload, seed=args.seed, device="cpu", **over)
     import oracle as orc
     ks = [budget["k"] if "k" in budget else orc.budget_from_ratio(n, budget["ratio"]) for n in w.seqlens]
-    k1s = [orc.budget_split(k, (1, 3))[0] for k in ks]
+    k1s = [orc.budget_split(k, _lam(args))[0] for k in ks]
     imgs = _oracle_images(w, 8)
     for i in range(args.warmup):
         b = i % len(imgs)
-        orc.select_image(*imgs[b], ks[b], k1s[b])
+        orc.select_image(*imgs[b], ks[b], k1s[b], args.stride)
     t_one = time.perf_counter()
-    orc.select_image(*imgs[0], ks[0], k1s[0])
+    orc.select_image(*imgs[0], ks[0], k1s[0], args.stride)
     t_one = time.perf_counter() - t_one
     steps = args.steps
     note = ""
@@ -226,7 +232,7 @@ def run_reference(args, world, rank):
     t0 = time.perf_counter()
     for i in range(steps):
         b = i % len(imgs)
-        orc.select_image(*imgs[b], ks[b], k1s[b])
+        orc.select_image(*imgs[b], ks[b], k1s[b], args.stride)
     el = time.perf_counter() - t0
     value = steps / el
     sample = (f"one image per step ({w.seqlens[0]} tokens x D={w.d}), cycling over the first {len(imgs)} images "
@@ -281,8 +287,8 @@ def run_ours(args, world, rank, local):
     w = synth.make(args.workload, seed=rank_seed(args.seed, rank), device=dev, **over)
     if args.per_frame:
         w = w.frames()
-    red = altr.Reducer(w.seqlens, w.d, w.x.dtype, dev, stride=args.stride, **budget)
-    pipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, slots=2, stride=args.stride, **budget)
+    red = altr.Reducer(w.seqlens, w.d, w.x.dtype, dev, stride=args.stride, lam=_lam(args), **budget)
+    pipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, slots=2, stride=args.stride, lam=_lam(args), **budget)
     e = 2 if w.x.dtype == torch.bfloat16 else 4
     total_rows = w.total
     in_bytes = 3 * total_rows * w.d * e
@@ -344,7 +350,7 @@ def run_ours(args, world, rank, local):
     x_h, p_h, q_h = pin(w.x), pin(w.x_pre), pin(w.x_post)
     y_h = torch.empty(red.total_k, w.d, dtype=w.x.dtype).pin_memory()
     idx_h = torch.empty(red.total_k, dtype=torch.int32).pin_memory()
-    epipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, slots=2, stride=args.stride, **budget)
+    epipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, slots=2, stride=args.stride, lam=_lam(args), **budget)
     for _ in range(3):
         epipe.submit_host(x_h, p_h, q_h, y_h, idx_h)
     epipe.synchronize()
@@ -389,7 +395,7 @@ def run_ours(args, world, rank, local):
         "status": st,
     }
     if rank == 0 and world == 1:
-        line["cpu_baseline"] = cpu_baseline(w, red.ks, red.k1s, args.cpu_seconds)
+        line["cpu_baseline"] = cpu_baseline(w, red.ks, red.k1s, args.cpu_seconds, args.stride)
     if rank == 0:
         print(json.dumps(line), flush=True)
     if world > 1:
