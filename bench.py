@@ -214,6 +214,8 @@ def run_reference(args, world, rank):
     budget = BUDGETS[args.workload]
     over = {"batch": args.batch} if args.batch else {}
     w = synth.make(args.workload, seed=args.seed, device="cpu", **over)
+    if args.per_frame:
+        w = w.frames()
     import oracle as orc
     ks = [budget["k"] if "k" in budget else orc.budget_from_ratio(n, budget["ratio"]) for n in w.seqlens]
     k1s = [orc.budget_split(k, _lam(args))[0] for k in ks]
