@@ -56,7 +56,7 @@ typedef enum {
   TR_ERR_UNSUPPORTED = 7  /* N_b > TR_MAX_N or d > TR_MAX_D                    */
 } tr_status;
 
-typedef enum { TR_F32 = 0, TR_BF16 = 1 } tr_dtype;
+typedef enum { TR_F32 = 0, TR_BF16 = 1, TR_F16 = 2 } tr_dtype;
 
 #define TR_MAX_N 16384        /* tokens per image (keys of one image stay in shared memory) */
 #define TR_MAX_D 16384        /* channels per token                                  */

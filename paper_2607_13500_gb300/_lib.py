@@ -9,7 +9,7 @@ _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libtr.so")
 HEADER = os.path.join(os.path.dirname(_HERE), "include", "tr.h")
 
-TR_F32, TR_BF16 = 0, 1
+TR_F32, TR_BF16, TR_F16 = 0, 1, 2
 TR_STRIDE_INTERVAL = 1
 STRIDE_MODES = {"alg1": 0, "interval": TR_STRIDE_INTERVAL}
 TR_STATS_WORDS = 8

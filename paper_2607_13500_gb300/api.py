@@ -12,7 +12,7 @@ from dataclasses import dataclass
 import torch
 
 from . import _lib
-from ._lib import STRIDE_MODES, TR_BF16, TR_F32, TR_STATS_WORDS, TR_STATUS_WORDS, TrTokens, check, load
+from ._lib import STRIDE_MODES, TR_BF16, TR_F16, TR_F32, TR_STATS_WORDS, TR_STATUS_WORDS, TrTokens, check, load
 
 _I32 = ctypes.c_int32
 
@@ -20,9 +20,11 @@ _I32 = ctypes.c_int32
 def _dtype_code(t: torch.Tensor) -> int:
     if t.dtype == torch.bfloat16:
         return TR_BF16
+    if t.dtype == torch.float16:
+        return TR_F16
     if t.dtype == torch.float32:
         return TR_F32
-    raise TypeError(f"unsupported dtype {t.dtype}: expected torch.bfloat16 or torch.float32")
+    raise TypeError(f"unsupported dtype {t.dtype}: expected torch.bfloat16, torch.float16 or torch.float32")
 
 
 def _ptr(t):

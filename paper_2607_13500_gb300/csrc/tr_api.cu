@@ -19,7 +19,7 @@ struct Shape {
 
 tr_status check_tokens(const tr_tokens *in, Shape *sh) {
   if (!in || !in->x || !in->x_post) return TR_ERR_ARG;
-  if (in->dtype != TR_F32 && in->dtype != TR_BF16) return TR_ERR_DTYPE;
+  if (in->dtype != TR_F32 && in->dtype != TR_BF16 && in->dtype != TR_F16) return TR_ERR_DTYPE;
   if (in->flags & ~TR_STRIDE_INTERVAL) return TR_ERR_ARG;
   if (in->d <= 0 || in->batch < 0) return TR_ERR_ARG;
   if (in->d > TR_MAX_D) return TR_ERR_UNSUPPORTED;

@@ -52,7 +52,7 @@ static_assert(sizeof(ExactRec) % 16 == 0, "ExactRec records keep 16-byte alignme
 // whose low parts' own rounding is bounded separately (at most lane_chunks
 // + 12 low-part additions on any path, folds and warp merges included), and
 // the keys are computed from the unrounded double-float.
-__host__ __device__ inline int elem_bytes(int dtype) { return dtype == TR_BF16 ? 2 : 4; }
+__host__ __device__ inline int elem_bytes(int dtype) { return dtype == TR_F32 ? 4 : 2; }
 
 __host__ __device__ inline int score_depth(int d, int dtype) {
   (void)d;
@@ -85,9 +85,10 @@ inline Bounds certification_bounds(int d, int dtype) {
   const double g = h * u / (1.0 - h * u) + m * m * u * u + 0x1p-34;  // relative error of L1, S2, A, B
   // P = P_hi + P_lo is exact up to the rounding of the P_lo additions:
   // at most u^2 (lane_terms^2 / 2 + 12 d) sum|x'x''| (doubled for fp32
-  // inputs, whose product errors also enter P_lo), and sum|x'x''| <= sqrt(A B).
+  // inputs, whose product errors also enter P_lo; bf16 and fp16 products,
+  // 16 and 22 significant bits, are exact), and sum|x'x''| <= sqrt(A B).
   double ep = 2.0 * u * u * (lane_terms * lane_terms + 12.0 * d) + 0x1p-52;
-  if (dtype != TR_BF16) ep *= 2.0;
+  if (dtype == TR_F32) ep *= 2.0;  // bf16 and fp16 products are exact in fp32
   Bounds b;
   // R32 = fl(R^) with R^ = L1^2 / S2 evaluated in double-float (2^-40) from
   // sums within relative g: R32 / R within (1 + g)^2 / (1 - g) (1 + 2^-40) (1 + u);

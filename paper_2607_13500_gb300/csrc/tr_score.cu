@@ -7,14 +7,14 @@
 namespace tr {
 namespace {
 
-template <bool kBf16>
+template <int kDt>
 __global__ void __launch_bounds__(kScoreWarps * 32)
     k_score(const uint4 *__restrict__ x, const uint4 *__restrict__ xp, const uint4 *__restrict__ xq, int nchunks,
             long long total, float4 *__restrict__ stats, float *__restrict__ h2, float *__restrict__ s_out) {
   const int lane = threadIdx.x & 31;
   const long long stride = (long long)gridDim.x * kScoreWarps;
   for (long long row = (long long)blockIdx.x * kScoreWarps + (threadIdx.x >> 5); row < total; row += stride)
-    score_row<kBf16>(x, xp, xq, nchunks, row, stats, h2, s_out, lane);
+    score_row<kDt>(x, xp, xq, nchunks, row, stats, h2, s_out, lane);
 }
 
 }  // namespace
@@ -22,7 +22,6 @@ __global__ void __launch_bounds__(kScoreWarps * 32)
 cudaError_t launch_score(const void *x, const void *x_pre, const void *x_post, int dtype, int d, long long total,
                          float *stats, float *h2, float *s, cudaStream_t st) {
   if (total == 0) return cudaSuccess;
-  const int which = dtype == TR_BF16 ? 1 : 0;
   const int row_bytes = d * elem_bytes(dtype);
   const unsigned char *bx = static_cast<const unsigned char *>(x);
   const unsigned char *bp = static_cast<const unsigned char *>(x_pre ? x_pre : x);
@@ -40,10 +39,12 @@ cudaError_t launch_score(const void *x, const void *x_pre, const void *x_post, i
   const uint4 *px = reinterpret_cast<const uint4 *>(bx);
   const uint4 *pp = reinterpret_cast<const uint4 *>(bp);
   const uint4 *pq = reinterpret_cast<const uint4 *>(bq);
-  if (which)
-    k_score<true><<<grid, kScoreWarps * 32, 0, st>>>(px, pp, pq, nchunks, total, ps, h2, s);
+  if (dtype == TR_BF16)
+    k_score<TR_BF16><<<grid, kScoreWarps * 32, 0, st>>>(px, pp, pq, nchunks, total, ps, h2, s);
+  else if (dtype == TR_F16)
+    k_score<TR_F16><<<grid, kScoreWarps * 32, 0, st>>>(px, pp, pq, nchunks, total, ps, h2, s);
   else
-    k_score<false><<<grid, kScoreWarps * 32, 0, st>>>(px, pp, pq, nchunks, total, ps, h2, s);
+    k_score<TR_F32><<<grid, kScoreWarps * 32, 0, st>>>(px, pp, pq, nchunks, total, ps, h2, s);
   return cudaGetLastError();
 }
 

@@ -3,12 +3,12 @@
 //
 // One warp per row; lane l reads 16-byte chunks l, l+32, l+64, ... of each of
 // the three streams (fully coalesced 512-byte warp requests), a batch of
-// chunks per stream in flight before any arithmetic.  Each chunk's partial
+// chunks per stream in flight before any arithmetic; bf16, fp16 or fp32.  Each chunk's partial
 // sums of |x|, x^2, x'^2, x''^2 come from a depth-3 fp32 tree; the partials
 // are accumulated error-free as double-floats (TwoSum), so every sum carries
 // at most score_depth() roundings whatever D is.  P = x'.x'' is accumulated
 // error-free term by term, since the ordering by s needs it to far better
-// than fp32.  bf16 chunks are processed two at a time with the packed f32x2
+// than fp32.  16-bit chunks are processed two at a time with the packed f32x2
 // instructions (half the issue slots; each half rounds exactly like the
 // scalar operation), so each lane carries two double-float accumulators per
 // sum, one for its even-numbered chunks and one for its odd ones.  The
@@ -41,8 +41,6 @@ __device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
   e = __fadd_rn(__fsub_rn(a, aa), __fsub_rn(b, bb));
 }
 
-__device__ __forceinline__ float lo_bf16(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float hi_bf16(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
 
 // Double-float accumulator: hi + lo carries the sum, hi exact in TwoSum.
 struct DF {
@@ -122,13 +120,32 @@ struct Acc2 {
   DF2 l1, s2, a, b, p;
 };
 
-// Two 16-byte chunks (u, v) of bf16 elements of each stream at once: half 0
-// of every packed value belongs to chunk u, half 1 to chunk v.  Per chunk:
-// depth-3 trees of |x|, x^2, x'^2, x''^2 (bf16 squares and products are exact
-// in fp32, so only the additions round; x^2 is taken as |x|^2, the same
-// value) and the eight exact products x'x'' through TwoSum one by one.
-// Chunk u's terms enter accumulator half 0, chunk v's half 1.
-__device__ __forceinline__ void chunk2_bf16(const uint4 &xu, const uint4 &xv, const uint4 &pu, const uint4 &pv,
+// fp32 bit patterns of the two 16-bit elements of word w (low half first):
+// bf16 by shifting, fp16 by exact conversion (subnormals included).
+template <int kDt>
+__device__ __forceinline__ void halves(uint32_t w, uint32_t &lo, uint32_t &hi) {
+  if (kDt == TR_BF16) {
+    lo = w << 16;
+    hi = w & 0xffff0000u;
+  } else {
+    float flo, fhi;
+    asm("{\n .reg .f16 l, h;\n mov.b32 {l, h}, %2;\n cvt.f32.f16 %0, l;\n cvt.f32.f16 %1, h;\n}"
+        : "=f"(flo), "=f"(fhi)
+        : "r"(w));
+    lo = __float_as_uint(flo);
+    hi = __float_as_uint(fhi);
+  }
+}
+
+// Two 16-byte chunks (u, v) of 16-bit elements (bf16 or fp16) of each stream
+// at once: half 0 of every packed value belongs to chunk u, half 1 to chunk
+// v.  Per chunk: depth-3 trees of |x|, x^2, x'^2, x''^2 (squares and products
+// of bf16 or fp16 values are exact in fp32, so only the additions round; x^2
+// is taken as |x|^2, the same value) and the eight exact products x'x''
+// through TwoSum one by one.  Chunk u's terms enter accumulator half 0,
+// chunk v's half 1.
+template <int kDt>
+__device__ __forceinline__ void chunk2_half(const uint4 &xu, const uint4 &xv, const uint4 &pu, const uint4 &pv,
                                             const uint4 &qu, const uint4 &qv, Acc2 &acc) {
   const uint32_t wxu[4] = {xu.x, xu.y, xu.z, xu.w}, wxv[4] = {xv.x, xv.y, xv.z, xv.w};
   const uint32_t wpu[4] = {pu.x, pu.y, pu.z, pu.w}, wpv[4] = {pv.x, pv.y, pv.z, pv.w};
@@ -136,10 +153,16 @@ __device__ __forceinline__ void chunk2_bf16(const uint4 &xu, const uint4 &xv, co
   uint64_t l[4], s[4], a[4], b[4];
 #pragma unroll
   for (int i = 0; i < 4; ++i) {
-    const uint32_t au = wxu[i] & 0x7fff7fffu, av = wxv[i] & 0x7fff7fffu;
-    const uint64_t x0 = pk(au << 16, av << 16), x1 = pk(au & 0xffff0000u, av & 0xffff0000u);
-    const uint64_t p0 = pk(wpu[i] << 16, wpv[i] << 16), p1 = pk(wpu[i] & 0xffff0000u, wpv[i] & 0xffff0000u);
-    const uint64_t q0 = pk(wqu[i] << 16, wqv[i] << 16), q1 = pk(wqu[i] & 0xffff0000u, wqv[i] & 0xffff0000u);
+    uint32_t x0u, x1u, x0v, x1v, p0u, p1u, p0v, p1v, q0u, q1u, q0v, q1v;
+    halves<kDt>(wxu[i] & 0x7fff7fffu, x0u, x1u);  // |x|: both formats keep the sign in bit 15
+    halves<kDt>(wxv[i] & 0x7fff7fffu, x0v, x1v);
+    halves<kDt>(wpu[i], p0u, p1u);
+    halves<kDt>(wpv[i], p0v, p1v);
+    halves<kDt>(wqu[i], q0u, q1u);
+    halves<kDt>(wqv[i], q0v, q1v);
+    const uint64_t x0 = pk(x0u, x0v), x1 = pk(x1u, x1v);
+    const uint64_t p0 = pk(p0u, p0v), p1 = pk(p1u, p1v);
+    const uint64_t q0 = pk(q0u, q0v), q1 = pk(q1u, q1v);
     l[i] = add2(x0, x1);
     s[i] = fma2(x0, x0, mul2(x1, x1));
     a[i] = fma2(p0, p0, mul2(p1, p1));
@@ -218,7 +241,7 @@ __device__ __forceinline__ void finish_row(Acc &acc, long long row, float4 *__re
 // One round: lane l takes chunks base + l + 32u (u < kB) of each stream,
 // all loads issued before any arithmetic; with kGuard, chunks at or past c1
 // are zeros (which add nothing).
-template <bool kBf16, int kB, bool kGuard>
+template <int kDt, int kB, bool kGuard>
 __device__ __forceinline__ void accumulate_round(const uint4 *__restrict__ rx, const uint4 *__restrict__ rp,
                                                  const uint4 *__restrict__ rq, int base, int c1, Acc &acc,
                                                  Acc2 &acc2, int lane) {
@@ -234,9 +257,9 @@ __device__ __forceinline__ void accumulate_round(const uint4 *__restrict__ rx, c
       vx[u] = vp[u] = vq[u] = make_uint4(0u, 0u, 0u, 0u);
     }
   }
-  if (kBf16) {
+  if (kDt != TR_F32) {
 #pragma unroll
-    for (int u = 0; u < kB; u += 2) chunk2_bf16(vx[u], vx[u + 1], vp[u], vp[u + 1], vq[u], vq[u + 1], acc2);
+    for (int u = 0; u < kB; u += 2) chunk2_half<kDt>(vx[u], vx[u + 1], vp[u], vp[u + 1], vq[u], vq[u + 1], acc2);
   } else {
 #pragma unroll
     for (int u = 0; u < kB; ++u) chunk_f32(vx[u], vp[u], vq[u], acc);
@@ -247,27 +270,27 @@ __device__ __forceinline__ void accumulate_round(const uint4 *__restrict__ rx, c
 // memory in rounds of kB chunks per lane and stream.  When the row's chunks
 // are a multiple of 32 (every lane has the same count) the last round is cut
 // to the chunks that remain (6, 4 or 2 per lane), so no lane works on padding.
-template <bool kBf16>
+template <int kDt>
 __device__ __forceinline__ void accumulate_global(const uint4 *__restrict__ rx, const uint4 *__restrict__ rp,
                                                   const uint4 *__restrict__ rq, int c0, int c1, Acc &acc,
                                                   int lane) {
-  constexpr int kB = kBf16 ? kScoreBatchBf16 : kScoreBatchF32;
+  constexpr int kB = kDt != TR_F32 ? kScoreBatchBf16 : kScoreBatchF32;
   static_assert(kB % 2 == 0, "bf16 chunks are summed in pairs");
   Acc2 acc2{};
   int base = c0;
-  for (; base + 32 * kB <= c1; base += 32 * kB) accumulate_round<kBf16, kB, false>(rx, rp, rq, base, c1, acc, acc2, lane);
+  for (; base + 32 * kB <= c1; base += 32 * kB) accumulate_round<kDt, kB, false>(rx, rp, rq, base, c1, acc, acc2, lane);
   const int rest = c1 - base;
   if (rest > 0) {
     if (kB == 8 && rest == 32 * 6)
-      accumulate_round<kBf16, 6, false>(rx, rp, rq, base, c1, acc, acc2, lane);
+      accumulate_round<kDt, 6, false>(rx, rp, rq, base, c1, acc, acc2, lane);
     else if (kB == 8 && rest == 32 * 4)
-      accumulate_round<kBf16, 4, false>(rx, rp, rq, base, c1, acc, acc2, lane);
+      accumulate_round<kDt, 4, false>(rx, rp, rq, base, c1, acc, acc2, lane);
     else if (rest == 32 * 2)
-      accumulate_round<kBf16, 2, false>(rx, rp, rq, base, c1, acc, acc2, lane);
+      accumulate_round<kDt, 2, false>(rx, rp, rq, base, c1, acc, acc2, lane);
     else
-      accumulate_round<kBf16, kB, true>(rx, rp, rq, base, c1, acc, acc2, lane);
+      accumulate_round<kDt, kB, true>(rx, rp, rq, base, c1, acc, acc2, lane);
   }
-  if (kBf16) {
+  if (kDt != TR_F32) {
     // Half 0 holds this lane's even-numbered chunks, half 1 its odd ones.
     const DF l1 = df2_fold(acc2.l1), s2 = df2_fold(acc2.s2), a = df2_fold(acc2.a), b = df2_fold(acc2.b),
              p = df2_fold(acc2.p);
@@ -280,13 +303,13 @@ __device__ __forceinline__ void accumulate_global(const uint4 *__restrict__ rx, 
 }
 
 // Scores one row (one warp) straight from global memory.
-template <bool kBf16>
+template <int kDt>
 __device__ __forceinline__ void score_row(const uint4 *__restrict__ x, const uint4 *__restrict__ xp,
                                           const uint4 *__restrict__ xq, int nchunks, long long row,
                                           float4 *__restrict__ stats, float *__restrict__ h2,
                                           float *__restrict__ s_out, int lane) {
   Acc acc{{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
-  accumulate_global<kBf16>(x + row * nchunks, xp + row * nchunks, xq + row * nchunks, 0, nchunks, acc, lane);
+  accumulate_global<kDt>(x + row * nchunks, xp + row * nchunks, xq + row * nchunks, 0, nchunks, acc, lane);
   finish_row(acc, row, stats, h2, s_out, lane);
 }
 

@@ -179,14 +179,22 @@ struct Term {
   int e;       // value = m * 2^e
   bool nonfinite;
 };
-__device__ __forceinline__ Term decode(const void *base, long long i, bool bf16) {
+// value = m 2^e of element i of a tensor of dtype dt (significand with the
+// hidden bit; subnormals use the smallest exponent).
+__device__ __forceinline__ Term decode(const void *base, long long i, int dt) {
   Term t;
-  if (bf16) {
+  if (dt == TR_BF16) {
     const uint32_t b = static_cast<const uint16_t *>(base)[i];
     const uint32_t ex = (b >> 7) & 0xffu, mant = b & 0x7fu;
     t.nonfinite = ex == 0xffu;
     t.m = ex ? (mant | 0x80u) : mant;
     t.e = (ex ? (int)ex : 1) - 134;
+  } else if (dt == TR_F16) {
+    const uint32_t b = static_cast<const uint16_t *>(base)[i];
+    const uint32_t ex = (b >> 10) & 0x1fu, mant = b & 0x3ffu;
+    t.nonfinite = ex == 0x1fu;
+    t.m = ex ? (mant | 0x400u) : mant;
+    t.e = (ex ? (int)ex : 1) - 25;
   } else {
     const uint32_t b = static_cast<const uint32_t *>(base)[i];
     const uint32_t ex = (b >> 23) & 0xffu, mant = b & 0x7fffffu;
@@ -196,8 +204,9 @@ __device__ __forceinline__ Term decode(const void *base, long long i, bool bf16)
   }
   return t;
 }
-__device__ __forceinline__ bool sign_bit(const void *base, long long i, bool bf16) {
-  return bf16 ? (static_cast<const uint16_t *>(base)[i] >> 15) != 0 : (static_cast<const uint32_t *>(base)[i] >> 31) != 0;
+__device__ __forceinline__ bool sign_bit(const void *base, long long i, int dt) {
+  return dt != TR_F32 ? (static_cast<const uint16_t *>(base)[i] >> 15) != 0
+                      : (static_cast<const uint32_t *>(base)[i] >> 31) != 0;
 }
 
 // Adds (+/-) m * 2^e into signed 32-bit digit positions relative to 2^base.
@@ -273,19 +282,20 @@ __device__ __forceinline__ void warp_sum_digits(long long *dg) {
 
 // Exact sums of one row, computed by one warp.  mode 0: L1 = sum|x| and
 // S2 = sum x^2; mode 1: A = sum x'^2, B = sum x''^2, P = sum x'x''.
-// Digit bases (multiples of 32): |x| has exponent >= -133 (bf16) or -149
-// (fp32), products >= -266 or -298; the top digit stays below kDig.
+// Digit bases (multiples of 32): |x| has exponent >= -133 (bf16), -24 (fp16)
+// or -149 (fp32), products >= -266, -48 or -298; the top digit stays below
+// kDig.
 __device__ __noinline__ void exact_row(const SelectArgs &a, long long row, int mode, ExactRec *rec, int lane) {
-  const bool bf16 = a.dtype == TR_BF16;
+  const int dt = a.dtype;
   const int base1 = -160;
-  const int base2 = bf16 ? -288 : -320;
+  const int base2 = dt != TR_F32 ? -288 : -320;
   long long d0[kDig], d1[kDig], d2[kDig];
   for (int k = 0; k < kDig; ++k) d0[k] = d1[k] = d2[k] = 0;
   bool nonfinite = false;
   const long long first = row * (long long)a.d;
   if (mode == 0) {
     for (int j = lane; j < a.d; j += 32) {
-      const Term t = decode(a.x, first + j, bf16);
+      const Term t = decode(a.x, first + j, dt);
       if (t.nonfinite) {
         nonfinite = true;
       } else if (t.m) {
@@ -296,8 +306,8 @@ __device__ __noinline__ void exact_row(const SelectArgs &a, long long row, int m
   } else {
     const void *xp = a.x_pre ? a.x_pre : a.x;
     for (int j = lane; j < a.d; j += 32) {
-      const Term p = decode(xp, first + j, bf16);
-      const Term q = decode(a.x_post, first + j, bf16);
+      const Term p = decode(xp, first + j, dt);
+      const Term q = decode(a.x_post, first + j, dt);
       if (p.nonfinite || q.nonfinite) {
         nonfinite = true;
         continue;
@@ -305,7 +315,7 @@ __device__ __noinline__ void exact_row(const SelectArgs &a, long long row, int m
       if (p.m) add_term(d0, base2, (unsigned long long)p.m * p.m, 2 * p.e, false);
       if (q.m) add_term(d1, base2, (unsigned long long)q.m * q.m, 2 * q.e, false);
       if (p.m && q.m) {
-        const bool neg = sign_bit(xp, first + j, bf16) != sign_bit(a.x_post, first + j, bf16);
+        const bool neg = sign_bit(xp, first + j, dt) != sign_bit(a.x_post, first + j, dt);
         add_term(d2, base2, (unsigned long long)p.m * q.m, p.e + q.e, neg);
       }
     }
@@ -353,14 +363,25 @@ __device__ __forceinline__ Dec dec32(uint32_t b) {
   return Dec{ex ? (mant | 0x800000u) : mant, (ex ? (int)ex : 1) - 150, (b >> 31) != 0, ex == 0xffu};
 }
 
-template <bool kBf16>
+__device__ __forceinline__ Dec dec16h(uint32_t h) {  // IEEE binary16
+  const uint32_t ex = (h >> 10) & 0x1fu, mant = h & 0x3ffu;
+  return Dec{ex ? (mant | 0x400u) : mant, (ex ? (int)ex : 1) - 25, (h >> 15) != 0, ex == 0x1fu};
+}
+
+template <int kDt>
 __device__ __forceinline__ void unpack(const uint4 &v, Dec *out) {
   const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-  if (kBf16) {
+  if (kDt == TR_BF16) {
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       out[2 * i] = dec16(w[i] & 0xffffu);
       out[2 * i + 1] = dec16(w[i] >> 16);
+    }
+  } else if (kDt == TR_F16) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      out[2 * i] = dec16h(w[i] & 0xffffu);
+      out[2 * i + 1] = dec16h(w[i] >> 16);
     }
   } else {
 #pragma unroll
@@ -456,10 +477,10 @@ struct Group {
 // Exact sums of one row computed by a group of warps (each thread takes
 // 16-byte chunks t, t + size, ...), in three 128-bit windows; false
 // (uniformly across the group) when a term does not fit its window.
-template <bool kBf16>
+template <int kDt>
 __device__ bool exact_row_block(const SelectArgs &a, long long row, int mode, const float *st, ExactRec *rec,
                                 Part128 &part, const Group &g) {
-  constexpr int kPer = kBf16 ? 8 : 4;  // elements per 16-byte chunk
+  constexpr int kPer = kDt == TR_F32 ? 4 : 8;  // elements per 16-byte chunk
   const int nchunks = a.d / kPer;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   bool fits = true;
@@ -472,7 +493,7 @@ __device__ bool exact_row_block(const SelectArgs &a, long long row, int mode, co
     const uint4 *px = static_cast<const uint4 *>(a.x) + row * nchunks;
 #pragma unroll 4
     for (int c = g.tid(); c < nchunks; c += g.size) {
-      unpack<kBf16>(__ldg(px + c), e0);
+      unpack<kDt>(__ldg(px + c), e0);
 #pragma unroll
       for (int i = 0; i < kPer; ++i) {
         const Dec &t = e0[i];
@@ -494,8 +515,8 @@ __device__ bool exact_row_block(const SelectArgs &a, long long row, int mode, co
     const uint4 *pq = static_cast<const uint4 *>(a.x_post) + row * nchunks;
 #pragma unroll 4
     for (int c = g.tid(); c < nchunks; c += g.size) {
-      unpack<kBf16>(__ldg(pp + c), e0);
-      unpack<kBf16>(__ldg(pq + c), e1);
+      unpack<kDt>(__ldg(pp + c), e0);
+      unpack<kDt>(__ldg(pq + c), e1);
 #pragma unroll
       for (int i = 0; i < kPer; ++i) {
         const Dec &p = e0[i], &q = e1[i];
@@ -556,8 +577,9 @@ __device__ __forceinline__ void exact_row_any(const SelectArgs &a, long long row
   const bool trusted = mode == 0 ? !isnan(key_r(st)) : !isnan(key_s(st));
   bool ok = false;
   if (trusted)
-    ok = a.dtype == TR_BF16 ? exact_row_block<true>(a, row, mode, st, rec, part, g)
-                            : exact_row_block<false>(a, row, mode, st, rec, part, g);
+    ok = a.dtype == TR_BF16  ? exact_row_block<TR_BF16>(a, row, mode, st, rec, part, g)
+         : a.dtype == TR_F16 ? exact_row_block<TR_F16>(a, row, mode, st, rec, part, g)
+                             : exact_row_block<TR_F32>(a, row, mode, st, rec, part, g);
   if (!ok) {
     if (g.tid() < 32) exact_row(a, row, mode, rec, threadIdx.x & 31);
     g.sync();

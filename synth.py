@@ -102,7 +102,7 @@ class Workload:
 
 
 def _torch_dtype(name: str):
-    return {"f32": torch.float32, "bf16": torch.bfloat16}[name]
+    return {"f32": torch.float32, "bf16": torch.bfloat16, "f16": torch.float16}[name]
 
 
 def _clustered(gen, n, d, clusters, device):

@@ -1,8 +1,8 @@
 """CUDA path versus the CPU oracle, element by element, through the C ABI.
 
 Kept indices and gathered rows must match bit for bit; H2 within 1e-5
-relative (fp32 inputs) or 2e-3 relative (bf16 inputs) and s within 1e-5
-absolute.  Small cases check every image; the full-size workloads (the
+relative (fp32 inputs), 2e-3 relative (bf16 inputs) or 1e-3 relative (fp16
+inputs) and s within 1e-5 absolute.  Small cases check every image; the full-size workloads (the
 launch configuration bench.py times) check sampled images one by one.
 """
 import numpy as np
@@ -14,7 +14,7 @@ import synth
 
 pytestmark = pytest.mark.gpu
 
-H2_RTOL = {torch.float32: 1e-5, torch.bfloat16: 2e-3}
+H2_RTOL = {torch.float32: 1e-5, torch.bfloat16: 2e-3, torch.float16: 1e-3}
 S_ATOL = 1e-5
 
 
@@ -36,7 +36,7 @@ def _f64(t):
 
 
 def _bits(t):
-    return t.view(torch.int16) if t.dtype == torch.bfloat16 else t.view(torch.int32)
+    return t.view(torch.int32) if t.dtype == torch.float32 else t.view(torch.int16)
 
 
 def check_reduce(x, x_pre, x_post, seqlens, budget, images=None, alias=False, expect_nonfinite=False,
@@ -293,6 +293,28 @@ def test_pipeline_edge_cases():
         assert r.idx.numel() == 0 and r.status.cpu().tolist() == [0, 0, 0, 0]
     finally:
         pipe.close()
+
+
+def test_fp16_inputs():
+    # IEEE half inputs: two shrunk workloads (uniform and ragged, both stride
+    # modes), then rows with subnormal halves, the largest finite half
+    # (65504), infinities and NaNs, which the exact path decodes itself.
+    for name, over, bud in [("llava576", dict(batch=4, d=1024), dict(k=128)),
+                            ("ragged_dynres", dict(batch=4, n=(256, 2500), d=512), dict(ratio=(2, 9)))]:
+        w = synth.make(name, seed=9, dtype="f16", **over)
+        for stride in ("alg1", "interval"):
+            check_reduce(w.x, w.x_pre, w.x_post, w.seqlens, _budget(w, **bud), stride=stride)
+    n, d = 64, 256
+    x, xp, xq = _rows(n, d, 14, dtype=torch.float16)
+    x[3] = x[3] * 2.0 ** -20                      # mostly subnormal halves
+    xp[4] = xp[4] * 2.0 ** -22
+    x[5, :8] = 65504.0
+    xq[6, 2] = 65504.0
+    x[7, 1] = float("inf")
+    xq[8, 0] = float("nan")
+    x[9] = x[10]                                  # an exact tie
+    for k, k1 in [(64, 60), (40, 13), (20, 0)]:
+        check_reduce(x, xp, xq, [n], ([k], [k1], [0, k]), expect_nonfinite=True)
 
 
 # ---------------------------------------------------------------- edge cases
