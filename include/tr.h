@@ -225,16 +225,18 @@ tr_status tr_reduce_noalloc(const tr_tokens *in, const int32_t *d_k, const int32
                             void *stream);
 
 /*
- * Overlapped reduction of successive batches, a two-stream pipeline.  A
- * submission scores its batch on `score_stream` (tr_score), then selects
- * (tr_select) and gathers (tr_gather) it on `select_stream`, which waits for
- * that scoring only; so the selection and gather of one batch run while the
- * next batch is scored.  Give `select_stream` the higher priority: the score
- * kernel's CTAs retire one by one, and a higher-priority kernel takes the
- * SMs they free.  Submission i uses workspace ws[i mod slots] (each of
- * ws_bytes >= tr_workspace_bytes bytes, 256-byte aligned, owned by the
- * caller) and waits, on score_stream, until the submission that used that
- * workspace last has been gathered.
+ * Overlapped reduction of successive batches, a stream pipeline over `slots`
+ * slots.  Submission i uses slot i mod slots: it scores its batch on
+ * score_streams[slot] (tr_score), then selects (tr_select) and gathers
+ * (tr_gather) it on `select_stream`, which waits for that scoring only.  So
+ * the selection and gather of one batch run while the next batch is scored,
+ * and with a score stream per slot one batch's scoring starts while the
+ * previous score kernel drains.  Give `select_stream` the higher priority:
+ * the score kernel's CTAs retire one by one, and a higher-priority kernel
+ * takes the SMs they free.  The slot's workspace ws[slot] (ws_bytes >=
+ * tr_workspace_bytes bytes, 256-byte aligned, owned by the caller) is reused
+ * only after the submission that used it last has been gathered (the score
+ * stream waits for it).
  *
  * Ordering the caller keeps: the inputs of a submission (x, x', x'') stay
  * unchanged, and its outputs (y, idx, h2, s, d_status) untouched by other
@@ -244,18 +246,21 @@ tr_status tr_reduce_noalloc(const tr_tokens *in, const int32_t *d_k, const int32
  * select_stream (or tr_pipeline_wait).
  *
  * The pipeline owns 2 x slots CUDA events, created on the current device by
- * tr_pipeline_create (make it the device of both streams) and destroyed by
+ * tr_pipeline_create (make it the device of every stream) and destroyed by
  * tr_pipeline_destroy; it allocates no device memory and never synchronises.
+ *   tr_pipeline_create: score_streams holds `slots` cudaStream_t (they may
+ *     repeat one stream); ws holds `slots` workspaces.
  *   tr_pipeline_submit: arguments as in tr_reduce, except that d_status is
  *     zeroed by the call itself (on select_stream, before the selection);
  *     score_begin / score_end are optional cudaEvent_t (or NULL) recorded on
- *     score_stream right before and after the score kernel, to time it.
- *     Host-detectable errors are returned before anything is enqueued.
+ *     the slot's score stream right before and after the score kernel, to
+ *     time it.  Host-detectable errors are returned before anything is
+ *     enqueued.
  *   tr_pipeline_wait: makes `stream` wait for every submission so far.
  */
 #define TR_PIPELINE_MAX_SLOTS 8
 typedef struct tr_pipeline tr_pipeline;
-tr_status tr_pipeline_create(void *score_stream, void *select_stream, int32_t slots, void *const *ws,
+tr_status tr_pipeline_create(void *const *score_streams, void *select_stream, int32_t slots, void *const *ws,
                              size_t ws_bytes, tr_pipeline **out);
 tr_status tr_pipeline_submit(tr_pipeline *p, const tr_tokens *in, const int32_t *d_k, const int32_t *d_k1,
                              const int32_t *d_cu_k, int32_t total_k, void *y, int32_t *idx, float *h2, float *s,

@@ -67,7 +67,7 @@ def load() -> ctypes.CDLL:
     lib.tr_gather.argtypes, lib.tr_gather.restype = [tok, VP, VP, I32, VP, VP], I32
     lib.tr_select_gather.argtypes = [tok, VP, VP, VP, VP, I32, VP, VP, VP, VP, VP, SZ, VP, VP]
     lib.tr_select_gather.restype = I32
-    lib.tr_pipeline_create.argtypes = [VP, VP, I32, P(VP), SZ, P(VP)]
+    lib.tr_pipeline_create.argtypes = [P(VP), VP, I32, P(VP), SZ, P(VP)]
     lib.tr_pipeline_create.restype = I32
     lib.tr_pipeline_submit.argtypes = [VP, tok, VP, VP, VP, I32, VP, VP, VP, VP, VP, VP, VP]
     lib.tr_pipeline_submit.restype = I32

@@ -291,17 +291,18 @@ class Reducer:
 
 
 class Pipeline:
-    """tr_pipeline: successive batches of one shape, each scored on
-    ``score_stream`` and then selected and gathered on ``select_stream``
-    (higher priority), so that the selection and gather of one batch overlap
-    the scoring of the next.  Submission i uses workspace and output set
-    i mod ``slots``; its ReduceResult holds that set's tensors, valid once
-    ``select_stream`` has passed the submission (``wait`` or
+    """tr_pipeline: successive batches of one shape, each scored on its slot's
+    stream of ``score_streams`` and then selected and gathered on
+    ``select_stream`` (higher priority), so that the selection and gather of
+    one batch overlap the scoring of the next, and one batch's scoring the
+    drain of the previous one.  Submission i uses workspace, score stream and
+    output set i mod ``slots``; its ReduceResult holds that set's tensors,
+    valid once ``select_stream`` has passed the submission (``wait`` or
     ``synchronize``) and until submission i + ``slots`` is made.
     """
 
     def __init__(self, seqlens, d, dtype, device, k=None, ratio=None, lam=(1, 3), alias_pre=False, scores=False,
-                 budget=None, slots=2, stride="alg1"):
+                 budget=None, slots=2, stride="alg1", score_streams=None):
         self.lib = load()
         self.seqlens = [int(v) for v in seqlens]
         self.device = torch.device(device)
@@ -318,7 +319,9 @@ class Pipeline:
                           h2=mk(t, dt=torch.float32) if scores else None, s=mk(t, dt=torch.float32) if scores else None,
                           status=torch.zeros(TR_STATUS_WORDS, dtype=torch.int32, device=dev))
                      for _ in range(self.slots)]
-        self.score_stream = torch.cuda.Stream(dev, priority=0)
+        n_streams = self.slots if score_streams is None else max(1, min(int(score_streams), self.slots))
+        own = [torch.cuda.Stream(dev, priority=0) for _ in range(n_streams)]
+        self.score_streams = [own[i % n_streams] for i in range(self.slots)]
         self.select_stream = torch.cuda.Stream(dev, priority=-100)  # the device's highest priority
         self._host = None  # submit_host: per-slot device inputs, copy streams and reuse events
         self._ws = None
@@ -341,28 +344,31 @@ class Pipeline:
             assert all(w.data_ptr() % 256 == 0 for w in self._ws)
             ptrs = (ctypes.c_void_p * self.slots)(*[w.data_ptr() for w in self._ws])
             handle = ctypes.c_void_p()
+            streams = (ctypes.c_void_p * self.slots)(*[st.cuda_stream for st in self.score_streams])
             with torch.cuda.device(self.device):
                 check("tr_pipeline_create", self.lib.tr_pipeline_create(
-                    ctypes.c_void_p(self.score_stream.cuda_stream), ctypes.c_void_p(self.select_stream.cuda_stream),
-                    self.slots, ptrs, nbytes, ctypes.byref(handle)))
+                    streams, ctypes.c_void_p(self.select_stream.cuda_stream), self.slots, ptrs, nbytes,
+                    ctypes.byref(handle)))
             self._handle = handle
         return self._tok
 
     def submit(self, x, x_pre, x_post, score_events=None, after_current=True) -> ReduceResult:
         """Enqueues one batch; ``score_events`` (two torch.cuda.Event, or
-        None) are recorded on score_stream around the score kernel.  With
+        None) are recorded on the slot's score stream around the score
+        kernel.  With
         ``after_current`` the scoring waits for the work already queued on
         the caller's current stream (where the inputs were written); pass
         False when the inputs are known to be ready."""
         tok = self._bind(x, x_pre, x_post)
         o = self.outs[self.submitted % self.slots]
+        sst = self.score_streams[self.submitted % self.slots]
         if after_current:
-            self.score_stream.wait_stream(torch.cuda.current_stream(self.device))
+            sst.wait_stream(torch.cuda.current_stream(self.device))
         ev = [None, None]
         if score_events is not None:
             for e in score_events:
                 if not e.cuda_event:  # torch creates its events lazily, at the first record
-                    e.record(self.score_stream)
+                    e.record(sst)
             ev = [ctypes.c_void_p(e.cuda_event) for e in score_events]
         check("tr_pipeline_submit", self.lib.tr_pipeline_submit(
             self._handle, tok.ref(), _ptr(self.d_k), _ptr(self.d_k1), _ptr(self.d_cu), self.total_k, _ptr(o["y"]),
@@ -416,7 +422,8 @@ class Pipeline:
 
     def synchronize(self):
         self.select_stream.synchronize()
-        self.score_stream.synchronize()
+        for st in self.score_streams:
+            st.synchronize()
         if self._host is not None:
             self._host["cin"].synchronize()
             self._host["cout"].synchronize()

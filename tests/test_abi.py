@@ -101,12 +101,14 @@ def test_pipeline_host_argument_checks(lib):
     v, VP = ctypes.c_void_p, ctypes.c_void_p
     out = VP()
     ws2 = (VP * 2)(0x100000, 0x200000)
-    assert lib.tr_pipeline_create(None, None, 2, ws2, 4096, None) == 1
-    assert lib.tr_pipeline_create(None, None, 0, ws2, 4096, ctypes.byref(out)) == 1
-    assert lib.tr_pipeline_create(None, None, 9, (VP * 9)(*[0x100000] * 9), 4096, ctypes.byref(out)) == 1
-    assert lib.tr_pipeline_create(None, None, 2, None, 4096, ctypes.byref(out)) == 1
-    assert lib.tr_pipeline_create(None, None, 2, (VP * 2)(0x100000, None), 4096, ctypes.byref(out)) == 5
-    assert lib.tr_pipeline_create(None, None, 2, (VP * 2)(0x100000, 0x200010), 4096, ctypes.byref(out)) == 5
+    st2 = (VP * 2)(None, None)
+    assert lib.tr_pipeline_create(st2, None, 2, ws2, 4096, None) == 1
+    assert lib.tr_pipeline_create(st2, None, 0, ws2, 4096, ctypes.byref(out)) == 1
+    assert lib.tr_pipeline_create((VP * 9)(), None, 9, (VP * 9)(*[0x100000] * 9), 4096, ctypes.byref(out)) == 1
+    assert lib.tr_pipeline_create(st2, None, 2, None, 4096, ctypes.byref(out)) == 1
+    assert lib.tr_pipeline_create(None, None, 2, ws2, 4096, ctypes.byref(out)) == 1
+    assert lib.tr_pipeline_create(st2, None, 2, (VP * 2)(0x100000, None), 4096, ctypes.byref(out)) == 5
+    assert lib.tr_pipeline_create(st2, None, 2, (VP * 2)(0x100000, 0x200010), 4096, ctypes.byref(out)) == 5
     assert out.value is None
     t = _tok()
     assert lib.tr_pipeline_submit(None, ctypes.byref(t), v(0x40000), v(0x40100), v(0x40200), 10, v(0x70000),
