@@ -245,9 +245,10 @@ tr_status tr_reduce_noalloc(const tr_tokens *in, const int32_t *d_k, const int32
  * Work that consumes a submission's outputs orders itself after it on
  * select_stream (or tr_pipeline_wait).
  *
- * The pipeline owns 2 x slots CUDA events, created on the current device by
+ * The pipeline owns 3 x slots CUDA events, created on the current device by
  * tr_pipeline_create (make it the device of every stream) and destroyed by
  * tr_pipeline_destroy; it allocates no device memory and never synchronises.
+ * One host thread at a time may submit to a pipeline (it keeps a count).
  *   tr_pipeline_create: score_streams holds `slots` cudaStream_t (they may
  *     repeat one stream); ws holds `slots` workspaces.
  *   tr_pipeline_submit: arguments as in tr_reduce, except that d_status is

@@ -40,13 +40,14 @@ __global__ void __launch_bounds__(kGatherWarps * 32)
     return;
   }
   const uint4 *src = x + (long long)g * nchunks;
+  constexpr int kU = 4;  // loads in flight per lane (8, and 2- or 4-warp CTAs, measured no faster)
   int c = lane;
-  for (; c + 96 < nchunks; c += 128) {
-    const uint4 v0 = ld_nc(src + c), v1 = ld_nc(src + c + 32), v2 = ld_nc(src + c + 64), v3 = ld_nc(src + c + 96);
-    st_cs(dst + c, v0);
-    st_cs(dst + c + 32, v1);
-    st_cs(dst + c + 64, v2);
-    st_cs(dst + c + 96, v3);
+  for (; c + 32 * (kU - 1) < nchunks; c += 32 * kU) {
+    uint4 v[kU];
+#pragma unroll
+    for (int u = 0; u < kU; ++u) v[u] = ld_nc(src + c + 32 * u);
+#pragma unroll
+    for (int u = 0; u < kU; ++u) st_cs(dst + c + 32 * u, v[u]);
   }
   for (; c < nchunks; c += 32) st_cs(dst + c, ld_nc(src + c));
 }
