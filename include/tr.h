@@ -27,9 +27,10 @@
  *  - Kept indices are local to their image, ascending, and image b's
  *    occupy positions [cu_k[b], cu_k[b+1]) of `idx` and of `y`.
  *  - Ties go to the lower token index, in the top-K1 and in the sort.
- *  - The library keeps no global state besides a per-device "shared memory
- *    limit already raised" flag; calls on different streams may run
- *    concurrently when they use different workspaces.
+ *  - The library keeps no global state besides two per-device caches (the
+ *    "shared memory limit already raised" flags and the SM count, both
+ *    atomic); calls from several host threads or on different streams may
+ *    run concurrently when they use different workspaces and outputs.
  *  - The single-call entry points only enqueue kernels (no allocation,
  *    synchronisation or copies), so they can be captured into a CUDA graph
  *    and replayed; make one call on the device outside the capture first

@@ -8,6 +8,8 @@
 // the same deterministic selection (only replica 0 writes idx and the status
 // words) and copies its 1/R share of the image's kept rows, so the copies of
 // one image overlap the selections of the others on SMs that would be idle.
+#include <atomic>
+
 #include "tr_select_dev.cuh"
 
 namespace tr {
@@ -70,8 +72,12 @@ __global__ void __launch_bounds__(kSelectThreads, 1)
   }
 }
 
-int g_smem_set[64];  // per device: dynamic shared memory limit already raised (bit 0 k_select, bit 1 k_select_gather)
-int g_sms[64];
+// Per device (index & 63): dynamic shared memory limit already raised (bit 0
+// k_select, bit 1 k_select_gather), and the SM count.  Atomic so that first
+// calls from several host threads are well defined (raising the limit twice
+// is harmless).
+std::atomic<int> g_smem_set[64];
+std::atomic<int> g_sms[64];
 
 }  // namespace
 
@@ -97,9 +103,9 @@ cudaError_t launch_select(const SelectArgs &a, cudaStream_t st, int max_ctas) {
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
   const size_t smem = select_smem_bytes(a.max_n);
-  if (!(g_smem_set[dev & 63] & 1)) {
+  if (!(g_smem_set[dev & 63].load() & 1)) {
     if ((err = raise_smem_limit(k_select, dev)) != cudaSuccess) return err;
-    g_smem_set[dev & 63] |= 1;
+    g_smem_set[dev & 63].fetch_or(1);
   }
   const int grid = max_ctas > 0 && max_ctas < a.batch ? max_ctas : a.batch;
   k_select<<<grid, kSelectThreads, smem, st>>>(a);
@@ -109,11 +115,11 @@ cudaError_t launch_select(const SelectArgs &a, cudaStream_t st, int max_ctas) {
 int sm_count() {
   int dev = 0, sms = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return 0;
-  if (!g_sms[dev & 63]) {
+  if (!g_sms[dev & 63].load()) {
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
-    g_sms[dev & 63] = sms;
+    g_sms[dev & 63].store(sms);
   }
-  return g_sms[dev & 63];
+  return g_sms[dev & 63].load();
 }
 
 cudaError_t launch_select_gather(const SelectArgs &a, void *y, cudaStream_t st) {
@@ -121,14 +127,13 @@ cudaError_t launch_select_gather(const SelectArgs &a, void *y, cudaStream_t st) 
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
-  if (!(g_smem_set[dev & 63] & 2)) {
+  if (!(g_smem_set[dev & 63].load() & 2)) {
     if ((err = raise_smem_limit(k_select_gather, dev)) != cudaSuccess) return err;
-    int sms = 0;
-    if ((err = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return err;
-    g_sms[dev & 63] = sms;
-    g_smem_set[dev & 63] |= 2;
+    g_smem_set[dev & 63].fetch_or(2);
   }
-  const int replicas = max(1, min(16, g_sms[dev & 63] / a.batch));
+  const int sms = sm_count();
+  if (sms <= 0) return cudaErrorInvalidDevice;
+  const int replicas = max(1, min(16, sms / a.batch));
   const size_t smem = select_smem_bytes(a.max_n);
   const int nchunks = a.d * elem_bytes(a.dtype) / 16;
   k_select_gather<<<a.batch * replicas, kSelectThreads, smem, st>>>(a, replicas, nchunks, static_cast<uint4 *>(y));

@@ -404,27 +404,44 @@ __device__ __forceinline__ __int128 warp_sum128(__int128 v) {
 }
 
 // value = v * 2^base as a trimmed Big (|v| < 2^127, so at most 5 limbs).
+// Built in registers (compile-time limb indices, selects instead of an
+// indexed array) and stored with one struct write.
 __device__ void int128_to_big(__int128 v, int base, Big &out) {
   const bool neg = v < 0;
   const unsigned __int128 mag = neg ? (unsigned __int128)(-v) : (unsigned __int128)v;
-  out.neg = neg ? 1 : 0;
+  Big t;
+#pragma unroll
+  for (int i = 0; i < kBigLimbs; ++i) t.l[i] = 0u;
   if (mag == 0) {
-    out.n = 0;
-    out.e = 0;
-    out.neg = 0;
+    t.n = 0;
+    t.e = 0;
+    t.neg = 0;
+    out = t;
     return;
   }
   const int q = base >> 5, r = base & 31;  // base = 32 q + r, 0 <= r < 32
   const unsigned __int128 lo = mag << r;
-  uint32_t limb[5] = {(uint32_t)lo, (uint32_t)(lo >> 32), (uint32_t)(lo >> 64), (uint32_t)(lo >> 96),
-                      r ? (uint32_t)(mag >> (128 - r)) : 0u};
-  int hi = 4;
-  while (limb[hi] == 0) --hi;
-  int l = 0;
-  while (limb[l] == 0) ++l;
-  out.n = (uint8_t)(hi - l + 1);
-  for (int i = 0; i < out.n; ++i) out.l[i] = limb[l + i];
-  out.e = (int16_t)(q + l);
+  const uint32_t limb[5] = {(uint32_t)lo, (uint32_t)(lo >> 32), (uint32_t)(lo >> 64), (uint32_t)(lo >> 96),
+                            r ? (uint32_t)(mag >> (128 - r)) : 0u};
+  int first = 4, last = 0;  // lowest and highest non-zero limbs
+#pragma unroll
+  for (int k = 4; k >= 0; --k)
+    if (limb[k]) first = k;
+#pragma unroll
+  for (int k = 0; k < 5; ++k)
+    if (limb[k]) last = k;
+#pragma unroll
+  for (int i = 0; i < 5; ++i) {
+    uint32_t w = 0u;
+#pragma unroll
+    for (int k = i; k < 5; ++k)
+      if (k - i == first) w = limb[k];
+    t.l[i] = w;
+  }
+  t.n = (uint8_t)(last - first + 1);
+  t.e = (int16_t)(q + first);
+  t.neg = neg ? 1 : 0;
+  out = t;
 }
 
 // Window for one exact sum: every term and the sum are below 2^top, where
@@ -1067,12 +1084,14 @@ __device__ __noinline__ uint16_t *sample_sort(const uint32_t *key, uint16_t *a, 
 // buckets: the float each key encodes (v = value, or -value for importance
 // keys, which are stored complemented) is mapped linearly from [vmin, vmax]
 // onto nb buckets -- a monotone map, so concatenated buckets are in order --
-// rows are scattered into their bucket with shared-memory atomics, and each
-// bucket (about one row on the workloads here) is insertion-sorted by
-// (key, row).  Returns nullptr, having changed nothing, when some bucket
-// would hold more than kBucketMax rows (ties, or keys crowded together) or
-// the keys span no usable range: the caller falls back to the radix sort.
-// hist: at least nb words.
+// rows are scattered into their bucket (in b) with shared-memory atomics,
+// and each row's final place is its bucket's start plus the number of
+// bucket members with a smaller (key, row), counted by one thread per row
+// (buckets hold about one row on the workloads here, at most kBucketMax).
+// Returns a, holding the order, or nullptr, having changed nothing, when
+// some bucket would hold more than kBucketMax rows (ties, or keys crowded
+// together), a key encodes NaN, or the keys span no usable range: the caller
+// then takes another sort.  hist: at least nb words.
 constexpr int kBucketMax = 32;
 constexpr int kBuckets = 4096;
 __device__ __forceinline__ float key_value(uint32_t k, bool complemented) {
@@ -1084,10 +1103,12 @@ __device__ uint16_t *bucket_sort(const uint32_t *key, uint16_t *a, uint16_t *b, 
   __shared__ int sh_big;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   float vmin = INFINITY, vmax = -INFINITY;
+  bool nan = false;
   for (int q = tid; q < m; q += blockDim.x) {
     const float v = key_value(key[a[q]], complemented);
     vmin = fminf(vmin, v);
     vmax = fmaxf(vmax, v);
+    nan |= v != v;
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -1103,6 +1124,7 @@ __device__ uint16_t *bucket_sort(const uint32_t *key, uint16_t *a, uint16_t *b, 
   for (int c = tid; c < nb; c += blockDim.x) hist[c] = 0u;
   if (tid == 0) sh_big = 0;
   __syncthreads();
+  if (__syncthreads_or(nan)) return nullptr;  // uniform; NaN has no place in a linear bucket map
   vmin = sh_min[0];
   vmax = sh_max[0];
   for (int w = 1; w < kWarps; ++w) {
@@ -1140,28 +1162,29 @@ __device__ uint16_t *bucket_sort(const uint32_t *key, uint16_t *a, uint16_t *b, 
   }
   __syncthreads();
   // hist[c] is now the end of bucket c, so bucket c spans [hist[c - 1], hist[c])
-  for (int c = tid; c < nb; c += blockDim.x) {
+  for (int q = tid; q < m; q += blockDim.x) {
+    const uint16_t row = b[q];
+    const uint32_t kr = key[row];
+    const int c = bucket(key_value(kr, complemented));
     const int lo = c ? (int)hist[c - 1] : 0, hi = (int)hist[c];
-    for (int i = lo + 1; i < hi; ++i) {
-      const uint16_t row = b[i];
-      const unsigned long long kk = ((unsigned long long)key[row] << 16) | row;
-      int j = i - 1;
-      while (j >= lo && (((unsigned long long)key[b[j]] << 16) | b[j]) > kk) {
-        b[j + 1] = b[j];
-        --j;
-      }
-      b[j + 1] = row;
+    const unsigned long long kk = ((unsigned long long)kr << 16) | row;
+    int rank = 0;
+    for (int j = lo; j < hi; ++j) {
+      const uint16_t r2 = b[j];
+      rank += (((unsigned long long)key[r2] << 16) | r2) < kk;
     }
+    a[lo + rank] = row;
   }
   __syncthreads();
-  return b;
+  return a;
 }
 
 // Ascending order of the m rows listed in a by (key[row], row), a listed in
-// ascending row order: a register bitonic sort up to 2048 rows; above that
-// value buckets, the sample sort when the values crowd into few buckets,
-// and the stable radix sort when the sample sort declines too.  Returns the
-// buffer holding the order.
+// ascending row order: a register bitonic sort up to 512 rows; above that
+// value buckets, and when the values crowd into few buckets a register
+// bitonic sort up to 2048 rows, the sample sort above, and the stable radix
+// sort when the sample sort declines too.  Returns the buffer holding the
+// order.
 __device__ uint16_t *sort_rows(const uint32_t *key, uint16_t *a, uint16_t *b, uint16_t *bid, int m,
                                uint32_t *hist, bool complemented) {
   if (m < 2) return a;
@@ -1171,6 +1194,7 @@ __device__ uint16_t *sort_rows(const uint32_t *key, uint16_t *a, uint16_t *b, ui
     sort_small<1>(key, a, m, scratch);
     return a;
   }
+  if (uint16_t *o = bucket_sort(key, a, b, m, hist, complemented)) return o;
   if (m <= 2 * kSelectThreads) {
     __syncthreads();
     sort_small<2>(key, a, m, scratch);
@@ -1181,7 +1205,6 @@ __device__ uint16_t *sort_rows(const uint32_t *key, uint16_t *a, uint16_t *b, ui
     sort_small<4>(key, a, m, scratch);
     return a;
   }
-  if (uint16_t *o = bucket_sort(key, a, b, m, hist, complemented)) return o;
   if (uint16_t *o = sample_sort(key, a, b, bid, m, hist)) return o;
   return radix_sort(key, a, b, m, hist);
 }

@@ -380,6 +380,26 @@ def test_sort_paths_uneven_and_tied_keys():
         check_reduce(x, xp, xq, [n], ([k], [k1], [0, k]))
 
 
+def test_sort_paths_mid_sizes():
+    # Between 512 and 2048 rows to order, the sort first tries value
+    # buckets (each row ranked inside its bucket by one thread); when a
+    # bucket would hold more than 32 rows it declines and a register bitonic
+    # sort of 1024 or 2048 places orders the rows.  Distinct rows take the
+    # buckets; rows of which three in four are copies of one row (equal s,
+    # the smallest R) take both bitonic sizes, for the consistency order
+    # and, with the importance cut inside the copies, the importance order.
+    for n in (700, 1500):
+        x, xp, xq = _rows(n, 64, 20 + n)
+        check_reduce(x, xp, xq, [n], ([n // 3], [n // 9], [0, n // 3]))
+        tied = [i for i in range(n) if i % 4]
+        x[tied] = 0
+        x[tied, 5] = 1.0
+        xp[tied] = xp[1].clone()
+        xq[tied] = xq[1].clone()
+        for k, k1 in [(n // 2, n // 3), (n // 3, 0)]:
+            check_reduce(x, xp, xq, [n], ([k], [k1], [0, k]))
+
+
 def _mix32(v):
     v &= 0xFFFFFFFF
     v ^= v >> 16
