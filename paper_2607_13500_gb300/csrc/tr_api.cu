@@ -75,7 +75,7 @@ SelectArgs select_args(const tr_tokens *in, const Shape &sh, const float *stats,
 
 tr_status select_capped(const tr_tokens *in, const float *stats, const int32_t *d_k, const int32_t *d_k1,
                         const int32_t *d_cu_k, int32_t *idx, uint8_t *role, float *h2, float *s, void *ws,
-                        size_t ws_bytes, int32_t *d_status, void *stream, int max_ctas) {
+                        size_t ws_bytes, int32_t *d_status, void *stream, int max_ctas, bool pdl) {
   Shape sh;
   tr_status rc = check_tokens(in, &sh);
   if (rc != TR_OK) return rc;
@@ -83,7 +83,20 @@ tr_status select_capped(const tr_tokens *in, const float *stats, const int32_t *
   if (misaligned(stats, 16)) return TR_ERR_ALIGN;
   if ((rc = check_ws(sh, ws, ws_bytes)) != TR_OK) return rc;
   SelectArgs a = select_args(in, sh, stats, d_k, d_k1, d_cu_k, idx, role, h2, s, ws, d_status);
-  cudaError_t err = launch_select(a, static_cast<cudaStream_t>(stream), max_ctas);
+  cudaError_t err = launch_select(a, static_cast<cudaStream_t>(stream), max_ctas, pdl);
+  return err == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+}
+
+tr_status gather_impl(const tr_tokens *in, const int32_t *d_cu_k, const int32_t *idx, int32_t total_k, void *y,
+                      void *stream, bool pdl) {
+  Shape sh;
+  tr_status rc = check_tokens(in, &sh);
+  if (rc != TR_OK) return rc;
+  if (total_k < 0 || total_k > sh.total) return TR_ERR_BUDGET;
+  if (total_k > 0 && (!d_cu_k || !idx || !y || in->batch == 0)) return TR_ERR_ARG;
+  if (misaligned(y, 16)) return TR_ERR_ALIGN;
+  cudaError_t err = launch_gather(in->x, sh.total, in->dtype, in->d, in->batch, in->cu_seqlens ? 0 : in->n,
+                                  in->cu_seqlens, d_cu_k, idx, total_k, y, static_cast<cudaStream_t>(stream), pdl);
   return err == cudaSuccess ? TR_OK : TR_ERR_CUDA;
 }
 
@@ -152,7 +165,7 @@ tr_status tr_score(const tr_tokens *in, float *stats, float *h2, float *s, void 
 tr_status tr_select(const tr_tokens *in, const float *stats, const int32_t *d_k, const int32_t *d_k1,
                     const int32_t *d_cu_k, int32_t *idx, uint8_t *role, float *h2, float *s, void *ws,
                     size_t ws_bytes, int32_t *d_status, void *stream) {
-  return select_capped(in, stats, d_k, d_k1, d_cu_k, idx, role, h2, s, ws, ws_bytes, d_status, stream, 0);
+  return select_capped(in, stats, d_k, d_k1, d_cu_k, idx, role, h2, s, ws, ws_bytes, d_status, stream, 0, true);
 }
 
 tr_status tr_select_gather(const tr_tokens *in, const float *stats, const int32_t *d_k, const int32_t *d_k1,
@@ -166,7 +179,7 @@ tr_status tr_select_gather(const tr_tokens *in, const float *stats, const int32_
   if (misaligned(stats, 16) || misaligned(y, 16)) return TR_ERR_ALIGN;
   if ((rc = check_ws(sh, ws, ws_bytes)) != TR_OK) return rc;
   SelectArgs a = select_args(in, sh, stats, d_k, d_k1, d_cu_k, idx, nullptr, h2, s, ws, d_status);
-  cudaError_t err = launch_select_gather(a, y, static_cast<cudaStream_t>(stream));
+  cudaError_t err = launch_select_gather(a, y, static_cast<cudaStream_t>(stream), true);
   return err == cudaSuccess ? TR_OK : TR_ERR_CUDA;
 }
 
@@ -195,15 +208,7 @@ tr_status tr_reduce(const tr_tokens *in, const int32_t *d_k, const int32_t *d_k1
 
 tr_status tr_gather(const tr_tokens *in, const int32_t *d_cu_k, const int32_t *idx, int32_t total_k, void *y,
                     void *stream) {
-  Shape sh;
-  tr_status rc = check_tokens(in, &sh);
-  if (rc != TR_OK) return rc;
-  if (total_k < 0 || total_k > sh.total) return TR_ERR_BUDGET;
-  if (total_k > 0 && (!d_cu_k || !idx || !y || in->batch == 0)) return TR_ERR_ARG;
-  if (misaligned(y, 16)) return TR_ERR_ALIGN;
-  cudaError_t err = launch_gather(in->x, sh.total, in->dtype, in->d, in->batch, in->cu_seqlens ? 0 : in->n,
-                                  in->cu_seqlens, d_cu_k, idx, total_k, y, static_cast<cudaStream_t>(stream));
-  return err == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+  return gather_impl(in, d_cu_k, idx, total_k, y, stream, true);
 }
 
 // ---------------------------------------------------------------- pipeline
@@ -288,10 +293,10 @@ tr_status tr_pipeline_submit(tr_pipeline *p, const tr_tokens *in, const int32_t 
   // caps of 1/2 and 1/8: best or equal on every workload; 256 per-frame
   // video images 198 us per step against 205 us uncapped.)
   const int cap = (sm_count() + 3) / 4;
-  if ((rc = select_capped(in, stats, d_k, d_k1, d_cu_k, idx, nullptr, h2, s, ws, p->ws_bytes, d_status, b,
-                          cap)) != TR_OK)
+  if ((rc = select_capped(in, stats, d_k, d_k1, d_cu_k, idx, nullptr, h2, s, ws, p->ws_bytes, d_status, b, cap,
+                          false)) != TR_OK)
     return rc;
-  if ((rc = tr_gather(in, d_cu_k, idx, total_k, y, b)) != TR_OK) return rc;
+  if ((rc = gather_impl(in, d_cu_k, idx, total_k, y, b, false)) != TR_OK) return rc;
   if (cudaEventRecord(p->done[slot], b) != cudaSuccess) return TR_ERR_CUDA;
   ++p->submitted;
   return TR_OK;

@@ -23,6 +23,7 @@ __global__ void __launch_bounds__(kGatherWarps * 32)
     k_gather(const uint4 *__restrict__ x, long long total_rows, int batch, int n_uniform,
              const int32_t *__restrict__ cu_seqlens, const int32_t *__restrict__ cu_k,
              const int32_t *__restrict__ idx, int total_k, int nchunks, uint4 *__restrict__ y) {
+  pdl_wait();  // idx comes from the kernel before this one
   const int lane = threadIdx.x & 31;
   const int row = blockIdx.x * kGatherWarps + (threadIdx.x >> 5);
   if (row >= total_k) return;
@@ -33,7 +34,7 @@ __global__ void __launch_bounds__(kGatherWarps * 32)
     if (__ldg(cu_k + mid) <= row) lo = mid; else hi = mid;
   }
   const long long first = cu_seqlens ? (long long)__ldg(cu_seqlens + lo) : (long long)lo * n_uniform;
-  const long long g = first + __ldg(idx + row);
+  const long long g = first + __ldcg(idx + row);  // through L2: idx may come from the kernel before
   uint4 *dst = y + (long long)row * nchunks;
   if (g < 0 || g >= total_rows) {  // never address outside x: bad indices write zeros
     for (int c = lane; c < nchunks; c += 32) st_cs(dst + c, make_uint4(0u, 0u, 0u, 0u));
@@ -56,13 +57,13 @@ __global__ void __launch_bounds__(kGatherWarps * 32)
 
 cudaError_t launch_gather(const void *x, long long total_rows, int dtype, int d, int batch, int n_uniform,
                           const int32_t *cu_seqlens, const int32_t *cu_k, const int32_t *idx, int total_k, void *y,
-                          cudaStream_t st) {
+                          cudaStream_t st, bool pdl) {
   if (total_k == 0) return cudaSuccess;
   const int nchunks = d * elem_bytes(dtype) / 16;
   const int grid = (total_k + kGatherWarps - 1) / kGatherWarps;
-  k_gather<<<grid, kGatherWarps * 32, 0, st>>>(static_cast<const uint4 *>(x), total_rows, batch, n_uniform,
-                                                cu_seqlens, cu_k, idx, total_k, nchunks, static_cast<uint4 *>(y));
-  return cudaGetLastError();
+  return launch_kernel(k_gather, dim3(grid), dim3(kGatherWarps * 32), 0, st, pdl, static_cast<const uint4 *>(x),
+                       total_rows, batch, n_uniform, cu_seqlens, cu_k, idx, total_k, nchunks,
+                       static_cast<uint4 *>(y));
 }
 
 }  // namespace tr

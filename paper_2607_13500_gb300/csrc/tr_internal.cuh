@@ -5,6 +5,7 @@
 
 #include <cstddef>
 #include <cstdint>
+#include <utility>
 
 #include "tr.h"
 
@@ -130,6 +131,34 @@ inline WsLayout ws_layout(long long total_rows) {
   return w;
 }
 
+// ---------------------------------------------------------------- launch order
+// Programmatic dependent launch: a kernel launched with pdl = true may be
+// scheduled while the kernel before it on the stream still runs, once every
+// CTA of that kernel has called pdl_trigger() (or exited); it calls
+// pdl_wait() before it reads anything that kernel writes (the wait returns
+// at once after a normal launch).  This hides the launch of a kernel behind
+// the tail of the one before it: the single-call entry points use it, the
+// pipeline does not (there a waiting grid would hold SMs that the next
+// batch's scoring needs).
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+template <typename... P, typename... A>
+cudaError_t launch_kernel(void (*kernel)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, bool pdl,
+                          A &&...args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<A>(args)...);
+}
+
 // ---------------------------------------------------------------- launchers
 struct SelectArgs {
   const void *x, *x_pre, *x_post;
@@ -150,12 +179,13 @@ struct SelectArgs {
 size_t select_smem_bytes(int max_n);  // dynamic shared memory of one select CTA
 cudaError_t launch_score(const void *x, const void *x_pre, const void *x_post, int dtype, int d, long long total,
                          float *stats, float *h2, float *s, cudaStream_t st);
-// max_ctas > 0 caps the grid (each CTA then selects several images in turn).
-cudaError_t launch_select(const SelectArgs &a, cudaStream_t st, int max_ctas = 0);
+// max_ctas > 0 caps the grid (each CTA then selects several images in turn);
+// pdl: programmatic dependent launch after the kernel before it on st.
+cudaError_t launch_select(const SelectArgs &a, cudaStream_t st, int max_ctas, bool pdl);
 int sm_count();  // SMs of the current device (cached), 0 on error
-cudaError_t launch_select_gather(const SelectArgs &a, void *y, cudaStream_t st);
+cudaError_t launch_select_gather(const SelectArgs &a, void *y, cudaStream_t st, bool pdl);
 cudaError_t launch_gather(const void *x, long long total_rows, int dtype, int d, int batch, int n_uniform,
                           const int32_t *cu_seqlens, const int32_t *cu_k, const int32_t *idx, int total_k, void *y,
-                          cudaStream_t st);
+                          cudaStream_t st, bool pdl);
 
 }  // namespace tr

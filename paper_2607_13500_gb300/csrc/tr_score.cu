@@ -11,6 +11,7 @@ template <int kDt>
 __global__ void __launch_bounds__(kScoreWarps * 32)
     k_score(const uint4 *__restrict__ x, const uint4 *__restrict__ xp, const uint4 *__restrict__ xq, int nchunks,
             long long total, float4 *__restrict__ stats, float *__restrict__ h2, float *__restrict__ s_out) {
+  pdl_trigger();  // a dependent selection may be scheduled once every CTA runs
   const int lane = threadIdx.x & 31;
   const long long stride = (long long)gridDim.x * kScoreWarps;
   for (long long row = (long long)blockIdx.x * kScoreWarps + (threadIdx.x >> 5); row < total; row += stride)

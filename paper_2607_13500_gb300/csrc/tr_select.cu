@@ -19,6 +19,8 @@ namespace {
 // launch caps the grid below the batch).
 __global__ void __launch_bounds__(kSelectThreads, 1) k_select(const SelectArgs a) {
   extern __shared__ __align__(16) unsigned char smem[];
+  pdl_trigger();
+  pdl_wait();  // the statistics come from the kernel before this one
   for (int b = blockIdx.x; b < a.batch; b += gridDim.x) select_image(a, b, smem);
 }
 
@@ -33,6 +35,7 @@ __device__ __forceinline__ uint4 ld_nc16(const uint4 *p) {
 __global__ void __launch_bounds__(kSelectThreads, 1)
     k_select_gather(const SelectArgs a, const int replicas, const int nchunks, uint4 *__restrict__ y) {
   extern __shared__ __align__(16) unsigned char smem[];
+  pdl_wait();  // the statistics come from the kernel before this one
   const int b = blockIdx.x / replicas, r = blockIdx.x % replicas;
   select_image(a, b, smem, r == 0);
   long long off;
@@ -97,7 +100,7 @@ cudaError_t raise_smem_limit(K kernel, int dev) {
   return cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, optin - (int)fa.sharedSizeBytes);
 }
 
-cudaError_t launch_select(const SelectArgs &a, cudaStream_t st, int max_ctas) {
+cudaError_t launch_select(const SelectArgs &a, cudaStream_t st, int max_ctas, bool pdl) {
   if (a.batch == 0) return cudaSuccess;
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
@@ -108,8 +111,7 @@ cudaError_t launch_select(const SelectArgs &a, cudaStream_t st, int max_ctas) {
     g_smem_set[dev & 63].fetch_or(1);
   }
   const int grid = max_ctas > 0 && max_ctas < a.batch ? max_ctas : a.batch;
-  k_select<<<grid, kSelectThreads, smem, st>>>(a);
-  return cudaGetLastError();
+  return launch_kernel(k_select, dim3(grid), dim3(kSelectThreads), smem, st, pdl, a);
 }
 
 int sm_count() {
@@ -122,7 +124,7 @@ int sm_count() {
   return g_sms[dev & 63].load();
 }
 
-cudaError_t launch_select_gather(const SelectArgs &a, void *y, cudaStream_t st) {
+cudaError_t launch_select_gather(const SelectArgs &a, void *y, cudaStream_t st, bool pdl) {
   if (a.batch == 0) return cudaSuccess;
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
@@ -136,8 +138,8 @@ cudaError_t launch_select_gather(const SelectArgs &a, void *y, cudaStream_t st) 
   const int replicas = max(1, min(16, sms / a.batch));
   const size_t smem = select_smem_bytes(a.max_n);
   const int nchunks = a.d * elem_bytes(a.dtype) / 16;
-  k_select_gather<<<a.batch * replicas, kSelectThreads, smem, st>>>(a, replicas, nchunks, static_cast<uint4 *>(y));
-  return cudaGetLastError();
+  return launch_kernel(k_select_gather, dim3(a.batch * replicas), dim3(kSelectThreads), smem, st, pdl, a, replicas,
+                       nchunks, static_cast<uint4 *>(y));
 }
 
 }  // namespace tr
