@@ -115,3 +115,20 @@ def test_pipeline_host_argument_checks(lib):
                                   v(0x50000), None, None, None, None, None) == 1
     assert lib.tr_pipeline_wait(None, None) == 1
     assert lib.tr_pipeline_destroy(None) == 0
+
+
+def test_missing_library_raises(monkeypatch, tmp_path):
+    # The product path has no CPU fallback: without libtr.so every entry
+    # point fails loudly instead of computing anything on the host.
+    monkeypatch.setattr(_lib, "LIB_PATH", str(tmp_path / "libtr.so"))
+    monkeypatch.setattr(_lib, "_lib", None)
+    with pytest.raises(RuntimeError, match="missing"):
+        _lib.load()
+    import torch
+
+    import paper_2607_13500_gb300 as altr
+    x = torch.zeros(1, 8, 64, dtype=torch.bfloat16)  # host tensors are refused too
+    with pytest.raises(ValueError, match="no CPU path"):
+        altr.reduce(x, x, x, k=2)
+    with pytest.raises(RuntimeError, match="missing"):
+        altr.budgets([8], k=2)
