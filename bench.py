@@ -66,6 +66,9 @@ def _args():
     ap.add_argument("--lam", default="1/3", help="balance lambda = K1 / K as a rational num/den (Algorithm 1)")
     ap.add_argument("--stride", choices=["alg1", "interval"], default="alg1",
                     help="diversity pick positions: Algorithm 1's integer stride or Section IV-B's real interval")
+    ap.add_argument("--sweep", default=None,
+                    help="also time the pipeline over one parameter, e.g. k=64,128,192 | ratio=1/9,2/9 | "
+                         "lam=0/1,1/3,1/1 | batch=1,8,64; results go to the line's \"sweep\" list")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     a = ap.parse_args()
@@ -273,6 +276,69 @@ def _traffic_per_row(workload):
     return float(m_bpr.group(1))
 
 
+# ---------------------------------------------------------------- parameter sweeps
+def _sweep_points(spec):
+    """'k=64,128' -> ('k', [64, 128]); ratios and lambdas as (num, den)."""
+    name, _, vals = spec.partition("=")
+    if name not in ("k", "ratio", "lam", "batch") or not vals:
+        raise SystemExit(f"--sweep: expected k=..., ratio=..., lam=... or batch=..., got {spec!r}")
+    out = []
+    for v in vals.split(","):
+        if name in ("ratio", "lam"):
+            num, den = (int(t) for t in v.split("/"))
+            out.append((num, den))
+        else:
+            out.append(int(v))
+    return name, out
+
+
+def run_sweep(args, dev, altr, w0, budget0, peak):
+    """The two-slot pipeline timed (CUDA events, inputs resident) at each
+    value of one parameter, the others as in the main line."""
+    name, points = _sweep_points(args.sweep)
+    res = []
+    for v in points:
+        budget, lam, w = dict(budget0), _lam(args), w0
+        if name == "k":
+            budget = dict(k=v)
+        elif name == "ratio":
+            budget = dict(ratio=v)
+        elif name == "lam":
+            lam = v
+        else:
+            w = synth.make(args.workload, seed=args.seed, device=dev, batch=v)
+            if args.per_frame:
+                w = w.frames()
+        pipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, slots=2, stride=args.stride, lam=lam, **budget)
+        for _ in range(max(3, args.warmup)):
+            pipe.submit(w.x, w.x_pre, w.x_post)
+        pipe.synchronize()
+        t0 = time.perf_counter()
+        pipe.submit(w.x, w.x_pre, w.x_post)
+        pipe.synchronize()
+        steps = int(max(10, min(args.steps, 1.0 / max(time.perf_counter() - t0, 1e-6))))
+        start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        cur = torch.cuda.current_stream(dev)
+        start.record(cur)
+        for strm in pipe.score_streams + [pipe.select_stream]:
+            strm.wait_stream(cur)
+        for _ in range(steps):
+            pipe.submit(w.x, w.x_pre, w.x_post, after_current=False)
+        pipe.wait(cur)
+        end.record(cur)
+        torch.cuda.synchronize()
+        ms = start.elapsed_time(end) / steps
+        e = 2 if w.x.dtype in (torch.bfloat16, torch.float16) else 4
+        gbs = synth.algorithmic_bytes(w.seqlens, pipe.ks, w.d, e) / (ms * 1e-3) / 1e9
+        status = pipe.outs[(pipe.submitted - 1) % pipe.slots]["status"].cpu().tolist()
+        pipe.close()
+        res.append({name: list(v) if isinstance(v, tuple) else v, "batch": w.batch, "total_k": pipe.total_k,
+                    "steps": steps, "ms_per_step": ms, "value": w.batch / (ms * 1e-3), "unit": "images/s",
+                    "hbm_gbs": gbs, "frac_of_measured": gbs / peak, "status": status})
+        del pipe
+    return res
+
+
 # ---------------------------------------------------------------- our arm
 def run_ours(args, world, rank, local):
     dev = torch.device("cuda", local)
@@ -413,6 +479,8 @@ def run_ours(args, world, rank, local):
         "clocks": clk,
         "status": st,
     }
+    if args.sweep:
+        line["sweep"] = run_sweep(args, dev, altr, w, budget, peak)
     if rank == 0 and world == 1:
         line["cpu_baseline"] = cpu_baseline(w, red.ks, red.k1s, args.cpu_seconds, args.stride)
     if rank == 0:
