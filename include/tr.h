@@ -35,6 +35,12 @@
  *    synchronisation or copies), so they can be captured into a CUDA graph
  *    and replayed; make one call on the device outside the capture first
  *    (it raises the kernels' shared-memory limit once).
+ *  - tr_select, tr_gather, tr_select_gather and tr_reduce launch their
+ *    kernels with programmatic dependent launch: a kernel may be scheduled
+ *    while the kernel before it on the stream finishes, and waits in
+ *    hardware for that kernel's completion before it reads anything, so
+ *    stream order is kept (tr_score's kernel lets such a successor in as
+ *    soon as all its CTAs run).  The pipeline launches normally.
  */
 #ifndef TR_H
 #define TR_H
