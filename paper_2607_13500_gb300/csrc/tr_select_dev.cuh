@@ -5,10 +5,11 @@
 // so ranking by H2 is ranking by R; s = P / sqrt(A B) (Eq. 6).  The score
 // pass leaves fp32 keys R32 and s32 in each row's statistics record.  Stage
 // I finds the K1-th key by a radix select and needs an order only near an
-// uncertain cut; Stage II sorts X_rem by s (register bitonic sort of keys
-// packed with the token index into 64-bit words up to 2048 rows, else value
-// buckets, a stratified sample sort or a stable radix sort), so that equal
-// keys order by the lower index.
+// uncertain cut; Stage II sorts X_rem by s (keys packed with the token index
+// into 64-bit words: a register bitonic sort up to 512 rows, else value
+// buckets ranked per row, and where the values crowd a register bitonic sort
+// up to 2048 rows, a stratified sample sort or a stable radix sort), so that
+// equal keys order by the lower index.
 //
 // Certification.  The score pass's sums carry proven error bounds (Bounds),
 // so a cut between sorted neighbours is certain when their key intervals do
