@@ -43,6 +43,9 @@ L2_BYTES = 129 * 2 ** 20
 
 # workload -> budget at which it is timed (the paper's headline K = 192 for the
 # 576-token LLaVA-1.5 images; the other shapes' larger budgets)
+GRAPH_STEPS = 16                   # pipelined steps per captured graph (--submit graph)
+GRAPH_BELOW_BYTES = 32 * 2 ** 20   # --submit auto: graph replays below this many input bytes per step
+
 BUDGETS = {
     "llava576": dict(k=192),
     "multitile2880": dict(k=320),
@@ -69,6 +72,9 @@ def _args():
     ap.add_argument("--sweep", default=None,
                     help="also time the pipeline over one parameter, e.g. k=64,128,192 | ratio=1/9,2/9 | "
                          "lam=0/1,1/3,1/1 | batch=1,8,64; results go to the line's \"sweep\" list")
+    ap.add_argument("--submit", choices=["auto", "host", "graph"], default="auto",
+                    help="timed steps submitted from the host, or as replays of a CUDA graph of pipelined steps "
+                         "(auto: graph below 32 MiB of input per step)")
     ap.add_argument("--e2e-steps", type=int, default=20)
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     a = ap.parse_args()
@@ -384,28 +390,52 @@ def run_ours(args, world, rank, local):
     latency_us = 1e3 * statistics.median(ev[0].elapsed_time(ev[1]) for ev in lat_evs[1:])
     del graph
 
-    clocks = ClockSampler(dev)
-    for _ in range(args.warmup):
-        pipe.submit(w.x, w.x_pre, w.x_post)
-    pipe.synchronize()
-    st = pipe.outs[(pipe.submitted - 1) % pipe.slots]["status"].cpu().tolist()
-    # timed region: K steps through the two-stream pipeline (the selection
-    # and gather of step i overlap the scoring of step i + 1), the score
-    # kernel bracketed by events on its stream in every step
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+    # Submission: from the host step by step, or -- for batches so small that
+    # a host submission (tens of microseconds from Python) outlasts the GPU
+    # work -- replays of a CUDA graph of S pipelined steps (S divides K).
+    mode = args.submit if args.submit != "auto" else ("graph" if in_bytes < GRAPH_BELOW_BYTES else "host")
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    barrier()
-    torch.cuda.synchronize()
     cur = torch.cuda.current_stream(dev)
-    start.record(cur)
-    for strm in pipe.score_streams + [pipe.select_stream]:
-        strm.wait_stream(cur)  # nothing of the timed steps starts before `start`
-    for i in range(args.steps):  # the inputs stay resident and unchanged
-        pipe.submit(w.x, w.x_pre, w.x_post, score_events=evs[i], after_current=False)
-    pipe.wait(cur)
-    end.record(cur)
-    torch.cuda.synchronize()
-    barrier()
+    clocks = ClockSampler(dev)
+    if mode == "graph":
+        per_graph = max(s_ for s_ in range(1, min(GRAPH_STEPS, args.steps) + 1) if args.steps % s_ == 0)
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(per_graph)]
+        graph = pipe.graph(w.x, w.x_pre, w.x_post, steps=per_graph, score_events=evs)
+        for _ in range(-(-args.warmup // per_graph)):
+            graph.replay()
+        torch.cuda.synchronize()
+        st = pipe.outs[(per_graph - 1) % pipe.slots]["status"].cpu().tolist()
+        barrier()
+        torch.cuda.synchronize()
+        start.record(cur)
+        for _ in range(args.steps // per_graph):  # the last replay's events time its score kernels
+            graph.replay()
+        end.record(cur)
+        torch.cuda.synchronize()
+        barrier()
+        submission = f"CUDA graph of {per_graph} pipelined steps, {args.steps // per_graph} replays"
+        del graph
+    else:
+        for _ in range(args.warmup):
+            pipe.submit(w.x, w.x_pre, w.x_post)
+        pipe.synchronize()
+        st = pipe.outs[(pipe.submitted - 1) % pipe.slots]["status"].cpu().tolist()
+        # timed region: K steps through the two-stream pipeline (the selection
+        # and gather of step i overlap the scoring of step i + 1), the score
+        # kernel bracketed by events on its stream in every step
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+        barrier()
+        torch.cuda.synchronize()
+        start.record(cur)
+        for strm in pipe.score_streams + [pipe.select_stream]:
+            strm.wait_stream(cur)  # nothing of the timed steps starts before `start`
+        for i in range(args.steps):  # the inputs stay resident and unchanged
+            pipe.submit(w.x, w.x_pre, w.x_post, score_events=evs[i], after_current=False)
+        pipe.wait(cur)
+        end.record(cur)
+        torch.cuda.synchronize()
+        barrier()
+        submission = "host, one submission per step"
     clk = clocks.stop()
     total_ms = start.elapsed_time(end)
     # k_score's launches overlap one another in the pipeline (a score stream
@@ -471,6 +501,7 @@ def run_ours(args, world, rank, local):
         "hbm_gbs": path_gbs, "frac_of_8tbs": path_gbs / NOMINAL_HBM_GBS, "frac_of_measured": path_gbs / peak,
         "kernels_ms": {"k_score_in_pipeline": score_ms, **{f"{k}_alone": v for k, v in alone.items()}},
         "pipeline": "2 slots, a score stream each: step i's k_select + k_gather (high-priority stream) overlap step i+1's k_score",
+        "submission": submission,
         "latency_us": {"tr_reduce_graph_replay": latency_us},
         "roofline": roofline,
         "e2e": {"value": images / e2e_s, "unit": "images/s", "h2d_bytes_per_step": in_bytes,

@@ -262,9 +262,17 @@ tr_status tr_reduce_noalloc(const tr_tokens *in, const int32_t *d_k, const int32
  *     zeroed by the call itself (on select_stream, before the selection);
  *     score_begin / score_end are optional cudaEvent_t (or NULL) recorded on
  *     the slot's score stream right before and after the score kernel, to
- *     time it.  Host-detectable errors are returned before anything is
- *     enqueued.
+ *     time it (as event-record nodes when the stream is being captured).
+ *     Host-detectable errors are returned before anything is enqueued.
  *   tr_pipeline_wait: makes `stream` wait for every submission so far.
+ *
+ * Graph capture: submissions made while the streams are captured into a
+ * CUDA graph (forked from the capturing stream, joined back with
+ * tr_pipeline_wait and a wait on each score stream) become one graph whose
+ * replay runs those steps, overlapped as above, with a single launch.  Use a
+ * pipeline created for the capture (no submission before it: the first
+ * `slots` submissions of a pipeline wait on no earlier event) and only
+ * replay it afterwards.
  */
 #define TR_PIPELINE_MAX_SLOTS 8
 typedef struct tr_pipeline tr_pipeline;

@@ -328,6 +328,7 @@ class Pipeline:
         self._handle = None
         self._tok = None
         self._in = None
+        self._graphed = False
         self.submitted = 0
 
     def _bind(self, x, x_pre, x_post):
@@ -340,7 +341,8 @@ class Pipeline:
             nbytes = self.lib.tr_workspace_bytes(self._tok.ref())
             if nbytes == 0:
                 raise ValueError("invalid token tensors for tr_pipeline")
-            self._ws = [torch.empty(nbytes, dtype=torch.uint8, device=self.device) for _ in range(self.slots)]
+            if self._ws is None or self._ws[0].numel() < nbytes:
+                self._ws = [torch.empty(nbytes, dtype=torch.uint8, device=self.device) for _ in range(self.slots)]
             assert all(w.data_ptr() % 256 == 0 for w in self._ws)
             ptrs = (ctypes.c_void_p * self.slots)(*[w.data_ptr() for w in self._ws])
             handle = ctypes.c_void_p()
@@ -359,6 +361,8 @@ class Pipeline:
         ``after_current`` the scoring waits for the work already queued on
         the caller's current stream (where the inputs were written); pass
         False when the inputs are known to be ready."""
+        if self._graphed and not torch.cuda.is_current_stream_capturing():
+            raise RuntimeError("this pipeline was captured by Pipeline.graph: replay the graph instead")
         tok = self._bind(x, x_pre, x_post)
         o = self.outs[self.submitted % self.slots]
         sst = self.score_streams[self.submitted % self.slots]
@@ -413,6 +417,42 @@ class Pipeline:
             out.record(h["cout"])
         h["out_free"][slot] = out
         return r
+
+    def graph(self, x, x_pre, x_post, steps=16, score_events=None) -> "torch.cuda.CUDAGraph":
+        """``steps`` pipelined submissions of these input tensors captured into
+        one CUDA graph: ``replay()`` runs them (each step's selection and
+        gather overlapping the next step's scoring) with a single launch, for
+        batches so small that submitting step by step from the host would
+        take longer than the GPU work.  ``score_events`` (``steps`` pairs of
+        timing torch.cuda.Event, or None) become event nodes around each score
+        kernel.  Step i writes output set i mod ``slots``.  The pipeline is
+        dedicated to replays afterwards (``submit`` raises)."""
+        if self.submitted and self._handle is not None:
+            raise RuntimeError("Pipeline.graph needs a pipeline without earlier submissions")
+        cur = torch.cuda.current_stream(self.device)
+        # one step outside the capture: the selection kernel's shared-memory
+        # limit is raised once per device, on its first launch
+        self.submit(x, x_pre, x_post)
+        self.synchronize()
+        self.lib.tr_pipeline_destroy(self._handle)  # a fresh handle: no earlier events to wait on
+        self._handle = None
+        self.submitted = 0
+        self._bind(x, x_pre, x_post)
+        if score_events is not None:
+            for pair in score_events:
+                for e in pair:
+                    e.record(cur)  # created before the capture
+        cur.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            cap = torch.cuda.current_stream(self.device)
+            for i in range(steps):
+                self.submit(x, x_pre, x_post, score_events=None if score_events is None else score_events[i])
+            self.wait(cap)
+            for st in self.score_streams:
+                cap.wait_stream(st)
+        self._graphed = True
+        return g
 
     def wait(self, stream=None):
         """Makes ``stream`` (default: the current stream) wait for every submission."""

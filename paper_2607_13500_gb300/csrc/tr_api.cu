@@ -1,5 +1,6 @@
 // Host side of the C ABI declared in include/tr.h: argument checks, budgets,
 // workspace carving and launches (tr_reduce: score, then select + gather).
+#include <algorithm>
 #include <climits>
 
 #include <new>
@@ -279,10 +280,19 @@ tr_status tr_pipeline_submit(tr_pipeline *p, const tr_tokens *in, const int32_t 
   const int prev = (int)((p->submitted + p->slots - 1) % p->slots);
   if (sh.total > 20 * wave_rows && p->submitted > 0 && cudaStreamWaitEvent(a, p->head[prev], 0) != cudaSuccess)
     return TR_ERR_CUDA;
-  if (score_begin && cudaEventRecord(static_cast<cudaEvent_t>(score_begin), a) != cudaSuccess) return TR_ERR_CUDA;
+  // The caller's timing events become event-record nodes when the stream is
+  // being captured into a graph (cudaEventRecordExternal, which is valid only
+  // during a capture), so that they time each replay.
+  cudaStreamCaptureStatus capturing = cudaStreamCaptureStatusNone;
+  if ((score_begin || score_end) && cudaStreamIsCapturing(a, &capturing) != cudaSuccess) return TR_ERR_CUDA;
+  const unsigned rec_flags =
+      capturing == cudaStreamCaptureStatusActive ? cudaEventRecordExternal : cudaEventRecordDefault;
+  if (score_begin && cudaEventRecordWithFlags(static_cast<cudaEvent_t>(score_begin), a, rec_flags) != cudaSuccess)
+    return TR_ERR_CUDA;
   if ((rc = tr_score(in, stats, h2, s, a)) != TR_OK) return rc;
   if (cudaEventRecord(p->head[slot], a) != cudaSuccess) return TR_ERR_CUDA;
-  if (score_end && cudaEventRecord(static_cast<cudaEvent_t>(score_end), a) != cudaSuccess) return TR_ERR_CUDA;
+  if (score_end && cudaEventRecordWithFlags(static_cast<cudaEvent_t>(score_end), a, rec_flags) != cudaSuccess)
+    return TR_ERR_CUDA;
   if (cudaEventRecord(p->scored[slot], a) != cudaSuccess || cudaStreamWaitEvent(b, p->scored[slot], 0) != cudaSuccess)
     return TR_ERR_CUDA;
   if (d_status && cudaMemsetAsync(d_status, 0, TR_STATUS_WORDS * sizeof(int32_t), b) != cudaSuccess)
@@ -292,11 +302,24 @@ tr_status tr_pipeline_submit(tr_pipeline *p, const tr_tokens *in, const int32_t 
   // next batch at full bandwidth.  (Measured on GB300 against no cap and
   // caps of 1/2 and 1/8: best or equal on every workload; 256 per-frame
   // video images 198 us per step against 205 us uncapped.)
-  const int cap = (sm_count() + 3) / 4;
-  if ((rc = select_capped(in, stats, d_k, d_k1, d_cu_k, idx, nullptr, h2, s, ws, p->ws_bytes, d_status, b, cap,
-                          false)) != TR_OK)
-    return rc;
-  if ((rc = gather_impl(in, d_cu_k, idx, total_k, y, b, false)) != TR_OK) return rc;
+  const int sms = sm_count();
+  const int cap = (sms + 3) / 4;
+  // A uniform batch of one or two small images (up to 1024 tokens) selects
+  // and gathers in one launch (tr_select_gather's replicas: the copy is split
+  // over them and one kernel boundary leaves the step's critical path) when
+  // the replicas stay within the same quarter of the SMs.  (Measured on
+  // GB300: one 576-token image 21.9 -> 20.0 us per step; one 6272-token clip
+  // 66 -> 74 us, its 16 replicas slowing one another, hence the size limit.)
+  const int replicas = in->batch > 0 ? std::max(1, std::min(16, sms / in->batch)) : 0;
+  if (!in->cu_seqlens && in->batch > 0 && in->n <= 1024 && in->batch * replicas <= cap) {
+    SelectArgs a = select_args(in, sh, stats, d_k, d_k1, d_cu_k, idx, nullptr, h2, s, ws, d_status);
+    if (launch_select_gather(a, y, b, false) != cudaSuccess) return TR_ERR_CUDA;
+  } else {
+    if ((rc = select_capped(in, stats, d_k, d_k1, d_cu_k, idx, nullptr, h2, s, ws, p->ws_bytes, d_status, b, cap,
+                            false)) != TR_OK)
+      return rc;
+    if ((rc = gather_impl(in, d_cu_k, idx, total_k, y, b, false)) != TR_OK) return rc;
+  }
   if (cudaEventRecord(p->done[slot], b) != cudaSuccess) return TR_ERR_CUDA;
   ++p->submitted;
   return TR_OK;

@@ -239,6 +239,50 @@ def test_graph_replay_and_limits():
     check_reduce(x, xp, xq, [25, 15], _alt().budgets([25, 15], k=10))
 
 
+@pytest.mark.parametrize("batch", [2, 3])
+def test_pipeline_graph_replay(batch):
+    # Five pipelined steps (two slots, so the slots are reused inside the
+    # graph) captured into one CUDA graph and replayed twice; every slot's
+    # outputs match the oracle, the score events time each replay's score
+    # kernels, and the captured pipeline refuses host submissions.  Two
+    # images select and gather in one launch per step, three in two.
+    altr = _alt()
+    dev = torch.device("cuda")
+    w = synth.make("single_clip336", seed=5, batch=batch)
+    budget = _budget(w, k=64)
+    pipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, budget=budget, scores=True, slots=2)
+    dx, dp, dq = w.x.to(dev), w.x_pre.to(dev), w.x_post.to(dev)
+    try:
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(5)]
+        g = pipe.graph(dx, dp, dq, steps=5, score_events=evs)
+        for o in pipe.outs:
+            o["y"].zero_()
+            o["idx"].fill_(-1)
+        for _ in range(2):
+            g.replay()
+        torch.cuda.synchronize()
+        for o in pipe.outs:
+            r = altr.ReduceResult(o["y"][:pipe.total_k], o["idx"][:pipe.total_k], pipe.cu_k, o["h2"], o["s"],
+                                  o["status"])
+            compare_result(r, w.x, w.x_pre, w.x_post, w.seqlens, budget)
+        assert all(0.0 < e0.elapsed_time(e1) < 1000.0 for e0, e1 in evs)
+        with pytest.raises(RuntimeError, match="captured"):
+            pipe.submit(dx, dp, dq)
+        del g
+    finally:
+        pipe.close()
+    # the same timing events on host submissions
+    pipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, budget=budget, scores=True, slots=2)
+    try:
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(3)]
+        rs = [pipe.submit(dx, dp, dq, score_events=ev) for ev in evs]
+        pipe.synchronize()
+        assert all(0.0 < e0.elapsed_time(e1) < 1000.0 for e0, e1 in evs)
+        compare_result(rs[-1], w.x, w.x_pre, w.x_post, w.seqlens, budget)
+    finally:
+        pipe.close()
+
+
 def test_pipeline_from_host():
     # Pinned host batches in, y and idx back to pinned host buffers, three
     # different batches through two slots (uploads overlap the work).
