@@ -115,6 +115,19 @@ def job_images_per_s(images_per_rank: int, world: int, ms_step_max: float) -> fl
     return images_per_rank * world / (ms_step_max * 1e-3)
 
 
+def step_bytes(w, ks):
+    """Bytes of one step over workload w with budgets ks: the three input
+    tensors (what an end-to-end step copies in), the path's algorithmic
+    traffic (inputs read + kept rows read and written + int32 indices), and
+    what an end-to-end step copies back (y and idx)."""
+    elem = 2 if w.x.dtype in (torch.bfloat16, torch.float16) else 4
+    n_in = 2 if w.x_pre is None else 3
+    total_k = int(sum(ks))
+    return (n_in * w.total * w.d * elem,
+            synth.algorithmic_bytes(w.seqlens, ks, w.d, elem, aliased_pre=w.x_pre is None),
+            total_k * (w.d * elem + 4))
+
+
 def _peaks():
     try:
         with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
@@ -334,8 +347,7 @@ def run_sweep(args, dev, altr, w0, budget0, peak):
         end.record(cur)
         torch.cuda.synchronize()
         ms = start.elapsed_time(end) / steps
-        e = 2 if w.x.dtype in (torch.bfloat16, torch.float16) else 4
-        gbs = synth.algorithmic_bytes(w.seqlens, pipe.ks, w.d, e) / (ms * 1e-3) / 1e9
+        gbs = step_bytes(w, pipe.ks)[1] / (ms * 1e-3) / 1e9
         status = pipe.outs[(pipe.submitted - 1) % pipe.slots]["status"].cpu().tolist()
         pipe.close()
         res.append({name: list(v) if isinstance(v, tuple) else v, "batch": w.batch, "total_k": pipe.total_k,
@@ -363,10 +375,8 @@ def run_ours(args, world, rank, local):
         w = w.frames()
     red = altr.Reducer(w.seqlens, w.d, w.x.dtype, dev, stride=args.stride, lam=_lam(args), **budget)
     pipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, slots=2, stride=args.stride, lam=_lam(args), **budget)
-    e = 2 if w.x.dtype == torch.bfloat16 else 4
     total_rows = w.total
-    in_bytes = 3 * total_rows * w.d * e
-    alg_bytes = synth.algorithmic_bytes(w.seqlens, red.ks, w.d, e)
+    in_bytes, alg_bytes, d2h_bytes = step_bytes(w, red.ks)
 
     def barrier():
         if world > 1:
@@ -443,13 +453,13 @@ def run_ours(args, world, rank, local):
     # [begin, end] intervals divided by their number
     spans = sorted((start.elapsed_time(ev[0]), start.elapsed_time(ev[1])) for ev in evs)
     union, lo, hi = 0.0, None, None
-    for b, e in spans:
-        if hi is None or b > hi:
+    for t_begin, t_end in spans:
+        if hi is None or t_begin > hi:
             if hi is not None:
                 union += hi - lo
-            lo, hi = b, e
+            lo, hi = t_begin, t_end
         else:
-            hi = max(hi, e)
+            hi = max(hi, t_end)
     union += (hi - lo) if hi is not None else 0.0
     t_score = [union / len(evs)] * len(evs)
     ms_step = max_over_ranks(total_ms / args.steps, world, dev)
@@ -465,16 +475,30 @@ def run_ours(args, world, rank, local):
     y_h = torch.empty(red.total_k, w.d, dtype=w.x.dtype).pin_memory()
     idx_h = torch.empty(red.total_k, dtype=torch.int32).pin_memory()
     epipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, slots=2, stride=args.stride, lam=_lam(args), **budget)
-    for _ in range(3):
-        epipe.submit_host(x_h, p_h, q_h, y_h, idx_h)
-    epipe.synchronize()
     e2e_steps = max(3, min(args.steps, args.e2e_steps))
-    barrier()
-    t0 = time.perf_counter()
-    for _ in range(e2e_steps):
-        epipe.submit_host(x_h, p_h, q_h, y_h, idx_h)
-    epipe.synchronize()
-    e2e_s = max_over_ranks((time.perf_counter() - t0) / e2e_steps, world, dev)
+    if mode == "graph":  # the copies and the steps captured together (Pipeline.graph_host)
+        per_graph = max(s_ for s_ in range(1, min(GRAPH_STEPS, e2e_steps) + 1) if e2e_steps % s_ == 0)
+        egraph = epipe.graph_host(x_h, p_h, q_h, y_h, idx_h, steps=per_graph)
+        for _ in range(3):
+            egraph.replay()
+        torch.cuda.synchronize()
+        barrier()
+        t0 = time.perf_counter()
+        for _ in range(e2e_steps // per_graph):
+            egraph.replay()
+        torch.cuda.synchronize()
+        e2e_s = max_over_ranks((time.perf_counter() - t0) / e2e_steps, world, dev)
+        del egraph
+    else:
+        for _ in range(3):
+            epipe.submit_host(x_h, p_h, q_h, y_h, idx_h)
+        epipe.synchronize()
+        barrier()
+        t0 = time.perf_counter()
+        for _ in range(e2e_steps):
+            epipe.submit_host(x_h, p_h, q_h, y_h, idx_h)
+        epipe.synchronize()
+        e2e_s = max_over_ranks((time.perf_counter() - t0) / e2e_steps, world, dev)
     epipe.close()
     del epipe
 
@@ -505,7 +529,7 @@ def run_ours(args, world, rank, local):
         "latency_us": {"tr_reduce_graph_replay": latency_us},
         "roofline": roofline,
         "e2e": {"value": images / e2e_s, "unit": "images/s", "h2d_bytes_per_step": in_bytes,
-                "d2h_bytes_per_step": red.total_k * (w.d * e + 4)},
+                "d2h_bytes_per_step": d2h_bytes},
         "gpu_launches": 3 * args.steps,
         "clocks": clk,
         "status": st,

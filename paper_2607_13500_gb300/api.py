@@ -454,6 +454,38 @@ class Pipeline:
         self._graphed = True
         return g
 
+    def graph_host(self, x_h, x_pre_h, x_post_h, y_h, idx_h, steps=16) -> "torch.cuda.CUDAGraph":
+        """``steps`` end-to-end steps (``submit_host``: pinned host inputs
+        copied in, reduced, y and idx copied back to the pinned ``y_h`` /
+        ``idx_h``) captured into one CUDA graph, so that a replay needs no
+        host work per step.  The host buffers are the graph's: refill them
+        between replays.  The pipeline is dedicated to replays afterwards."""
+        if self.submitted and self._handle is not None:
+            raise RuntimeError("Pipeline.graph_host needs a pipeline without earlier submissions")
+        # one step outside the capture: device buffers and copy streams, and
+        # the selection kernel's shared-memory limit
+        self.submit_host(x_h, x_pre_h, x_post_h, y_h, idx_h)
+        self.synchronize()
+        self.lib.tr_pipeline_destroy(self._handle)
+        self._handle = None
+        self.submitted = 0
+        h = self._host
+        h["in_free"], h["out_free"] = [None] * self.slots, [None] * self.slots
+        self._bind(*h["bufs"][0])
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            cap = torch.cuda.current_stream(self.device)
+            h["cin"].wait_stream(cap)
+            h["cout"].wait_stream(cap)
+            self.select_stream.wait_stream(cap)
+            for _ in range(steps):
+                self.submit_host(x_h, x_pre_h, x_post_h, y_h, idx_h)
+            self.wait(cap)
+            for st in self.score_streams + [h["cin"], h["cout"], self.select_stream]:
+                cap.wait_stream(st)
+        self._graphed = True
+        return g
+
     def wait(self, stream=None):
         """Makes ``stream`` (default: the current stream) wait for every submission."""
         st = stream if stream is not None else torch.cuda.current_stream(self.device)

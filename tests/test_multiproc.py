@@ -53,3 +53,18 @@ def test_two_gloo_ranks_max_and_aggregate():
 def test_single_rank_is_identity():
     assert bench.max_over_ranks(3.5, 1) == 3.5
     assert bench.job_images_per_s(64, 1, 0.25) == pytest.approx(256000.0)
+
+
+def test_step_bytes():
+    # bench.py's byte accounting for one step: the three inputs an
+    # end-to-end step copies in, the path's algorithmic traffic, and y plus
+    # the int32 indices copied back
+    w = synth.make("llava576", seed=0, batch=3, n=40, d=64)
+    ks = [8, 8, 8]
+    in_b, alg_b, d2h_b = bench.step_bytes(w, ks)
+    assert in_b == 3 * 120 * 64 * 2
+    assert alg_b == in_b + 2 * 24 * 64 * 2 + 4 * 24
+    assert d2h_b == 24 * (64 * 2 + 4)
+    w = synth.make("single_clip336", seed=0, n=40)  # fp32
+    in_b, alg_b, d2h_b = bench.step_bytes(w, [5])
+    assert (in_b, d2h_b) == (3 * 40 * 1024 * 4, 5 * (1024 * 4 + 4))

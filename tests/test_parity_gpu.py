@@ -313,6 +313,39 @@ def test_pipeline_from_host():
         pipe.close()
 
 
+def test_pipeline_graph_from_host():
+    # The end-to-end steps (copy in, reduce, copy out) captured into one graph
+    # and replayed: the pinned outputs hold the reduction of whatever the
+    # pinned inputs held when the graph ran.
+    altr = _alt()
+    ws = [synth.make("single_clip336", seed=60 + s, batch=2) for s in range(2)]
+    budget = _budget(ws[0], k=64)
+    pipe = altr.Pipeline(ws[0].seqlens, ws[0].d, ws[0].x.dtype, "cuda", budget=budget)
+    try:
+        x_h, p_h, q_h = (t.clone().pin_memory() for t in (ws[0].x, ws[0].x_pre, ws[0].x_post))
+        y_h = torch.zeros(budget[2][-1], ws[0].d, dtype=ws[0].x.dtype).pin_memory()
+        idx_h = torch.zeros(budget[2][-1], dtype=torch.int32).pin_memory()
+        g = pipe.graph_host(x_h, p_h, q_h, y_h, idx_h, steps=3)
+        for w in ws:
+            x_h.copy_(w.x)
+            p_h.copy_(w.x_pre)
+            q_h.copy_(w.x_post)
+            y_h.zero_()
+            idx_h.fill_(-1)
+            g.replay()
+            torch.cuda.synchronize()
+            ks, k1s, cu = budget
+            for b in range(w.batch):
+                xb, pb, qb = (_f64(t[b * 576:(b + 1) * 576]) for t in (w.x, w.x_pre, w.x_post))
+                ref = oracle.select_image(xb, pb, qb, ks[b], k1s[b])
+                assert np.array_equal(idx_h[cu[b]:cu[b + 1]].numpy(), ref["kept"]), b
+                rows = w.x[b * 576:(b + 1) * 576][torch.from_numpy(ref["kept"].astype(np.int64))]
+                assert torch.equal(_bits(y_h[cu[b]:cu[b + 1]]), _bits(rows)), b
+        del g
+    finally:
+        pipe.close()
+
+
 def test_pipeline_edge_cases():
     # one slot and three slots, an empty image and K = 0 images in a ragged
     # batch, fp32 inputs, and a batch that keeps nothing at all
