@@ -265,6 +265,9 @@ tr_status tr_reduce_noalloc(const tr_tokens *in, const int32_t *d_k, const int32
  *     time it (as event-record nodes when the stream is being captured).
  *     Host-detectable errors are returned before anything is enqueued.
  *   tr_pipeline_wait: makes `stream` wait for every submission so far.
+ *   tr_pipeline_kernels: kernels launched by the submissions so far (three
+ *     per submission -- score, select, gather -- or two when a tiny uniform
+ *     batch is selected and gathered in one launch); 0 for NULL.
  *
  * Graph capture: submissions made while the streams are captured into a
  * CUDA graph (forked from the capturing stream, joined back with
@@ -282,6 +285,7 @@ tr_status tr_pipeline_submit(tr_pipeline *p, const tr_tokens *in, const int32_t 
                              const int32_t *d_cu_k, int32_t total_k, void *y, int32_t *idx, float *h2, float *s,
                              int32_t *d_status, void *score_begin, void *score_end);
 tr_status tr_pipeline_wait(tr_pipeline *p, void *stream);
+long long tr_pipeline_kernels(const tr_pipeline *p);
 tr_status tr_pipeline_destroy(tr_pipeline *p);
 
 #ifdef __cplusplus

@@ -72,6 +72,7 @@ def load() -> ctypes.CDLL:
     lib.tr_pipeline_submit.argtypes = [VP, tok, VP, VP, VP, I32, VP, VP, VP, VP, VP, VP, VP]
     lib.tr_pipeline_submit.restype = I32
     lib.tr_pipeline_wait.argtypes, lib.tr_pipeline_wait.restype = [VP, VP], I32
+    lib.tr_pipeline_kernels.argtypes, lib.tr_pipeline_kernels.restype = [VP], ctypes.c_longlong
     lib.tr_pipeline_destroy.argtypes, lib.tr_pipeline_destroy.restype = [VP], I32
     lib.tr_reduce.argtypes = [tok, VP, VP, VP, I32, VP, VP, VP, VP, VP, SZ, VP, VP]
     lib.tr_reduce.restype = I32

@@ -486,6 +486,13 @@ class Pipeline:
         self._graphed = True
         return g
 
+    @property
+    def kernels(self) -> int:
+        """Kernels launched by the submissions of the current handle
+        (tr_pipeline_kernels; after ``graph``/``graph_host``: those the
+        captured graph launches per replay)."""
+        return int(self.lib.tr_pipeline_kernels(self._handle)) if self._handle is not None else 0
+
     def wait(self, stream=None):
         """Makes ``stream`` (default: the current stream) wait for every submission."""
         st = stream if stream is not None else torch.cuda.current_stream(self.device)

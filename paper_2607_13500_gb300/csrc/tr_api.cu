@@ -222,6 +222,7 @@ struct tr_pipeline {
   cudaEvent_t done[TR_PIPELINE_MAX_SLOTS] = {};
   cudaEvent_t head[TR_PIPELINE_MAX_SLOTS] = {};  // the slot's batch scored
   long long submitted = 0;
+  long long kernels = 0;  // kernels launched by the submissions
 };
 
 tr_status tr_pipeline_create(void *const *score_streams, void *select_stream, int32_t slots, void *const *ws,
@@ -314,11 +315,13 @@ tr_status tr_pipeline_submit(tr_pipeline *p, const tr_tokens *in, const int32_t 
   if (!in->cu_seqlens && in->batch > 0 && in->n <= 1024 && in->batch * replicas <= cap) {
     SelectArgs a = select_args(in, sh, stats, d_k, d_k1, d_cu_k, idx, nullptr, h2, s, ws, d_status);
     if (launch_select_gather(a, y, b, false) != cudaSuccess) return TR_ERR_CUDA;
+    p->kernels += (sh.total > 0) + 1;
   } else {
     if ((rc = select_capped(in, stats, d_k, d_k1, d_cu_k, idx, nullptr, h2, s, ws, p->ws_bytes, d_status, b, cap,
                             false)) != TR_OK)
       return rc;
     if ((rc = gather_impl(in, d_cu_k, idx, total_k, y, b, false)) != TR_OK) return rc;
+    p->kernels += (sh.total > 0) + (in->batch > 0) + (total_k > 0);
   }
   if (cudaEventRecord(p->done[slot], b) != cudaSuccess) return TR_ERR_CUDA;
   ++p->submitted;
@@ -332,6 +335,8 @@ tr_status tr_pipeline_wait(tr_pipeline *p, void *stream) {
     if (cudaStreamWaitEvent(static_cast<cudaStream_t>(stream), p->done[i], 0) != cudaSuccess) return TR_ERR_CUDA;
   return TR_OK;
 }
+
+long long tr_pipeline_kernels(const tr_pipeline *p) { return p ? p->kernels : 0; }
 
 tr_status tr_pipeline_destroy(tr_pipeline *p) {
   if (!p) return TR_OK;

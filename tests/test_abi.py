@@ -115,6 +115,7 @@ def test_pipeline_host_argument_checks(lib):
                                   v(0x50000), None, None, None, None, None) == 1
     assert lib.tr_pipeline_wait(None, None) == 1
     assert lib.tr_pipeline_destroy(None) == 0
+    assert lib.tr_pipeline_kernels(None) == 0
 
 
 def test_missing_library_raises(monkeypatch, tmp_path):

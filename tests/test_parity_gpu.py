@@ -255,6 +255,7 @@ def test_pipeline_graph_replay(batch):
     try:
         evs = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(5)]
         g = pipe.graph(dx, dp, dq, steps=5, score_events=evs)
+        assert pipe.kernels == 5 * (2 if batch == 2 else 3)  # fused select + gather for two small images
         for o in pipe.outs:
             o["y"].zero_()
             o["idx"].fill_(-1)
