@@ -418,17 +418,20 @@ class Pipeline:
         h["out_free"][slot] = out
         return r
 
-    def graph(self, x, x_pre, x_post, steps=16, score_events=None) -> "torch.cuda.CUDAGraph":
+    def graph(self, x, x_pre, x_post, steps=16, score_events=None, inputs=None) -> "torch.cuda.CUDAGraph":
         """``steps`` pipelined submissions of these input tensors captured into
         one CUDA graph: ``replay()`` runs them (each step's selection and
         gather overlapping the next step's scoring) with a single launch, for
         batches so small that submitting step by step from the host would
-        take longer than the GPU work.  ``score_events`` (``steps`` pairs of
-        timing torch.cuda.Event, or None) become event nodes around each score
-        kernel.  Step i writes output set i mod ``slots``.  The pipeline is
-        dedicated to replays afterwards (``submit`` raises)."""
+        take longer than the GPU work.  ``inputs`` (a list of (x, x_pre,
+        x_post) of this shape, or None) gives step i the tensors
+        inputs[i mod len(inputs)] instead.  ``score_events`` (``steps`` pairs
+        of timing torch.cuda.Event, or None) become event nodes around each
+        score kernel.  Step i writes output set i mod ``slots``.  The pipeline
+        is dedicated to replays afterwards (``submit`` raises)."""
         if self.submitted and self._handle is not None:
             raise RuntimeError("Pipeline.graph needs a pipeline without earlier submissions")
+        inputs = [(x, x_pre, x_post)] if inputs is None else list(inputs)
         cur = torch.cuda.current_stream(self.device)
         # one step outside the capture: the selection kernel's shared-memory
         # limit is raised once per device, on its first launch
@@ -447,7 +450,7 @@ class Pipeline:
         with torch.cuda.graph(g):
             cap = torch.cuda.current_stream(self.device)
             for i in range(steps):
-                self.submit(x, x_pre, x_post, score_events=None if score_events is None else score_events[i])
+                self.submit(*inputs[i % len(inputs)], score_events=None if score_events is None else score_events[i])
             self.wait(cap)
             for st in self.score_streams:
                 cap.wait_stream(st)

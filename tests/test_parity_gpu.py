@@ -272,6 +272,22 @@ def test_pipeline_graph_replay(batch):
         del g
     finally:
         pipe.close()
+    # steps over rotating inputs: with two slots and two input sets, slot j
+    # always holds the reduction of input set j
+    w2 = synth.make("single_clip336", seed=6, batch=batch)
+    pipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, budget=budget, scores=True, slots=2)
+    try:
+        sets = [(dx, dp, dq), tuple(t.to(dev) for t in (w2.x, w2.x_pre, w2.x_post))]
+        g = pipe.graph(*sets[0], steps=4, inputs=sets)
+        g.replay()
+        torch.cuda.synchronize()
+        for o, src in zip(pipe.outs, (w, w2)):
+            r = altr.ReduceResult(o["y"][:pipe.total_k], o["idx"][:pipe.total_k], pipe.cu_k, o["h2"], o["s"],
+                                  o["status"])
+            compare_result(r, src.x, src.x_pre, src.x_post, src.seqlens, budget)
+        del g
+    finally:
+        pipe.close()
     # the same timing events on host submissions
     pipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, budget=budget, scores=True, slots=2)
     try:
