@@ -393,9 +393,13 @@ def run_ours(args, world, rank, local):
         if world > 1:
             torch.distributed.barrier()
 
-    # each kernel alone (one stream, back to back), outside the timed region
+    # each kernel alone (one stream, back to back), outside the timed region;
+    # a short device-side delay queued first lets the host's launches get
+    # ahead, so the events time the kernels and not the host
     alone_evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(max(3, args.warmup))]
     for ev in alone_evs:
+        if hasattr(torch.cuda, "_sleep"):
+            torch.cuda._sleep(200000)
         red.run_separate(w.x, w.x_pre, w.x_post, ev)
     torch.cuda.synchronize()
     alone = {name: statistics.median(ev[j].elapsed_time(ev[j + 1]) for ev in alone_evs[1:])
