@@ -431,6 +431,30 @@ def test_edge_budgets_and_sizes():
     check_reduce(x, xp, xq, [333, 1, 666], ([100, 1, 66], [33, 0, 22], [0, 100, 101, 167]))
 
 
+def test_many_tiny_images():
+    # 3000 images of 1-9 tokens (ragged) and 2000 of 7 (uniform): the
+    # selection grid loops over images (the pipeline caps it at a quarter of
+    # the SMs) and most images keep everything or nothing but one token.
+    altr = _alt()
+    dev = torch.device("cuda")
+    g = torch.Generator().manual_seed(77)
+    seqlens = torch.randint(1, 10, (3000,), generator=g).tolist()
+    t = sum(seqlens)
+    x, xp, xq = _rows(t, 64, 78)
+    budget = altr.budgets(seqlens, k=None, ratio=(1, 3))
+    sample = list(range(0, 3000, 97))
+    check_reduce(x, xp, xq, seqlens, budget, images=sample)
+    pipe = altr.Pipeline(seqlens, 64, torch.bfloat16, dev, budget=budget, scores=True)
+    try:
+        r = pipe.submit(x.to(dev), xp.to(dev), xq.to(dev))
+        pipe.synchronize()
+        compare_result(r, x, xp, xq, seqlens, budget, images=sample)
+    finally:
+        pipe.close()
+    x, xp, xq = _rows(2000 * 7, 64, 79)
+    check_reduce(x, xp, xq, [7] * 2000, altr.budgets([7] * 2000, k=3), images=list(range(0, 2000, 61)))
+
+
 def test_exact_ties_and_degenerate_rows():
     d, n = 512, 96
     g = torch.Generator().manual_seed(3)
