@@ -235,7 +235,9 @@ tr_status tr_reduce_noalloc(const tr_tokens *in, const int32_t *d_k, const int32
  * Overlapped reduction of successive batches, a stream pipeline over `slots`
  * slots.  Submission i uses slot i mod slots: it scores its batch on
  * score_streams[slot] (tr_score), then selects (tr_select) and gathers
- * (tr_gather) it on `select_stream`, which waits for that scoring only.  So
+ * (tr_gather) it on `select_stream`, which waits for that scoring only (a
+ * uniform batch of one or two images of at most 1024 tokens is selected and
+ * gathered by one tr_select_gather launch instead).  So
  * the selection and gather of one batch run while the next batch is scored,
  * and with a score stream per slot one batch's scoring starts while the
  * previous score kernel drains.  Give `select_stream` the higher priority:
