@@ -115,6 +115,12 @@ def job_images_per_s(images_per_rank: int, world: int, ms_step_max: float) -> fl
     return images_per_rank * world / (ms_step_max * 1e-3)
 
 
+def steps_per_graph(steps):
+    """The largest divisor of `steps` up to GRAPH_STEPS: replays of a graph of
+    that many steps time exactly `steps` steps."""
+    return max(d for d in range(1, min(GRAPH_STEPS, steps) + 1) if steps % d == 0)
+
+
 def step_bytes(w, ks):
     """Bytes of one step over workload w with budgets ks: the three input
     tensors (what an end-to-end step copies in), the path's algorithmic
@@ -430,7 +436,7 @@ def run_ours(args, world, rank, local):
     cur = torch.cuda.current_stream(dev)
     clocks = ClockSampler(dev)
     if mode == "graph":
-        per_graph = max(s_ for s_ in range(1, min(GRAPH_STEPS, args.steps) + 1) if args.steps % s_ == 0)
+        per_graph = steps_per_graph(args.steps)
         reps = args.steps // per_graph
         # one graph per window of per_graph input copies, replayed in turn
         n_graphs = min(reps, -(-rot // per_graph))
@@ -515,7 +521,7 @@ def run_ours(args, world, rank, local):
     epipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, dev, slots=2, stride=args.stride, lam=_lam(args), **budget)
     e2e_steps = max(3, min(args.steps, args.e2e_steps))
     if mode == "graph":  # the copies and the steps captured together (Pipeline.graph_host)
-        per_graph = max(s_ for s_ in range(1, min(GRAPH_STEPS, e2e_steps) + 1) if e2e_steps % s_ == 0)
+        per_graph = steps_per_graph(e2e_steps)
         egraph = epipe.graph_host(x_h, p_h, q_h, y_h, idx_h, steps=per_graph)
         for _ in range(3):
             egraph.replay()

@@ -68,3 +68,17 @@ def test_step_bytes():
     w = synth.make("single_clip336", seed=0, n=40)  # fp32
     in_b, alg_b, d2h_b = bench.step_bytes(w, [5])
     assert (in_b, d2h_b) == (3 * 40 * 1024 * 4, 5 * (1024 * 4 + 4))
+
+
+def test_bench_sweep_and_graph_steps():
+    assert bench._sweep_points("k=64,128,192") == ("k", [64, 128, 192])
+    assert bench._sweep_points("lam=0/1,1/3") == ("lam", [(0, 1), (1, 3)])
+    assert bench._sweep_points("ratio=1/9,2/9") == ("ratio", [(1, 9), (2, 9)])
+    assert bench._sweep_points("batch=1,8,64") == ("batch", [1, 8, 64])
+    with pytest.raises(SystemExit):
+        bench._sweep_points("d=64")
+    # replays of a graph of S steps time exactly K steps
+    for k in (1, 3, 7, 16, 17, 20, 300, 2000, 4000):
+        s = bench.steps_per_graph(k)
+        assert 1 <= s <= bench.GRAPH_STEPS and k % s == 0
+    assert bench.steps_per_graph(2000) == 16 and bench.steps_per_graph(300) == 15 and bench.steps_per_graph(17) == 1
