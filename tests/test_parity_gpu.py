@@ -564,6 +564,26 @@ def test_nonfinite_huge_and_tiny_rows():
         check_reduce(x, xp, xq, [n], ([k], [k1], [0, k]), expect_nonfinite=True)
 
 
+def test_exact_sums_past_the_window():
+    # Every row is a channel permutation of one fp32 vector that also holds
+    # 2^-60 and 2^-75 entries: R and s tie exactly across rows, so every
+    # decision goes to the exact sums, and the tiny squares fall below the
+    # 128-bit window anchored at the row's sum: the digit accumulator takes
+    # over (the fp32 sums themselves stay inside the error model).
+    n, d = 64, 256
+    g = torch.Generator().manual_seed(9)
+    base = torch.randn(d, generator=g)
+    base[:6] = torch.tensor([2.0 ** -60, -(2.0 ** -60), 2.0 ** -75, 3 * 2.0 ** -75, 2.0 ** -62, -(2.0 ** -70)])
+    other = torch.randn(d, generator=g)
+    other[:3] = torch.tensor([2.0 ** -64, 2.0 ** -71, -(2.0 ** -66)])
+    perms = [torch.randperm(d, generator=g) for _ in range(n)]
+    x = torch.stack([base[p] for p in perms])
+    xp = torch.stack([base[p] for p in perms])
+    xq = torch.stack([other[p] for p in perms])
+    for k, k1 in [(20, 7), (40, 0), (30, 30)]:
+        check_reduce(x, xp, xq, [n], ([k], [k1], [0, k]))
+
+
 def test_fp32_wide_range():
     n, d = 300, 1024
     g = torch.Generator().manual_seed(5)
