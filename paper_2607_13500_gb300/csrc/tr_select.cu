@@ -32,12 +32,10 @@ __device__ __forceinline__ uint4 ld_nc16(const uint4 *p) {
   return r;
 }
 
-__global__ void __launch_bounds__(kSelectThreads, 1)
-    k_select_gather(const SelectArgs a, const int replicas, const int nchunks, uint4 *__restrict__ y) {
-  extern __shared__ __align__(16) unsigned char smem[];
-  pdl_wait();  // the statistics come from the kernel before this one
-  const int b = blockIdx.x / replicas, r = blockIdx.x % replicas;
-  select_image(a, b, smem, r == 0);
+// Replica r of `replicas` copies its share of image b's kept rows, whose
+// local indices select_image left in this CTA's shared memory.
+__device__ __forceinline__ void copy_kept(const SelectArgs &a, const int b, const int r, const int replicas,
+                                          const int nchunks, uint4 *__restrict__ y, unsigned char *smem) {
   long long off;
   int n;
   if (a.cu_seqlens) {
@@ -73,6 +71,15 @@ __global__ void __launch_bounds__(kSelectThreads, 1)
       }
     }
   }
+}
+
+__global__ void __launch_bounds__(kSelectThreads, 1)
+    k_select_gather(const SelectArgs a, const int replicas, const int nchunks, uint4 *__restrict__ y) {
+  extern __shared__ __align__(16) unsigned char smem[];
+  pdl_wait();  // the statistics come from the kernel before this one
+  const int b = blockIdx.x / replicas, r = blockIdx.x % replicas;
+  select_image(a, b, smem, r == 0);
+  copy_kept(a, b, r, replicas, nchunks, y, smem);
 }
 
 // Per device (index & 63): dynamic shared memory limit already raised (bit 0
@@ -135,9 +142,9 @@ cudaError_t launch_select_gather(const SelectArgs &a, void *y, cudaStream_t st, 
   }
   const int sms = sm_count();
   if (sms <= 0) return cudaErrorInvalidDevice;
-  const int replicas = max(1, min(16, sms / a.batch));
   const size_t smem = select_smem_bytes(a.max_n);
   const int nchunks = a.d * elem_bytes(a.dtype) / 16;
+  const int replicas = max(1, min(16, sms / a.batch));
   return launch_kernel(k_select_gather, dim3(a.batch * replicas), dim3(kSelectThreads), smem, st, pdl, a, replicas,
                        nchunks, static_cast<uint4 *>(y));
 }

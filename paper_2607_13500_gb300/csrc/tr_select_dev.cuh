@@ -1322,9 +1322,24 @@ __device__ __forceinline__ bool is_pick(int q, int m, int k2, int t, bool interv
 // the K kept local indices, ascending, in the second order buffer of smem
 // (kept_rows); only a primary CTA writes idx, role, H2/s and the status words
 // (replicas that run the same deterministic selection write nothing).
-__device__ void select_image(const SelectArgs &a, const int b, unsigned char *smem, const bool primary = true) {
-  __shared__ int sh_lo, sh_hi;
-  const int tid = threadIdx.x, nthr = blockDim.x;
+// The state of one image's selection in a CTA: where its rows are, its
+// budgets and the CTA's shared-memory arrays (layout in select_smem_bytes).
+struct ImageCtx {
+  long long off;
+  int n, k, k1, k2, ko;
+  bool need_r, need_s, primary;
+  uint32_t *key, *hist;
+  uint16_t *ia, *ib, *bid;
+  uint8_t *fl;
+  const float *st;
+  ExactRec *rec;
+};
+
+// Sets up c for image b; false when there is nothing to select (an invalid
+// budget, counted in status[3] by the primary CTA, or an empty image).
+__device__ __forceinline__ bool image_ctx(const SelectArgs &a, const int b, unsigned char *smem, const bool primary,
+                                          ImageCtx &c) {
+  const int tid = threadIdx.x;
   long long off;
   int n;
   if (a.cu_seqlens) {
@@ -1334,27 +1349,50 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
     off = (long long)b * a.n_uniform;
     n = a.n_uniform;
   }
-  const int k = a.k[b], k1 = a.k1[b], k2 = k - k1, ko = a.cu_k[b];
+  const int k = a.k[b], k1 = a.k1[b];
   if (n < 0 || n > a.max_n || k < 0 || k > n || k1 < 0 || k1 > k) {
     if (tid == 0 && a.status && primary) atomicAdd(&a.status[3], 1);
-    return;
+    return false;
   }
-  if (n == 0) return;
+  if (n == 0) return false;
   const int cap = row_capacity(a.max_n);
-  uint32_t *key = reinterpret_cast<uint32_t *>(smem);        // [cap] sort key per row
-  uint16_t *ia = reinterpret_cast<uint16_t *>(key + cap);    // [cap] order buffers
-  uint16_t *ib = ia + cap;                                   // [cap]
-  uint32_t *hist = reinterpret_cast<uint32_t *>(ib + cap);   // [kWarps x 256]
-  uint16_t *bid = reinterpret_cast<uint16_t *>(hist + kWarps * 256);  // [cap] sort scratch
-  uint8_t *fl = reinterpret_cast<uint8_t *>(bid + cap);             // [cap] row flags
-  const float *st = a.stats + off * TR_STATS_WORDS;
-  ExactRec *rec = a.exact + off;
-  const bool need_r = k1 > 0 && k1 < n;  // the importance order decides something
-  const bool need_s = k2 > 0;
+  c.off = off;
+  c.n = n;
+  c.k = k;
+  c.k1 = k1;
+  c.k2 = k - k1;
+  c.ko = a.cu_k[b];
+  c.need_r = k1 > 0 && k1 < n;  // the importance order decides something
+  c.need_s = k - k1 > 0;
+  c.primary = primary;
+  c.key = reinterpret_cast<uint32_t *>(smem);                          // [cap] sort key per row
+  c.ia = reinterpret_cast<uint16_t *>(c.key + cap);                    // [cap] order buffers
+  c.ib = c.ia + cap;                                                   // [cap]
+  c.hist = reinterpret_cast<uint32_t *>(c.ib + cap);                   // [kWarps x 256]
+  c.bid = reinterpret_cast<uint16_t *>(c.hist + kWarps * 256);         // [cap] sort scratch
+  c.fl = reinterpret_cast<uint8_t *>(c.bid + cap);                     // [cap] row flags
+  c.st = a.stats + off * TR_STATS_WORDS;
+  c.rec = a.exact + off;
+  return true;
+}
 
-  // 1. Rows whose fp32 sums left the error model are settled exactly first
-  //    (also when only their H2 / s outputs need it).  The same pass lays
-  //    out the importance keys ~ord32(R32) and the identity order.
+// 1. Rows whose fp32 sums left the error model are settled exactly first
+//    (also when only their H2 / s outputs need it): the importance side
+//    (want_l) and / or the consistency side (want_s).  The same pass lays
+//    out the importance keys ~ord32(R32) and the identity order.
+__device__ __forceinline__ void settle_unreliable(const SelectArgs &a, ImageCtx &c, const bool want_l,
+                                                  const bool want_s) {
+  const int tid = threadIdx.x;
+  const int nthr = blockDim.x;
+  const int n = c.n;
+  const long long off = c.off;
+  uint32_t *key = c.key;
+  uint16_t *ia = c.ia;
+  uint8_t *fl = c.fl;
+  const float *st = c.st;
+  ExactRec *rec = c.rec;
+  const bool primary = c.primary;
+  const bool need_r = c.need_r, need_s = c.need_s;
   for (int i0 = tid; i0 < n; i0 += kKeyIlp * nthr) {
     float2 kk[kKeyIlp];
 #pragma unroll
@@ -1367,8 +1405,8 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
       const int i = i0 + u * nthr;
       if (i < n) {
         uint8_t f = 0;
-        if ((need_r || a.h2) && isnan(kk[u].x)) f |= F_NEEDL;
-        if ((need_s || a.s) && isnan(kk[u].y)) f |= F_NEEDS;
+        if (want_l && (need_r || a.h2) && isnan(kk[u].x)) f |= F_NEEDL;
+        if (want_s && (need_s || a.s) && isnan(kk[u].y)) f |= F_NEEDS;
         fl[i] = f;
         key[i] = ~ord32(kk[u].x);
         ia[i] = (uint16_t)i;
@@ -1379,7 +1417,26 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
   refine_pending(a, off, n, fl, rec, primary);
   __syncthreads();
 
-  // 2. Stage I: top-K1 by R (equivalently H2), descending, lower index first.
+}
+
+// 2. Stage I: top-K1 by R (equivalently H2), descending, lower index first.
+//    Marks X_imp (F_IMP) in the flags.
+__device__ __forceinline__ void stage_one(const SelectArgs &a, ImageCtx &c) {
+  __shared__ int sh_lo, sh_hi;
+  const int tid = threadIdx.x;
+  const int nthr = blockDim.x;
+  const int n = c.n;
+  const long long off = c.off;
+  uint32_t *key = c.key;
+  uint32_t *hist = c.hist;
+  uint16_t *ia = c.ia;
+  uint16_t *ib = c.ib;
+  uint16_t *bid = c.bid;
+  uint8_t *fl = c.fl;
+  ExactRec *rec = c.rec;
+  const bool primary = c.primary;
+  const int k1 = c.k1;
+  const bool need_r = c.need_r;
   if (need_r) {
     for (int i = tid; i < n; i += nthr)  // rows settled exactly carry their exact key
       if (fl[i] & F_XL) key[i] = ~ord32(exact_r_key(rec[i]));
@@ -1500,81 +1557,121 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
     __syncthreads();
   }
 
-  // 3. Stage II: sort X_rem by s ascending, pick positions 0, t, 2t, ...
-  if (need_s) {
-    // consistency keys ord32(s32) of every row (stage I's keys are no longer
-    // needed; X_imp rows' keys are never read), exact ones for settled rows
-    for (int i0 = tid; i0 < n; i0 += kKeyIlp * nthr) {
-      float sv[kKeyIlp];
-#pragma unroll
-      for (int u = 0; u < kKeyIlp; ++u) {
-        const int i = i0 + u * nthr;
-        sv[u] = i < n ? key_s(st + (long long)i * TR_STATS_WORDS) : 0.f;
-      }
-#pragma unroll
-      for (int u = 0; u < kKeyIlp; ++u) {
-        const int i = i0 + u * nthr;
-        if (i < n) key[i] = ord32((fl[i] & F_XS) ? exact_s_key(rec[i]) : sv[u]);
-      }
-    }
-    // X_rem in ascending index order (the stable sort's tie order)
-    const int per = (n + nthr - 1) / nthr;
-    const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
-    int cnt = 0;
-    for (int i = i0; i < i1; ++i) cnt += !(fl[i] & F_IMP);
-    int m = 0;
-    int pos = block_exclusive_scan(cnt, &m);
-    for (int i = i0; i < i1; ++i)
-      if (!(fl[i] & F_IMP)) ia[pos++] = (uint16_t)i;
-    __syncthreads();
-    const uint16_t *ord = sort_rows(key, ia, ib, bid, m, hist, false);
-    const int t = max(1, m / k2);
-    for (int j = tid; j < k2; j += nthr) {
-      const int p = pick_position(j, m, k2, t, a.stride_interval);
-      const bool c0 = p == 0 || cert_s(key, ord, p, a.bounds);
-      const bool c1 = p + 1 >= m || cert_s(key, ord, p + 1, a.bounds);
-      if (c0 && c1) {
-        fl[ord[p]] |= F_DIV;
-      } else {
-        int lo = p;
-        while (lo > 0 && !cert_s(key, ord, lo, a.bounds)) --lo;
-        int hi = p + 1;
-        while (hi < m && !cert_s(key, ord, hi, a.bounds)) ++hi;
-        // Threads whose runs coincide write the same bits: the races are benign.
-        for (int q = lo; q < hi; ++q) {
-          const int r = ord[q];
-          fl[r] |= (uint8_t)(F_RUN | ((fl[r] & F_XS) ? 0 : F_NEEDS));
-        }
-      }
-    }
-    __syncthreads();
-    refine_pending(a, off, n, fl, rec, primary);
-    __syncthreads();
-    for (int q = tid; q < m; q += nthr) {
-      const int r = ord[q];
-      if (!(fl[r] & F_RUN)) continue;
-      int lo = q;
-      while (lo > 0 && !cert_s(key, ord, lo, a.bounds)) --lo;
-      int hi = q + 1;
-      while (hi < m && !cert_s(key, ord, hi, a.bounds)) ++hi;
-      const bool ovf = rec[r].flags_s & kRecOverflowS;
-      int rank = 0;
-      for (int q2 = lo; q2 < hi; ++q2) {
-        if (q2 == q) continue;
-        const int r2 = ord[q2];
-        int c;
-        if (ovf || (rec[r2].flags_s & kRecOverflowS))
-          c = q2 < q ? -1 : 1;
-        else
-          c = cmp_s(rec[r2], rec[r]);
-        if (c < 0 || (c == 0 && r2 < r)) ++rank;
-      }
-      if (is_pick(lo + rank, m, k2, t, a.stride_interval)) fl[r] |= F_DIV;
-    }
-    __syncthreads();
-  }
+}
 
-  // 4. X* = X_imp union X_div in ascending token order (Eq. 7), plus outputs.
+// 3a. Consistency keys ord32(s32) of every row (stage I's keys are no
+//     longer needed; X_imp rows' keys are never read), exact ones for
+//     settled rows.
+__device__ __forceinline__ void consistency_keys(const SelectArgs &a, ImageCtx &c) {
+  const int tid = threadIdx.x;
+  const int nthr = blockDim.x;
+  const int n = c.n;
+  uint32_t *key = c.key;
+  uint8_t *fl = c.fl;
+  const float *st = c.st;
+  ExactRec *rec = c.rec;
+    for (int i0 = tid; i0 < n; i0 += kKeyIlp * nthr) {
+    float sv[kKeyIlp];
+#pragma unroll
+    for (int u = 0; u < kKeyIlp; ++u) {
+      const int i = i0 + u * nthr;
+      sv[u] = i < n ? key_s(st + (long long)i * TR_STATS_WORDS) : 0.f;
+    }
+#pragma unroll
+    for (int u = 0; u < kKeyIlp; ++u) {
+      const int i = i0 + u * nthr;
+      if (i < n) key[i] = ord32((fl[i] & F_XS) ? exact_s_key(rec[i]) : sv[u]);
+    }
+  }
+}
+
+// The rows of the image (all, or those outside X_imp) in ascending index
+// order -- the stable sort's tie order -- into dst; returns their number.
+__device__ __forceinline__ int list_rows(ImageCtx &c, uint16_t *dst, const bool skip_imp) {
+  const int tid = threadIdx.x, nthr = blockDim.x, n = c.n;
+  const uint8_t *fl = c.fl;
+  const int per = (n + nthr - 1) / nthr;
+  const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
+  int cnt = 0;
+  for (int i = i0; i < i1; ++i) cnt += !(skip_imp && (fl[i] & F_IMP));
+  int m = 0;
+  int pos = block_exclusive_scan(cnt, &m);
+  for (int i = i0; i < i1; ++i)
+    if (!(skip_imp && (fl[i] & F_IMP))) dst[pos++] = (uint16_t)i;
+  __syncthreads();
+  return m;
+}
+
+// 3b. Stage II along ord, X_rem sorted by s (m rows): the stride picks
+//     (F_DIV), with uncertain neighbourhoods settled exactly.
+__device__ __forceinline__ void stage_two_picks(const SelectArgs &a, ImageCtx &c, const uint16_t *ord, const int m) {
+  const int tid = threadIdx.x;
+  const int nthr = blockDim.x;
+  const int n = c.n;
+  const long long off = c.off;
+  uint32_t *key = c.key;
+  uint8_t *fl = c.fl;
+  ExactRec *rec = c.rec;
+  const bool primary = c.primary;
+  const int k2 = c.k2;
+  const int t = max(1, m / k2);
+  for (int j = tid; j < k2; j += nthr) {
+    const int p = pick_position(j, m, k2, t, a.stride_interval);
+    const bool c0 = p == 0 || cert_s(key, ord, p, a.bounds);
+    const bool c1 = p + 1 >= m || cert_s(key, ord, p + 1, a.bounds);
+    if (c0 && c1) {
+      fl[ord[p]] |= F_DIV;
+    } else {
+      int lo = p;
+      while (lo > 0 && !cert_s(key, ord, lo, a.bounds)) --lo;
+      int hi = p + 1;
+      while (hi < m && !cert_s(key, ord, hi, a.bounds)) ++hi;
+      // Threads whose runs coincide write the same bits: the races are benign.
+      for (int q = lo; q < hi; ++q) {
+        const int r = ord[q];
+        fl[r] |= (uint8_t)(F_RUN | ((fl[r] & F_XS) ? 0 : F_NEEDS));
+      }
+    }
+  }
+  __syncthreads();
+  refine_pending(a, off, n, fl, rec, primary);
+  __syncthreads();
+  for (int q = tid; q < m; q += nthr) {
+    const int r = ord[q];
+    if (!(fl[r] & F_RUN)) continue;
+    int lo = q;
+    while (lo > 0 && !cert_s(key, ord, lo, a.bounds)) --lo;
+    int hi = q + 1;
+    while (hi < m && !cert_s(key, ord, hi, a.bounds)) ++hi;
+    const bool ovf = rec[r].flags_s & kRecOverflowS;
+    int rank = 0;
+    for (int q2 = lo; q2 < hi; ++q2) {
+      if (q2 == q) continue;
+      const int r2 = ord[q2];
+      int c;
+      if (ovf || (rec[r2].flags_s & kRecOverflowS))
+        c = q2 < q ? -1 : 1;
+      else
+        c = cmp_s(rec[r2], rec[r]);
+      if (c < 0 || (c == 0 && r2 < r)) ++rank;
+    }
+    if (is_pick(lo + rank, m, k2, t, a.stride_interval)) fl[r] |= F_DIV;
+  }
+  __syncthreads();
+}
+
+// 4. X* = X_imp union X_div in ascending token order (Eq. 7), plus outputs;
+//    the kept local indices are also left in ia (kept_rows).
+__device__ __forceinline__ void emit_outputs(const SelectArgs &a, ImageCtx &c) {
+  const int tid = threadIdx.x;
+  const int nthr = blockDim.x;
+  const int n = c.n;
+  const long long off = c.off;
+  uint16_t *ia = c.ia;
+  uint8_t *fl = c.fl;
+  ExactRec *rec = c.rec;
+  const bool primary = c.primary;
+  const int k = c.k, ko = c.ko;
   const int per = (n + nthr - 1) / nthr;
   const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
   int cnt = 0;
@@ -1612,6 +1709,21 @@ __device__ void select_image(const SelectArgs &a, const int b, unsigned char *sm
   }
   if (tid == 0 && kept_total != k && a.status && primary) atomicAdd(&a.status[3], 1);
   __syncthreads();
+}
+
+// The selection of image b by one CTA (Algorithm 1 with exact decisions).
+__device__ void select_image(const SelectArgs &a, const int b, unsigned char *smem, const bool primary = true) {
+  ImageCtx c;
+  if (!image_ctx(a, b, smem, primary, c)) return;
+  settle_unreliable(a, c, true, true);
+  stage_one(a, c);
+  if (c.need_s) {
+    consistency_keys(a, c);
+    const int m = list_rows(c, c.ia, true);
+    const uint16_t *ord = sort_rows(c.key, c.ia, c.ib, c.bid, m, c.hist, false);
+    stage_two_picks(a, c, ord, m);
+  }
+  emit_outputs(a, c);
 }
 
 // Where select_image leaves the kept local indices.
