@@ -608,7 +608,9 @@ FULL = [
 def test_workloads_full_size(name, bk, sample):
     # The full-size batch through tr_reduce and through the two-slot
     # pipeline bench.py times (three submissions: both slots, then slot 0
-    # again), each checked image by image on the sampled images.
+    # again; for a batch small enough that bench.py replays graphs of
+    # pipelined steps, a replayed graph of three too), each checked image by
+    # image on the sampled images.
     altr = _alt()
     w = synth.make(name, seed=0, device="cuda")
     if sample == "largest3":
@@ -616,10 +618,25 @@ def test_workloads_full_size(name, bk, sample):
     budget = altr.budgets(w.seqlens, **bk)
     single = altr.reduce(w.x, w.x_pre, w.x_post, seqlens=w.seqlens, budget=budget, scores=True)
     pipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, w.x.device, budget=budget, scores=True, slots=2)
+    results = [single]
     try:
-        piped = [pipe.submit(w.x, w.x_pre, w.x_post) for _ in range(3)][-1]
+        results.append([pipe.submit(w.x, w.x_pre, w.x_post) for _ in range(3)][-1])
         pipe.synchronize()
+        import bench
+        gpipe = None
+        if bench.step_bytes(w, budget[0])[0] < bench.GRAPH_BELOW_BYTES:
+            # bench.py replays CUDA graphs of pipelined steps for a batch this small
+            gpipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, w.x.device, budget=budget, scores=True, slots=2)
+            g = gpipe.graph(w.x, w.x_pre, w.x_post, steps=3)
+            g.replay()
+            torch.cuda.synchronize()
+            o = gpipe.outs[2 % gpipe.slots]
+            results.append(altr.ReduceResult(o["y"][:gpipe.total_k], o["idx"][:gpipe.total_k], gpipe.cu_k, o["h2"],
+                                             o["s"], o["status"]))
         x, xp, xq = w.x.cpu(), w.x_pre.cpu(), w.x_post.cpu()
-        compare_results([single, piped], x, xp, xq, w.seqlens, budget, images=sample)
+        compare_results(results, x, xp, xq, w.seqlens, budget, images=sample)
+        if gpipe is not None:
+            del g
+            gpipe.close()
     finally:
         pipe.close()
