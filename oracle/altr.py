@@ -7,20 +7,22 @@ baseline / reference arm use it.  It shares no code with the CUDA path.
 Plain, slow and obviously correct: numpy in float64 on the stored (already
 rounded) inputs, which convert to float64 exactly from bf16 and fp32.
 
-What it computes, step by step in the order of Algorithm 1:
+What it computes (Section IV, Eq. 3-7; the selection in the order the
+paper's Algorithm 1 gives it):
 
-1. budgets  K1 = floor(lambda K), K2 = K - K1                (Alg. 1 step 1, Eq. 7)
-2. p_ij = |x_ij| / sum_k |x_ik|                              (Eq. 3)
-3. H2(x_i) = -log sum_j p_ij^2                               (Eq. 4)
-4. X_imp = the K1 tokens with the highest H2                 (Section IV-A, Alg. 1)
-5. X_rem = X minus X_imp                                     (Alg. 1)
-6. s_i = x'_i . x''_i / (||x'_i|| ||x''_i||)                 (Eq. 6)
-7. sort X_rem by s ascending                                 (Section IV-B, Alg. 1)
-8. t = max(1, floor(|X_rem| / K2)); take sorted positions
-   0, t, 2t, ... up to K2 tokens (the 1-based 1, 1+t, ... of Alg. 1);
-   or, as the text of Section IV-B states it, a fixed real interval
-   |X_rem| / K2: positions floor(j |X_rem| / K2), j < K2
-9. X* = X_imp union X_div, returned in ascending token order (Eq. 7)
+* the budget split K1 = floor(lambda K), K2 = K - K1 (Eq. 7);
+* per token, the channel-magnitude distribution p_ij = |x_ij| / sum_k |x_ik|
+  (Eq. 3) and its Renyi-2 entropy H2(x_i) = -log sum_j p_ij^2 (Eq. 4);
+* Stage I: X_imp, the K1 tokens with the highest H2 (Section IV-A), and
+  X_rem, the tokens left over;
+* per token, the consistency signal s_i = x'_i . x''_i / (||x'_i|| ||x''_i||)
+  (Eq. 6), with x', x'' the final-layer MLP input and output (Eq. 5);
+* Stage II: X_rem sorted by s ascending and K2 tokens taken along that order
+  at the stride t = max(1, floor(|X_rem| / K2)), i.e. sorted positions
+  0, t, 2t, ... (Algorithm 1's 1-based 1, 1+t, ...), or, as the text of
+  Section IV-B states it, at the fixed real interval |X_rem| / K2:
+  positions floor(j |X_rem| / K2), j < K2 (Section IV-B);
+* X* = X_imp union X_div, returned in ascending token order (Eq. 7).
 
 Readings of points the paper leaves open:
 
@@ -54,7 +56,7 @@ NEAR_TIE = 1e-10
 
 
 # --------------------------------------------------------------------------
-# Step 1: budgets (Algorithm 1, first step; Eq. 7)
+# Budgets (Eq. 7)
 # --------------------------------------------------------------------------
 def budget_split(k: int, lam=(1, 3)):
     """K1 = floor(lambda K), K2 = K - K1 with lambda = lam[0] / lam[1]."""
@@ -98,7 +100,7 @@ def pick_positions(n_rem: int, k2: int, mode: str = "alg1") -> np.ndarray:
 
 
 # --------------------------------------------------------------------------
-# Steps 2-3: Renyi-2 entropy (Eq. 3, Eq. 4)
+# Importance: Renyi-2 entropy (Eq. 3, Eq. 4)
 # --------------------------------------------------------------------------
 def renyi2_entropy(x: np.ndarray) -> np.ndarray:
     """H2 per row of ``x`` [N, D] following Eq. 3 then Eq. 4, in float64."""
@@ -114,7 +116,7 @@ def renyi2_entropy(x: np.ndarray) -> np.ndarray:
 
 
 # --------------------------------------------------------------------------
-# Step 6: consistency signal (Eq. 6)
+# Consistency signal (Eq. 6)
 # --------------------------------------------------------------------------
 def consistency(x_pre: np.ndarray, x_post: np.ndarray) -> np.ndarray:
     """s_i = cos(x'_i, x''_i) per row, float64 (Eq. 6)."""
@@ -205,7 +207,7 @@ def _order(values: np.ndarray, exact_key, descending: bool) -> np.ndarray:
 
 
 # --------------------------------------------------------------------------
-# Steps 4-9: one image (Algorithm 1)
+# One image: Stage I and Stage II (Section IV-A, IV-B; Algorithm 1)
 # --------------------------------------------------------------------------
 def select_image(x, x_pre, x_post, k: int, k1: int, stride_mode: str = "alg1") -> dict:
     """Run Algorithm 1 on one image: x, x', x'' are [N, D] arrays.
@@ -236,22 +238,3 @@ def select_image(x, x_pre, x_post, k: int, k1: int, stride_mode: str = "alg1") -
         div = np.zeros(0, dtype=np.int64)
     kept = np.sort(np.concatenate([imp, div]))
     return dict(imp=imp, div=div, kept=kept, h2=h2, s=s, t=t, rem_sorted=rem_sorted)
-
-
-def reduce_batch(x, x_pre, x_post, seqlens, ks, k1s, stride_mode="alg1"):
-    """Algorithm 1 per image over a packed [T, D] batch.
-
-    Returns (idx, cu_k, rows): ``idx`` int32 local kept indices ascending per
-    image, ``cu_k`` the int32 prefix sums of K, and ``rows`` the global row
-    numbers of the kept tokens (the gather ``y = x[rows]`` is a bit copy).
-    """
-    idx, rows, cu_k = [], [], [0]
-    off = 0
-    for n, k, k1 in zip(seqlens, ks, k1s):
-        r = select_image(x[off:off + n], x_pre[off:off + n], x_post[off:off + n], k, k1, stride_mode)
-        idx.append(r["kept"].astype(np.int32))
-        rows.append(r["kept"].astype(np.int64) + off)
-        cu_k.append(cu_k[-1] + k)
-        off += n
-    cat = lambda a, t: np.concatenate(a).astype(t) if a else np.zeros(0, t)
-    return cat(idx, np.int32), np.asarray(cu_k, dtype=np.int32), cat(rows, np.int64)

@@ -70,6 +70,7 @@ SelectArgs select_args(const tr_tokens *in, const Shape &sh, const float *stats,
   a.status = d_status;
   a.bounds = certification_bounds(in->d, in->dtype);
   a.max_n = sh.max_n;
+  a.total_rows = sh.total;
   a.stride_interval = (in->flags & TR_STRIDE_INTERVAL) != 0;
   return a;
 }

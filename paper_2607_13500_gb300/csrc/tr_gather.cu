@@ -34,9 +34,13 @@ __global__ void __launch_bounds__(kGatherWarps * 32)
     if (__ldg(cu_k + mid) <= row) lo = mid; else hi = mid;
   }
   const long long first = cu_seqlens ? (long long)__ldg(cu_seqlens + lo) : (long long)lo * n_uniform;
-  const long long g = first + __ldcg(idx + row);  // through L2: idx may come from the kernel before
+  const long long n_b = cu_seqlens ? (long long)__ldg(cu_seqlens + lo + 1) - first : (long long)n_uniform;
+  const int local = __ldcg(idx + row);  // through L2: idx may come from the kernel before
+  const long long g = first + local;
   uint4 *dst = y + (long long)row * nchunks;
-  if (g < 0 || g >= total_rows) {  // never address outside x: bad indices write zeros
+  // an index outside its own image's tokens (or an image outside x) writes
+  // zeros: never a row of another image, never an address outside x
+  if (local < 0 || local >= n_b || first < 0 || g >= total_rows) {
     for (int c = lane; c < nchunks; c += 32) st_cs(dst + c, make_uint4(0u, 0u, 0u, 0u));
     return;
   }

@@ -173,6 +173,7 @@ struct SelectArgs {
   int32_t *status;    // or NULL
   Bounds bounds;
   int max_n;
+  long long total_rows;  // rows of x, x', x'' and of the statistics
   bool stride_interval;  // diversity picks at floor(j M / K2) instead of j t
 };
 

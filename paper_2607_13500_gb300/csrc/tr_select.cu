@@ -46,7 +46,8 @@ __device__ __forceinline__ void copy_kept(const SelectArgs &a, const int b, cons
     n = a.n_uniform;
   }
   const int k = a.k[b], k1 = a.k1[b], ko = a.cu_k[b];
-  if (n <= 0 || n > a.max_n || k < 0 || k > n || k1 < 0 || k1 > k) return;  // counted by select_image
+  if (n <= 0 || n > a.max_n || off < 0 || off + n > a.total_rows || k < 0 || k > n || k1 < 0 || k1 > k)
+    return;  // counted by select_image
   // this replica's share of the image's kept rows
   const uint16_t *kept = kept_rows(a, smem);
   const int j0 = (int)((long long)r * k / replicas), j1 = (int)((long long)(r + 1) * k / replicas);

@@ -230,6 +230,13 @@ __device__ __forceinline__ void add_term(long long *dg, int base, unsigned long 
 // Carry-propagates signed digits (value = sum dg[k] 2^(32k + base)) into a
 // trimmed sign-magnitude Big.  Returns false when more than kBigLimbs limbs
 // would be needed.
+//
+// The record is built in local storage and written to `out` (global memory)
+// with one struct store at the end: every store into an exact record carries
+// its final value.  Replica CTAs of one image (k_select_gather) recompute
+// the same rows into the same records; a replica that has finished a record
+// may already be reading it while another is still writing it, which is
+// harmless only because no store ever writes anything but the final bytes.
 __device__ bool normalize(const long long *dg, int base, Big &out) {
   uint32_t limb[kDig + 2];
   long long carry = 0;
@@ -249,27 +256,29 @@ __device__ bool normalize(const long long *dg, int base, Big &out) {
   }
   limb[kDig] = (uint32_t)carry;
   limb[kDig + 1] = (uint32_t)(carry >> 32);
+  Big t;
+  for (int i = 0; i < kBigLimbs; ++i) t.l[i] = 0u;
+  t.n = 0;
+  t.e = 0;
+  t.neg = 0;
   int hi = kDig + 1;
   while (hi >= 0 && limb[hi] == 0) --hi;
-  out.neg = 0;
-  if (hi < 0) {
-    out.n = 0;
-    out.e = 0;
-    return true;
+  bool ok = true;
+  if (hi >= 0) {
+    int lo = 0;
+    while (limb[lo] == 0) ++lo;
+    const int n = hi - lo + 1;
+    if (n > kBigLimbs) {
+      ok = false;  // stays the value 0; the caller flags the overflow
+    } else {
+      for (int i = 0; i < n; ++i) t.l[i] = limb[lo + i];
+      t.n = (uint8_t)n;
+      t.e = (int16_t)(lo + base / 32);
+      t.neg = neg ? 1 : 0;
+    }
   }
-  int lo = 0;
-  while (limb[lo] == 0) ++lo;
-  const int n = hi - lo + 1;
-  if (n > kBigLimbs) {
-    out.n = 0;
-    out.e = 0;
-    return false;
-  }
-  for (int i = 0; i < n; ++i) out.l[i] = limb[lo + i];
-  out.n = (uint8_t)n;
-  out.e = (int16_t)(lo + base / 32);
-  out.neg = neg ? 1 : 0;
-  return true;
+  out = t;
+  return ok;
 }
 
 __device__ __forceinline__ void warp_sum_digits(long long *dg) {
@@ -1350,7 +1359,9 @@ __device__ __forceinline__ bool image_ctx(const SelectArgs &a, const int b, unsi
     n = a.n_uniform;
   }
   const int k = a.k[b], k1 = a.k1[b];
-  if (n < 0 || n > a.max_n || k < 0 || k > n || k1 < 0 || k1 > k) {
+  // an image whose rows lie outside the packed tensors (malformed
+  // cu_seqlens) is skipped like an invalid budget: nothing is read or written
+  if (n < 0 || n > a.max_n || off < 0 || off + n > a.total_rows || k < 0 || k > n || k1 < 0 || k1 > k) {
     if (tid == 0 && a.status && primary) atomicAdd(&a.status[3], 1);
     return false;
   }

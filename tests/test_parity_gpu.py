@@ -115,6 +115,54 @@ def test_workloads_small(name, over, budgets):
         check_reduce(x, xp, xq, w.seqlens, _budget(w, **bk))
 
 
+# ---------------------------------------------------------------- full-size workloads (sampled)
+FULL = [
+    ("llava576", dict(k=192), None),
+    ("multitile2880", dict(k=320), None),
+    ("ragged_dynres", dict(ratio=(2, 9)), "largest3"),
+    ("video6272", dict(ratio=(1, 8)), [0, 7]),
+    ("single_clip336", dict(k=64), None),
+]
+
+
+@pytest.mark.parametrize("name,bk,sample", FULL, ids=[f[0] for f in FULL])
+def test_workloads_full_size(name, bk, sample):
+    # The full-size batch through tr_reduce and through the two-slot
+    # pipeline bench.py times (three submissions: both slots, then slot 0
+    # again; for a batch small enough that bench.py replays graphs of
+    # pipelined steps, a replayed graph of three too), each checked image by
+    # image on the sampled images.
+    altr = _alt()
+    w = synth.make(name, seed=0, device="cuda")
+    if sample == "largest3":
+        sample = sorted(range(w.batch), key=lambda b: -w.seqlens[b])[:2] + [0]
+    budget = altr.budgets(w.seqlens, **bk)
+    single = altr.reduce(w.x, w.x_pre, w.x_post, seqlens=w.seqlens, budget=budget, scores=True)
+    pipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, w.x.device, budget=budget, scores=True, slots=2)
+    results = [single]
+    try:
+        results.append([pipe.submit(w.x, w.x_pre, w.x_post) for _ in range(3)][-1])
+        pipe.synchronize()
+        import bench
+        gpipe = None
+        if bench.step_bytes(w, budget[0])[0] < bench.GRAPH_BELOW_BYTES:
+            # bench.py replays CUDA graphs of pipelined steps for a batch this small
+            gpipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, w.x.device, budget=budget, scores=True, slots=2)
+            g = gpipe.graph(w.x, w.x_pre, w.x_post, steps=3)
+            g.replay()
+            torch.cuda.synchronize()
+            o = gpipe.outs[2 % gpipe.slots]
+            results.append(altr.ReduceResult(o["y"][:gpipe.total_k], o["idx"][:gpipe.total_k], gpipe.cu_k, o["h2"],
+                                             o["s"], o["status"]))
+        x, xp, xq = w.x.cpu(), w.x_pre.cpu(), w.x_post.cpu()
+        compare_results(results, x, xp, xq, w.seqlens, budget, images=sample)
+        if gpipe is not None:
+            del g
+            gpipe.close()
+    finally:
+        pipe.close()
+
+
 @pytest.mark.parametrize("name,over,bud", [
     ("llava576", dict(batch=4), dict(k=64)),            # |X_rem| = 555, K2 = 43: interval 12.9
     ("multitile2880", dict(batch=2), dict(k=160)),      # 2827 / 107: interval 26.4
@@ -594,49 +642,65 @@ def test_fp32_wide_range():
     check_reduce(x, xp, xq, [100, 200], ([33, 66], [11, 22], [0, 33, 99]))
 
 
-# ---------------------------------------------------------------- full-size workloads (sampled)
-FULL = [
-    ("llava576", dict(k=192), None),
-    ("multitile2880", dict(k=320), None),
-    ("ragged_dynres", dict(ratio=(2, 9)), "largest3"),
-    ("video6272", dict(ratio=(1, 8)), [0, 7]),
-    ("single_clip336", dict(k=64), None),
-]
+# ---------------------------------------------------------------- malformed offsets and indices
+def _raw_tokens(x, xp, xq, batch, n=0, cu=None, total=None, max_n=0):
+    from paper_2607_13500_gb300 import _lib
+    return _lib.TrTokens(x=x.data_ptr(), x_pre=xp.data_ptr(), x_post=xq.data_ptr(), dtype=1, d=x.shape[1],
+                         batch=batch, n=n, cu_seqlens=None if cu is None else cu.data_ptr(),
+                         total=x.shape[0] if total is None else total, max_n=max_n, flags=0)
 
 
-@pytest.mark.parametrize("name,bk,sample", FULL, ids=[f[0] for f in FULL])
-def test_workloads_full_size(name, bk, sample):
-    # The full-size batch through tr_reduce and through the two-slot
-    # pipeline bench.py times (three submissions: both slots, then slot 0
-    # again; for a batch small enough that bench.py replays graphs of
-    # pipelined steps, a replayed graph of three too), each checked image by
-    # image on the sampled images.
-    altr = _alt()
-    w = synth.make(name, seed=0, device="cuda")
-    if sample == "largest3":
-        sample = sorted(range(w.batch), key=lambda b: -w.seqlens[b])[:2] + [0]
-    budget = altr.budgets(w.seqlens, **bk)
-    single = altr.reduce(w.x, w.x_pre, w.x_post, seqlens=w.seqlens, budget=budget, scores=True)
-    pipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, w.x.device, budget=budget, scores=True, slots=2)
-    results = [single]
-    try:
-        results.append([pipe.submit(w.x, w.x_pre, w.x_post) for _ in range(3)][-1])
-        pipe.synchronize()
-        import bench
-        gpipe = None
-        if bench.step_bytes(w, budget[0])[0] < bench.GRAPH_BELOW_BYTES:
-            # bench.py replays CUDA graphs of pipelined steps for a batch this small
-            gpipe = altr.Pipeline(w.seqlens, w.d, w.x.dtype, w.x.device, budget=budget, scores=True, slots=2)
-            g = gpipe.graph(w.x, w.x_pre, w.x_post, steps=3)
-            g.replay()
-            torch.cuda.synchronize()
-            o = gpipe.outs[2 % gpipe.slots]
-            results.append(altr.ReduceResult(o["y"][:gpipe.total_k], o["idx"][:gpipe.total_k], gpipe.cu_k, o["h2"],
-                                             o["s"], o["status"]))
-        x, xp, xq = w.x.cpu(), w.x_pre.cpu(), w.x_post.cpu()
-        compare_results(results, x, xp, xq, w.seqlens, budget, images=sample)
-        if gpipe is not None:
-            del g
-            gpipe.close()
-    finally:
-        pipe.close()
+def test_malformed_offsets_are_skipped():
+    # cu_seqlens whose second image runs past the packed rows (100 rows,
+    # image 1 claims rows 60..130): the selection counts that image in
+    # status[3] and reads and writes nothing for it, image 0 is reduced as
+    # usual, and the gather writes zeros into the skipped image's slots
+    # (its indices were never written).
+    import ctypes
+    from paper_2607_13500_gb300 import _lib
+    from paper_2607_13500_gb300.api import _ptr, _stream
+    lib = _lib.load()
+    dev = torch.device("cuda")
+    x, xp, xq = (t.to(dev) for t in _rows(100, 256, 41))
+    cu = torch.tensor([0, 60, 130], dtype=torch.int32, device=dev)
+    tok = _raw_tokens(x, xp, xq, 2, cu=cu, max_n=70)
+    ks, k1s, cuk = [20, 20], [6, 6], [0, 20, 40]
+    d_k, d_k1, d_cu = (torch.tensor(v, dtype=torch.int32, device=dev) for v in (ks, k1s, cuk))
+    nbytes = lib.tr_workspace_bytes(ctypes.byref(tok))
+    ws = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    y = torch.full((40, 256), float("nan"), dtype=torch.bfloat16, device=dev)
+    idx = torch.full((40,), -1, dtype=torch.int32, device=dev)
+    status = torch.zeros(4, dtype=torch.int32, device=dev)
+    _lib.check("tr_reduce", lib.tr_reduce(ctypes.byref(tok), _ptr(d_k), _ptr(d_k1), _ptr(d_cu), 40, _ptr(y),
+                                          _ptr(idx), None, None, _ptr(ws), nbytes, _ptr(status), _stream(dev)))
+    torch.cuda.synchronize()
+    assert status.cpu().tolist()[3] == 1
+    ref = oracle.select_image(_f64(x[:60]), _f64(xp[:60]), _f64(xq[:60]), 20, 6)
+    assert np.array_equal(idx[:20].cpu().numpy(), ref["kept"])
+    assert torch.equal(_bits(y[:20].cpu()), _bits(x[:60].cpu()[torch.from_numpy(ref["kept"].astype(np.int64))]))
+    assert idx[20:].cpu().tolist() == [-1] * 20
+    assert torch.equal(y[20:].cpu(), torch.zeros(20, 256, dtype=torch.bfloat16))
+
+
+@pytest.mark.parametrize("ragged", [False, True])
+def test_gather_index_outside_its_image_writes_zeros(ragged):
+    # tr_gather with indices that leave their own image (55 is a valid row
+    # of the next image, -3 is negative, 50 is one past the end) writes zeros
+    # for those slots and copies the others bit for bit.
+    import ctypes
+    from paper_2607_13500_gb300 import _lib
+    from paper_2607_13500_gb300.api import _ptr, _stream
+    lib = _lib.load()
+    dev = torch.device("cuda")
+    x, xp, xq = (t.to(dev) for t in _rows(100, 128, 42))
+    cu = torch.tensor([0, 50, 100], dtype=torch.int32, device=dev) if ragged else None
+    tok = _raw_tokens(x, xp, xq, 2, n=0 if ragged else 50, cu=cu, max_n=50)
+    idx = torch.tensor([0, 10, 55, -3, 1, 49, 50], dtype=torch.int32, device=dev)
+    d_cu = torch.tensor([0, 4, 7], dtype=torch.int32, device=dev)
+    y = torch.full((7, 128), float("nan"), dtype=torch.bfloat16, device=dev)
+    _lib.check("tr_gather", lib.tr_gather(ctypes.byref(tok), _ptr(d_cu), _ptr(idx), 7, _ptr(y), _stream(dev)))
+    torch.cuda.synchronize()
+    want = torch.zeros(7, 128, dtype=torch.bfloat16)
+    for slot, row in [(0, 0), (1, 10), (4, 51), (5, 99)]:
+        want[slot] = x[row].cpu()
+    assert torch.equal(_bits(y.cpu()), _bits(want))
