@@ -290,6 +290,68 @@ tr_status tr_pipeline_wait(tr_pipeline *p, void *stream);
 long long tr_pipeline_kernels(const tr_pipeline *p);
 tr_status tr_pipeline_destroy(tr_pipeline *p);
 
+/*
+ * ---- The encoder's final-layer MLP with the scoring fused in (Eq. 5) ----
+ *
+ * Section IV-B takes x' (the input of the vision encoder's last MLP) and
+ * x'' = f(x') = W2 sigma(W1 x') (its output, Eq. 5) from the encoder's
+ * forward pass.  These two calls run that MLP on the tensor cores, and the
+ * second one scores every token in its epilogue, so the selection needs no
+ * separate pass over x, x', x'':
+ *
+ *   tr_mlp_hidden:  H = sigma(x' W1^T + b1)                       [t, d_hidden]
+ *   tr_mlp_score:   x'' = H W2^T + b2, rounded to bf16 and stored  [t, d]
+ *                   x   = resid + x'' (the block's output tokens X, the
+ *                         Stage-I input and gather source), rounded to bf16
+ *                         and stored; x = x'' when resid is NULL
+ *                   stats: the per-row record of tr_score, with its sums
+ *                         taken over the stored x, x' and x''.
+ *
+ * tr_select (or tr_select_gather) then takes tokens {x, x', x''} and these
+ * stats exactly as it takes tr_score's; the result is the selection defined
+ * by the stored tensors.  The sums of each record carry less rounding than
+ * tr_score's (every term enters through TwoSum), within the same
+ * certification bounds.
+ *
+ * Operands and outputs are bf16, row-major, 16-byte aligned; d and d_hidden
+ * are multiples of 16.  Accumulation is fp32 in tensor memory; sigma is
+ * evaluated in fp32 on the accumulator plus b1 and rounded once to bf16.
+ * d_error (optional device int32, zero it first) gets a non-zero bit when a
+ * pipeline wait inside the kernel timed out (not expected in a correct run;
+ * the kernel then stops early and its outputs are incomplete).
+ */
+#define TR_ACT_GELU 0        /* x Phi(x), the erf form                        */
+#define TR_ACT_QUICK_GELU 1  /* x / (1 + exp(-1.702 x)), CLIP's variant        */
+#define TR_ACT_NONE 2
+#define TR_MLP_MAX_HIDDEN 65536
+typedef struct {
+  const void *x_pre;   /* [t, d] bf16: the MLP input x' (Eq. 5)                        */
+  const void *resid;   /* [t, d] bf16 added to x'' to form x, or NULL (x = x'')        */
+  const void *w1;      /* [d_hidden, d] bf16 (nn.Linear layout)                        */
+  const void *w2;      /* [d, d_hidden] bf16                                           */
+  const float *b1;     /* [d_hidden] fp32 or NULL                                      */
+  const float *b2;     /* [d] fp32 or NULL                                             */
+  int32_t t;           /* rows (tokens of the whole batch)                              */
+  int32_t d;           /* channels D                                                    */
+  int32_t d_hidden;    /* hidden width of the MLP                                       */
+  int32_t act;         /* sigma: TR_ACT_GELU, TR_ACT_QUICK_GELU or TR_ACT_NONE          */
+} tr_mlp;
+
+/* H = sigma(x' W1^T + b1): h is device bf16 [t, d_hidden]. */
+tr_status tr_mlp_hidden(const tr_mlp *m, void *h, int32_t *d_error, void *stream);
+
+/* Scratch bytes of tr_mlp_score (256-byte aligned device memory); 0 on invalid input. */
+size_t tr_mlp_workspace_bytes(const tr_mlp *m);
+
+/*
+ * x'' = H W2^T + b2 and x = resid + x'' (both stored, bf16 [t, d]) with the
+ * scoring of every row in the same pass: stats is device fp32
+ * [t, TR_STATS_WORDS] laid out as in tr_score, h2 / s optional fp32 [t].
+ * x_post and x must not overlap the inputs.
+ */
+tr_status tr_mlp_score(const tr_mlp *m, const void *h, void *x_post, void *x, float *stats, float *h2, float *s,
+                       void *ws, size_t ws_bytes, int32_t *d_error, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -7,8 +7,12 @@ the K1 most important tokens plus K2 tokens at a stride along the rest sorted
 by consistency (Algorithm 1), gathered into a compact [sum K, D] tensor.
 
 The work runs in libtr.so (hand-written CUDA for sm_103a, C ABI in
-include/tr.h); this package is its Python binding.
+include/tr.h); this package is its Python binding.  ``mlp`` runs the vision
+encoder's final-layer MLP (Eq. 5) on the tensor cores with the scoring fused
+into its second GEMM, for callers that own that MLP.
 """
-from .api import Pipeline, Reducer, ReduceResult, budgets, reduce, score, select, workspace_bytes
+from .api import (Mlp, MlpResult, Pipeline, Reducer, ReduceResult, budgets, mlp, reduce, score, select,
+                  workspace_bytes)
 
-__all__ = ["Pipeline", "Reducer", "ReduceResult", "budgets", "reduce", "score", "select", "workspace_bytes"]
+__all__ = ["Mlp", "MlpResult", "Pipeline", "Reducer", "ReduceResult", "budgets", "mlp", "reduce", "score", "select",
+           "workspace_bytes"]

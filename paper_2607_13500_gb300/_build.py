@@ -16,7 +16,7 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(HERE, "libtr.so")
-SOURCES = ["tr_api.cu", "tr_score.cu", "tr_select.cu", "tr_gather.cu", "tr_noalloc.cu"]
+SOURCES = ["tr_api.cu", "tr_score.cu", "tr_select.cu", "tr_gather.cu", "tr_noalloc.cu", "tr_mlp.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2", "-I", INCLUDE, "-I", CSRC]
 

@@ -36,6 +36,24 @@ class TrTokens(ctypes.Structure):
     ]
 
 
+TR_ACT = {"gelu": 0, "quick_gelu": 1, "none": 2}
+
+
+class TrMlp(ctypes.Structure):
+    _fields_ = [
+        ("x_pre", ctypes.c_void_p),
+        ("resid", ctypes.c_void_p),
+        ("w1", ctypes.c_void_p),
+        ("w2", ctypes.c_void_p),
+        ("b1", ctypes.c_void_p),
+        ("b2", ctypes.c_void_p),
+        ("t", ctypes.c_int32),
+        ("d", ctypes.c_int32),
+        ("d_hidden", ctypes.c_int32),
+        ("act", ctypes.c_int32),
+    ]
+
+
 class TrError(RuntimeError):
     def __init__(self, fn, code, lib):
         self.code = code
@@ -76,6 +94,11 @@ def load() -> ctypes.CDLL:
     lib.tr_pipeline_destroy.argtypes, lib.tr_pipeline_destroy.restype = [VP], I32
     lib.tr_reduce.argtypes = [tok, VP, VP, VP, I32, VP, VP, VP, VP, VP, SZ, VP, VP]
     lib.tr_reduce.restype = I32
+    mlp = P(TrMlp)
+    lib.tr_mlp_hidden.argtypes, lib.tr_mlp_hidden.restype = [mlp, VP, VP, VP], I32
+    lib.tr_mlp_workspace_bytes.argtypes, lib.tr_mlp_workspace_bytes.restype = [mlp], SZ
+    lib.tr_mlp_score.argtypes = [mlp, VP, VP, VP, VP, VP, VP, VP, SZ, VP, VP]
+    lib.tr_mlp_score.restype = I32
     _lib = lib
     return lib
 

@@ -12,7 +12,8 @@ from dataclasses import dataclass
 import torch
 
 from . import _lib
-from ._lib import STRIDE_MODES, TR_BF16, TR_F16, TR_F32, TR_STATS_WORDS, TR_STATUS_WORDS, TrTokens, check, load
+from ._lib import (STRIDE_MODES, TR_ACT, TR_BF16, TR_F16, TR_F32, TR_STATS_WORDS, TR_STATUS_WORDS, TrMlp,
+                   TrTokens, check, load)
 
 _I32 = ctypes.c_int32
 
@@ -532,3 +533,93 @@ def reduce(x, x_pre, x_post, k=None, ratio=None, lam=(1, 3), seqlens=None, score
                 scores=scores, budget=budget, stride=stride)
     out = r.run(x2, p2, q2)
     return out
+
+
+# ---------------------------------------------------------------- encoder MLP with fused scoring
+@dataclass
+class MlpResult:
+    h: torch.Tensor        # [T, d_hidden] sigma(x' W1^T + b1), bf16
+    x_post: torch.Tensor   # [T, D] x'' = H W2^T + b2, bf16 (Eq. 5)
+    x: torch.Tensor        # [T, D] block output resid + x'' (the tokens X), bf16
+    stats: torch.Tensor    # [T, 8] fp32 row records, as tr_score writes them
+    h2: torch.Tensor | None
+    s: torch.Tensor | None
+    error: torch.Tensor    # int32[1]: non-zero if a pipeline wait in a kernel timed out
+
+
+class Mlp:
+    """The encoder's final-layer MLP (Eq. 5) on the tensor cores with the
+    scoring fused into its second GEMM (tr_mlp_hidden, tr_mlp_score), for a
+    fixed shape; outputs and scratch are allocated once.
+
+    ``w1`` [d_hidden, D] and ``w2`` [D, d_hidden] bf16 (nn.Linear layout),
+    ``b1``/``b2`` fp32 or None, ``act`` "gelu", "quick_gelu" or "none"."""
+
+    def __init__(self, t, w1, w2, b1=None, b2=None, act="gelu", scores=False):
+        self.lib = load()
+        if w1.dtype != torch.bfloat16 or w2.dtype != torch.bfloat16:
+            raise TypeError("the MLP weights must be bf16")
+        dh, d = w1.shape
+        if tuple(w2.shape) != (d, dh):
+            raise ValueError("w2 must be [D, d_hidden] for w1 [d_hidden, D]")
+        if act not in TR_ACT:
+            raise ValueError(f"act must be one of {sorted(TR_ACT)}")
+        self.t, self.d, self.dh, self.act = int(t), int(d), int(dh), act
+        self.device = w1.device
+        dev = self.device
+        self.w1, self.w2 = w1.contiguous(), w2.contiguous()
+        self.b1 = None if b1 is None else b1.float().contiguous()
+        self.b2 = None if b2 is None else b2.float().contiguous()
+        self.h = torch.empty(max(self.t, 1), dh, dtype=torch.bfloat16, device=dev)
+        self.x_post = torch.empty(max(self.t, 1), d, dtype=torch.bfloat16, device=dev)
+        self.x = torch.empty(max(self.t, 1), d, dtype=torch.bfloat16, device=dev)
+        self.stats = torch.empty(max(self.t, 1), TR_STATS_WORDS, dtype=torch.float32, device=dev)
+        self.h2 = torch.empty(max(self.t, 1), dtype=torch.float32, device=dev) if scores else None
+        self.s = torch.empty(max(self.t, 1), dtype=torch.float32, device=dev) if scores else None
+        self.error = torch.zeros(1, dtype=torch.int32, device=dev)
+        self._ws = None
+
+    def _struct(self, x_pre, resid):
+        for t in (x_pre, resid):
+            if t is None:
+                continue
+            if t.dtype != torch.bfloat16 or tuple(t.shape) != (self.t, self.d) or not t.is_contiguous():
+                raise ValueError(f"x_pre / resid must be contiguous bf16 [{self.t}, {self.d}]")
+            if t.device != self.device:
+                raise ValueError("x_pre / resid must be on the weights' device")
+        return TrMlp(x_pre=x_pre.data_ptr(), resid=None if resid is None else resid.data_ptr(),
+                     w1=self.w1.data_ptr(), w2=self.w2.data_ptr(),
+                     b1=None if self.b1 is None else self.b1.data_ptr(),
+                     b2=None if self.b2 is None else self.b2.data_ptr(),
+                     t=self.t, d=self.d, d_hidden=self.dh, act=TR_ACT[self.act])
+
+    def run(self, x_pre, resid=None, events=None) -> MlpResult:
+        """Both GEMMs on the current stream; ``events`` (three torch.cuda.Event
+        or None) are recorded before, between and after them."""
+        m = self._struct(x_pre, resid)
+        ref = ctypes.byref(m)
+        if self._ws is None:
+            nbytes = self.lib.tr_mlp_workspace_bytes(ref)
+            self._ws = torch.empty(max(nbytes, 256), dtype=torch.uint8, device=self.device)
+            self._ws_bytes = nbytes
+        st = _stream(self.device)
+        if events:
+            events[0].record()
+        check("tr_mlp_hidden", self.lib.tr_mlp_hidden(ref, _ptr(self.h), _ptr(self.error), st))
+        if events:
+            events[1].record()
+        check("tr_mlp_score", self.lib.tr_mlp_score(ref, _ptr(self.h), _ptr(self.x_post), _ptr(self.x),
+                                                    _ptr(self.stats), _ptr(self.h2), _ptr(self.s), _ptr(self._ws),
+                                                    self._ws_bytes, _ptr(self.error), st))
+        if events:
+            events[2].record()
+        t = self.t
+        return MlpResult(self.h[:t], self.x_post[:t], self.x[:t], self.stats[:t],
+                         None if self.h2 is None else self.h2[:t], None if self.s is None else self.s[:t],
+                         self.error)
+
+
+def mlp(x_pre, w1, w2, b1=None, b2=None, resid=None, act="gelu", scores=False) -> MlpResult:
+    """The encoder's final-layer MLP with the scoring fused in, in one call
+    (Eq. 5; see Mlp)."""
+    return Mlp(x_pre.shape[0], w1, w2, b1, b2, act, scores).run(x_pre, resid)

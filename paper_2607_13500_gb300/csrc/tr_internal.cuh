@@ -90,6 +90,18 @@ inline Bounds certification_bounds(int d, int dtype) {
   // 16 and 22 significant bits, are exact), and sum|x'x''| <= sqrt(A B).
   double ep = 2.0 * u * u * (lane_terms * lane_terms + 12.0 * d) + 0x1p-52;
   if (dtype == TR_F32) ep *= 2.0;  // bf16 and fp16 products are exact in fp32
+  // The encoder-MLP GEMM's epilogue (tr_mlp_score, bf16) writes the same
+  // records: each term enters its double-float sum through TwoSum, over at
+  // most 256 columns per partial (low-part roundings below
+  // u^2 256 * 257 / 2 of the partial's sum|x'x''|), and the ceil(d / 256)
+  // partials are merged (2 roundings of at most u^2 257 of the total each).
+  // The bounds cover both producers of a record.  Its L1, S2, A and B are
+  // within that same tiny relative error, far inside g below.
+  if (dtype == TR_BF16) {
+    const double col_blocks = (double)((d + 255) / 256);
+    const double ep_mlp = u * u * (256.0 * 257.0 / 2.0 + 2.0 * 257.0 * col_blocks) + 0x1p-52;
+    if (ep_mlp > ep) ep = ep_mlp;
+  }
   Bounds b;
   // R32 = fl(R^) with R^ = L1^2 / S2 evaluated in double-float (2^-40) from
   // sums within relative g: R32 / R within (1 + g)^2 / (1 - g) (1 + 2^-40) (1 + u);

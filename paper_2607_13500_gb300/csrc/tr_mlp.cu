@@ -1,0 +1,509 @@
+// The vision encoder's final-layer MLP, x'' = W2 sigma(W1 x') (Eq. 5), on
+// the 5th-generation tensor cores, with ALTR's token scoring (Eq. 3-4 and
+// Eq. 6) fused into the epilogue of its second GEMM.
+//
+// The paper takes x' and x'' from the encoder's forward pass "at no extra
+// cost" (Section IV-B).  Here the second GEMM's epilogue, which produces
+// x'' anyway, rounds each element to bf16, stores it, forms the block
+// output x = bf16(resid + x'') and accumulates the five row sums of the
+// selection -- L1 = sum|x|, S2 = sum x^2, A = sum x'^2, B = sum x''^2,
+// P = sum x'x'' -- from the stored values, so a separate scoring pass over
+// x, x', x'' is not needed and the selection stays a function of the stored
+// tensors.  The row records it writes are the ones tr_score writes.
+//
+// One kernel serves both GEMMs (C[m, n] = A[m, k] B[n, k]^T, bf16 operands,
+// fp32 accumulation): a persistent grid of one CTA per SM walks 128 x 256
+// output tiles (tile t: row block t / n_tiles, column block t % n_tiles,
+// so the CTAs running at one time share row blocks of A in L2).  Per CTA:
+//   warp 0      TMA producer: A and B k-blocks (64 wide, 128-byte swizzle)
+//               into a 4-stage shared-memory ring;
+//   warp 1      allocates 512 TMEM columns (two 128 x 256 fp32
+//               accumulators) and issues tcgen05.mma (M 128, N 256, K 16)
+//               from one thread, committing each stage back to the
+//               producer and each finished accumulator to the epilogue;
+//   warps 2-5   epilogue: one thread per accumulator row (TMEM lane),
+//               16 columns per tcgen05.ld; the hidden GEMM applies
+//               bias + activation and stores H, the score GEMM stores x''
+//               and x and accumulates the row sums.
+// The epilogue of tile i overlaps the main loop of tile i + 1 (two TMEM
+// accumulators).  A row's sums over its n_tiles column blocks are combined
+// by the last of the CTAs that worked on its row block (an arrival counter;
+// no CTA waits for another), in column-block order, so the record does not
+// depend on which CTA finished first.
+#include <cuda.h>
+#include <cuda_bf16.h>
+
+#include <atomic>
+#include <climits>
+#include <mutex>
+
+#include "tr_internal.cuh"
+#include "tr_record.cuh"
+#include "tr_tc.cuh"
+
+namespace tr {
+namespace {
+
+constexpr int kBM = 128, kBN = 256, kBK = 64, kStages = 4;
+constexpr int kATile = kBM * kBK * 2;             // bytes of one A k-block
+constexpr int kBTile = kBN * kBK * 2;             // bytes of one B k-block
+constexpr int kStageBytes = kATile + kBTile;      // 48 KiB
+constexpr int kGemmThreads = 192;                 // 6 warps
+constexpr int kTmemCols = 2 * kBN;                // two accumulators
+constexpr int kChunk = 16;                        // columns per tcgen05.ld
+constexpr int kPartWords = 10;                    // hi, lo of L1, S2, A, B, P
+constexpr uint32_t kIdesc = tc::idesc_bf16(kBM, kBN);
+constexpr size_t kGemmSmem = (size_t)kStages * kStageBytes + 1024 + 256;
+
+struct GemmArgs {
+  int m, n, k;          // C[m, n] = A[m, k] B[n, k]^T
+  int n_tiles, tiles, kblocks;
+  const float *bias;    // [n] or NULL
+  int act;              // hidden GEMM: TR_ACT_*
+  uint16_t *out;        // hidden: H [m, n]; score: x'' [m, n] (bf16 bits)
+  const uint16_t *x_pre, *resid;  // score: x' [m, n], residual [m, n] or NULL
+  uint16_t *x;          // score: block output [m, n]
+  float *part;          // score: [row blocks][n_tiles][4][kPartWords][32] partial sums
+  int *arrivals;        // score: [row blocks][4], zero at launch
+  float4 *stats;        // score: [m] records (two float4 each)
+  float *h2, *s;        // score: optional outputs
+  int32_t *err;         // optional: set when a pipeline wait timed out
+};
+
+__device__ __forceinline__ float bf16_val(uint32_t bits16) { return __uint_as_float(bits16 << 16); }
+__device__ __forceinline__ uint32_t bf16_bits(float v) {  // round to nearest even
+  return static_cast<uint32_t>(__bfloat16_as_ushort(__float2bfloat16_rn(v)));
+}
+
+__device__ __forceinline__ float activate(float v, int act) {
+  if (act == TR_ACT_GELU) return 0.5f * v * (1.f + erff(v * 0.70710678118654752f));
+  if (act == TR_ACT_QUICK_GELU) return v / (1.f + expf(-1.702f * v));
+  return v;
+}
+
+__device__ __forceinline__ void flag_error(const GemmArgs &g, int code) {
+  if (g.err) atomicOr(g.err, code);
+}
+
+// Hidden GEMM epilogue for 16 columns of one row: H = bf16(act(acc + b1)).
+__device__ __forceinline__ void epi_hidden(const GemmArgs &g, long long row, int col0, const float (&v)[16]) {
+  uint32_t w[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    float a = v[2 * i], b = v[2 * i + 1];
+    if (g.bias) {
+      a += __ldg(g.bias + col0 + 2 * i);
+      b += __ldg(g.bias + col0 + 2 * i + 1);
+    }
+    w[i] = bf16_bits(activate(a, g.act)) | (bf16_bits(activate(b, g.act)) << 16);
+  }
+  uint4 *dst = reinterpret_cast<uint4 *>(g.out + row * g.n + col0);
+  dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
+  dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
+}
+
+// Score GEMM epilogue for 16 columns of one row: x'' = bf16(acc + b2),
+// x = bf16(resid + x''), both stored; the five sums take the stored values
+// (products and squares of bf16 values are exact in fp32; each term enters
+// its double-float sum through TwoSum).
+__device__ __forceinline__ void epi_score(const GemmArgs &g, long long row, int col0, const float (&v)[16],
+                                          Acc &acc) {
+  const long long base = row * g.n + col0;
+  const uint4 *pp = reinterpret_cast<const uint4 *>(g.x_pre + base);
+  const uint4 p0 = __ldg(pp), p1 = __ldg(pp + 1);
+  uint4 r0 = make_uint4(0u, 0u, 0u, 0u), r1 = r0;
+  if (g.resid) {
+    const uint4 *rp = reinterpret_cast<const uint4 *>(g.resid + base);
+    r0 = __ldg(rp);
+    r1 = __ldg(rp + 1);
+  }
+  const uint32_t pw[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
+  const uint32_t rw[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
+  uint32_t qo[8], xo[8];
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    uint32_t qb[2], xb[2];
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      const int c = 2 * i + h;
+      float a = v[c];
+      if (g.bias) a += __ldg(g.bias + col0 + c);
+      qb[h] = bf16_bits(a);
+      const float q = bf16_val(qb[h]);                         // x''
+      const float xp = bf16_val(h ? pw[i] >> 16 : pw[i] & 0xffffu);  // x'
+      float xv = q;                                            // x = resid + x'' (or x'')
+      if (g.resid) {
+        xb[h] = bf16_bits(bf16_val(h ? rw[i] >> 16 : rw[i] & 0xffffu) + q);
+        xv = bf16_val(xb[h]);
+      } else {
+        xb[h] = qb[h];
+      }
+      df_add(acc.l1, fabsf(xv));
+      df_add(acc.s2, xv * xv);
+      df_add(acc.a, xp * xp);
+      df_add(acc.b, q * q);
+      df_add(acc.p, xp * q);
+    }
+    qo[i] = qb[0] | (qb[1] << 16);
+    xo[i] = xb[0] | (xb[1] << 16);
+  }
+  uint4 *dq = reinterpret_cast<uint4 *>(g.out + base);
+  dq[0] = make_uint4(qo[0], qo[1], qo[2], qo[3]);
+  dq[1] = make_uint4(qo[4], qo[5], qo[6], qo[7]);
+  uint4 *dx = reinterpret_cast<uint4 *>(g.x + base);
+  dx[0] = make_uint4(xo[0], xo[1], xo[2], xo[3]);
+  dx[1] = make_uint4(xo[4], xo[5], xo[6], xo[7]);
+}
+
+// This warp's 32 rows of one tile are done: publish their partial sums; the
+// warp that completes a row block's quadrant (the last of its n_tiles
+// column blocks to arrive) merges the partials in column-block order and
+// writes the rows' records.
+__device__ __forceinline__ void publish_rows(const GemmArgs &g, int rb, int nt, int q, long long row, bool row_ok,
+                                             const Acc &acc) {
+  const int lane = threadIdx.x & 31;
+  float *dst = g.part + ((long long)(rb * g.n_tiles + nt) * 4 + q) * (kPartWords * 32) + lane;
+  const float vals[kPartWords] = {acc.l1.hi, acc.l1.lo, acc.s2.hi, acc.s2.lo, acc.a.hi,
+                                  acc.a.lo,  acc.b.hi,  acc.b.lo,  acc.p.hi,  acc.p.lo};
+#pragma unroll
+  for (int j = 0; j < kPartWords; ++j) __stcg(dst + 32 * j, vals[j]);
+  __threadfence();
+  __syncwarp();
+  int last = 0;
+  if (lane == 0) last = atomicAdd(g.arrivals + rb * 4 + q, 1) == g.n_tiles - 1;
+  last = __shfl_sync(0xffffffffu, last, 0);
+  if (!last) return;
+  __threadfence();
+  Acc tot{{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
+  for (int t = 0; t < g.n_tiles; ++t) {
+    const float *src = g.part + ((long long)(rb * g.n_tiles + t) * 4 + q) * (kPartWords * 32) + lane;
+    float w[kPartWords];
+#pragma unroll
+    for (int j = 0; j < kPartWords; ++j) w[j] = __ldcg(src + 32 * j);
+    df_merge(tot.l1, w[0], w[1]);
+    df_merge(tot.s2, w[2], w[3]);
+    df_merge(tot.a, w[4], w[5]);
+    df_merge(tot.b, w[6], w[7]);
+    df_merge(tot.p, w[8], w[9]);
+  }
+  if (row_ok) write_record(tot, row, g.stats, g.h2, g.s);
+  if (lane == 0) g.arrivals[rb * 4 + q] = 0;  // ready for the next launch
+}
+
+template <bool kScore>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+    k_mlp_gemm(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
+               const GemmArgs g) {
+  extern __shared__ unsigned char smem_raw[];
+  // stage tiles at a 1024-byte boundary (the swizzle atom), barriers after them
+  unsigned char *smem = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                          ~static_cast<uintptr_t>(1023));
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)kStages * kStageBytes);
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * kStages + 5);
+  const uint32_t sbase = tc::smem_u32(smem);
+  const uint32_t b0 = tc::smem_u32(bars);
+  auto full = [&](int s) { return b0 + 8u * s; };
+  auto empty = [&](int s) { return b0 + 8u * (kStages + s); };
+  auto tfull = [&](int a) { return b0 + 8u * (2 * kStages + a); };
+  auto tempty = [&](int a) { return b0 + 8u * (2 * kStages + 2 + a); };
+  const uint32_t done = b0 + 8u * (2 * kStages + 4);
+  auto sa = [&](int s) { return sbase + (uint32_t)(s * kStageBytes); };
+  auto sb = [&](int s) { return sbase + (uint32_t)(s * kStageBytes + kATile); };
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      tc::mbar_init(full(s), 1);
+      tc::mbar_init(empty(s), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      tc::mbar_init(tfull(a), 1);
+      tc::mbar_init(tempty(a), 4 * 32);
+    }
+    tc::mbar_init(done, 1);
+    tc::mbar_fence_init();
+    tc::tma_prefetch_map(&map_a);
+    tc::tma_prefetch_map(&map_b);
+  }
+  if (warp == 1) {
+    tc::tmem_alloc(tc::smem_u32(tmem_slot), kTmemCols);
+    tc::tmem_relinquish();
+  }
+  tc::fence_before_sync();
+  __syncthreads();
+  tc::fence_after_sync();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer
+    int stage = 0;
+    uint32_t phase = 0, filled = 0, last_parity = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < g.tiles && ok; tile += gridDim.x) {
+      const int rb = tile / g.n_tiles, nt = tile - rb * g.n_tiles;
+      for (int kb = 0; kb < g.kblocks; ++kb) {
+        if (!tc::mbar_wait_warp(empty(stage), phase ^ 1u)) {
+          ok = false;
+          break;
+        }
+        if (lane == 0) {
+          tc::mbar_expect_tx(full(stage), kStageBytes);
+          tc::tma_load_2d(sa(stage), &map_a, kb * kBK, rb * kBM, full(stage));
+          tc::tma_load_2d(sb(stage), &map_b, kb * kBK, nt * kBN, full(stage));
+        }
+        __syncwarp();
+        filled |= 1u << stage;
+        last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
+        if (++stage == kStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+    }
+    if (!ok && lane == 0) flag_error(g, 1);
+    // the loads already issued land before the CTA may exit
+    for (int s = 0; s < kStages; ++s)
+      if (filled & (1u << s)) tc::mbar_wait_warp(full(s), (last_parity >> s) & 1u);
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer
+    int stage = 0, acc = 0;
+    uint32_t phase = 0, acc_phase = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < g.tiles && ok; tile += gridDim.x) {
+      if (!tc::mbar_wait_warp(tempty(acc), acc_phase ^ 1u)) {
+        ok = false;
+        break;
+      }
+      tc::fence_after_sync();
+      const uint32_t d = tmem + (uint32_t)(acc * kBN);
+      for (int kb = 0; kb < g.kblocks; ++kb) {
+        if (!tc::mbar_wait_warp(full(stage), phase)) {
+          ok = false;
+          break;
+        }
+        tc::fence_after_sync();
+        if (lane == 0) {
+          const uint64_t da = tc::sw128_desc(sa(stage)), db = tc::sw128_desc(sb(stage));
+#pragma unroll
+          for (int k = 0; k < kBK / 16; ++k)  // 32 bytes further along K per step (start address >> 4: + 2)
+            tc::mma_bf16(d, da + 2u * k, db + 2u * k, kIdesc, (kb | k) != 0);
+          tc::mma_commit(empty(stage));  // the stage is free once these MMAs have read it
+        }
+        __syncwarp();
+        if (++stage == kStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+      if (!ok) break;
+      if (lane == 0) tc::mma_commit(tfull(acc));  // the accumulator is complete
+      __syncwarp();
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1u;
+    }
+    if (!ok && lane == 0) flag_error(g, 2);
+    // every MMA issued has completed before TMEM is released
+    if (lane == 0) tc::mma_commit(done);
+    __syncwarp();
+    tc::mbar_wait_warp(done, 0);
+  } else {
+    // ---------------------------------------------------------------- epilogue
+    const int q = warp & 3;  // TMEM lane quadrant this warp may read
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = blockIdx.x; tile < g.tiles; tile += gridDim.x) {
+      const int rb = tile / g.n_tiles, nt = tile - rb * g.n_tiles;
+      if (!tc::mbar_wait_warp(tfull(acc), acc_phase)) {
+        if (lane == 0) flag_error(g, 4);
+        break;
+      }
+      tc::fence_after_sync();
+      const long long row = (long long)rb * kBM + 32 * q + lane;
+      const bool row_ok = row < g.m;
+      const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(acc * kBN);
+      Acc sums{{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
+      for (int c = 0; c < kBN / kChunk; ++c) {
+        const int col0 = nt * kBN + c * kChunk;
+        if (col0 >= g.n) break;  // uniform across the warp
+        float v[16];
+        tc::tmem_ld16(taddr + (uint32_t)(c * kChunk), v);
+        if (row_ok) {
+          if (kScore)
+            epi_score(g, row, col0, v, sums);
+          else
+            epi_hidden(g, row, col0, v);
+        }
+      }
+      tc::fence_before_sync();
+      tc::mbar_arrive(tempty(acc));  // the MMA warp may refill this accumulator
+      if (kScore) publish_rows(g, rb, nt, q, row, row_ok, sums);
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1u;
+    }
+  }
+
+  tc::fence_before_sync();
+  __syncthreads();
+  if (warp == 1) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ---------------------------------------------------------------- host side
+using EncodeTiled = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                 const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                 CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiled encode_fn() {
+  static std::once_flag once;
+  static EncodeTiled fn = nullptr;
+  std::call_once(once, [] {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiled>(p);
+  });
+  return fn;
+}
+
+// Row-major bf16 [rows, cols] read in boxes of box_rows x 64 columns with the
+// 128-byte swizzle; out-of-range rows and columns read as zeros.
+bool make_map(CUtensorMap *map, const void *base, long long rows, long long cols, int box_rows) {
+  EncodeTiled fn = encode_fn();
+  if (!fn) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+  const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)box_rows};
+  const cuuint32_t estr[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+std::atomic<int> g_gemm_smem_set[64];
+
+template <bool kScore>
+cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, const GemmArgs &g, cudaStream_t st) {
+  if (g.tiles == 0) return cudaSuccess;
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err != cudaSuccess) return err;
+  const int bit = kScore ? 2 : 1;
+  if (!(g_gemm_smem_set[dev & 63].load() & bit)) {
+    err = cudaFuncSetAttribute(k_mlp_gemm<kScore>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmem);
+    if (err != cudaSuccess) return err;
+    g_gemm_smem_set[dev & 63].fetch_or(bit);
+  }
+  const int sms = sm_count();
+  if (sms <= 0) return cudaErrorInvalidDevice;
+  const int grid = g.tiles < sms ? g.tiles : sms;
+  k_mlp_gemm<kScore><<<grid, kGemmThreads, kGemmSmem, st>>>(ma, mb, g);
+  return cudaGetLastError();
+}
+
+bool misaligned16(const void *p) { return p && (reinterpret_cast<uintptr_t>(p) & 15u) != 0; }
+
+tr_status check_mlp(const tr_mlp *m) {
+  if (!m || !m->x_pre || !m->w1 || !m->w2) return TR_ERR_ARG;
+  if (m->t < 0 || m->d <= 0 || m->d_hidden <= 0) return TR_ERR_ARG;
+  if (m->act != TR_ACT_GELU && m->act != TR_ACT_QUICK_GELU && m->act != TR_ACT_NONE) return TR_ERR_ARG;
+  if (m->d % 16 != 0 || m->d_hidden % 16 != 0) return TR_ERR_ALIGN;
+  if (m->d > TR_MAX_D || m->d_hidden > TR_MLP_MAX_HIDDEN) return TR_ERR_UNSUPPORTED;
+  const long long rblocks = ((long long)m->t + kBM - 1) / kBM;  // tile counts stay in int
+  if (rblocks * ((m->d_hidden + kBN - 1) / kBN) > INT_MAX) return TR_ERR_UNSUPPORTED;
+  if (misaligned16(m->x_pre) || misaligned16(m->resid) || misaligned16(m->w1) || misaligned16(m->w2) ||
+      misaligned16(m->b1) || misaligned16(m->b2))
+    return TR_ERR_ALIGN;
+  return TR_OK;
+}
+
+struct MlpWs {
+  size_t part, arrivals, total;
+};
+MlpWs mlp_ws(const tr_mlp *m) {
+  const long long rblocks = ((long long)m->t + kBM - 1) / kBM;
+  const long long n_tiles = (m->d + kBN - 1) / kBN;
+  MlpWs w;
+  w.part = 0;
+  w.arrivals = align_up((size_t)rblocks * n_tiles * 4 * kPartWords * 32 * sizeof(float), 256);
+  w.total = align_up(w.arrivals + (size_t)rblocks * 4 * sizeof(int), 256);
+  return w;
+}
+
+}  // namespace
+}  // namespace tr
+
+using namespace tr;
+
+extern "C" {
+
+tr_status tr_mlp_hidden(const tr_mlp *m, void *h, int32_t *d_error, void *stream) {
+  tr_status rc = check_mlp(m);
+  if (rc != TR_OK) return rc;
+  if (!h) return TR_ERR_ARG;
+  if (misaligned16(h)) return TR_ERR_ALIGN;
+  if (m->t == 0) return TR_OK;
+  GemmArgs g{};
+  g.m = m->t;
+  g.n = m->d_hidden;
+  g.k = m->d;
+  g.n_tiles = (g.n + kBN - 1) / kBN;
+  g.tiles = ((g.m + kBM - 1) / kBM) * g.n_tiles;
+  g.kblocks = (g.k + kBK - 1) / kBK;
+  g.bias = m->b1;
+  g.act = m->act;
+  g.out = static_cast<uint16_t *>(h);
+  g.err = d_error;
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, m->x_pre, m->t, m->d, kBM) || !make_map(&mb, m->w1, m->d_hidden, m->d, kBN))
+    return TR_ERR_CUDA;
+  return launch_gemm<false>(ma, mb, g, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+}
+
+size_t tr_mlp_workspace_bytes(const tr_mlp *m) {
+  if (check_mlp(m) != TR_OK) return 0;
+  return mlp_ws(m).total;
+}
+
+tr_status tr_mlp_score(const tr_mlp *m, const void *h, void *x_post, void *x, float *stats, float *h2, float *s,
+                       void *ws, size_t ws_bytes, int32_t *d_error, void *stream) {
+  tr_status rc = check_mlp(m);
+  if (rc != TR_OK) return rc;
+  if (!h || !x_post || !x || !stats) return TR_ERR_ARG;
+  if (misaligned16(h) || misaligned16(x_post) || misaligned16(x) || misaligned16(stats) ||
+      (reinterpret_cast<uintptr_t>(h2) & 3u) || (reinterpret_cast<uintptr_t>(s) & 3u))
+    return TR_ERR_ALIGN;
+  const MlpWs w = mlp_ws(m);
+  if (!ws || (reinterpret_cast<uintptr_t>(ws) & 255u) || ws_bytes < w.total) return TR_ERR_WORKSPACE;
+  if (m->t == 0) return TR_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  char *wsb = static_cast<char *>(ws);
+  if (cudaMemsetAsync(wsb + w.arrivals, 0, w.total - w.arrivals, st) != cudaSuccess) return TR_ERR_CUDA;
+  GemmArgs g{};
+  g.m = m->t;
+  g.n = m->d;
+  g.k = m->d_hidden;
+  g.n_tiles = (g.n + kBN - 1) / kBN;
+  g.tiles = ((g.m + kBM - 1) / kBM) * g.n_tiles;
+  g.kblocks = (g.k + kBK - 1) / kBK;
+  g.bias = m->b2;
+  g.out = static_cast<uint16_t *>(x_post);
+  g.x_pre = static_cast<const uint16_t *>(m->x_pre);
+  g.resid = static_cast<const uint16_t *>(m->resid);
+  g.x = static_cast<uint16_t *>(x);
+  g.part = reinterpret_cast<float *>(wsb + w.part);
+  g.arrivals = reinterpret_cast<int *>(wsb + w.arrivals);
+  g.stats = reinterpret_cast<float4 *>(stats);
+  g.h2 = h2;
+  g.s = s;
+  g.err = d_error;
+  CUtensorMap ma, mb;
+  if (!make_map(&ma, h, m->t, m->d_hidden, kBM) || !make_map(&mb, m->w2, m->d, m->d_hidden, kBN))
+    return TR_ERR_CUDA;
+  return launch_gemm<true>(ma, mb, g, st) == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+}
+
+}  // extern "C"

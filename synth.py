@@ -192,3 +192,57 @@ def algorithmic_bytes(seqlens, ks, d, elem_bytes, aliased_pre=False):
     n = sum(seqlens)
     k = sum(ks)
     return streams * n * d * elem_bytes + 2 * k * d * elem_bytes + 4 * k
+
+
+# ---------------------------------------------------------------- encoder-MLP inputs
+# The encoder's final-layer MLP (Eq. 5) run on the device: its input x', the
+# residual stream it is added to, and seeded weights of the shape of a
+# CLIP-ViT-L/14 block (D = 1024, hidden 4096).  x'' and x are *not* drawn
+# here: the MLP kernels compute them.
+MLP_SPECS = {
+    "clip_mlp576": dict(batch=64, n=576, d=1024, d_hidden=4096, clusters=32, k=192),
+}
+
+
+@dataclass
+class MlpInputs:
+    name: str
+    x_pre: torch.Tensor    # [T, D] bf16: the MLP input x'
+    resid: torch.Tensor    # [T, D] bf16: the residual stream (x = resid + x'')
+    w1: torch.Tensor       # [d_hidden, D] bf16
+    w2: torch.Tensor       # [D, d_hidden] bf16
+    b1: torch.Tensor       # [d_hidden] fp32
+    b2: torch.Tensor       # [D] fp32
+    seqlens: list
+    k: int
+
+    @property
+    def total(self) -> int:
+        return self.x_pre.shape[0]
+
+    @property
+    def batch(self) -> int:
+        return len(self.seqlens)
+
+
+def make_mlp(name: str = "clip_mlp576", seed: int = 0, device="cpu", **over) -> MlpInputs:
+    """x' drawn with the cluster recipe above (1% activation outliers), the
+    residual equal to x' (the recipe's x = x' + x''), W1 ~ N(0, 1/D),
+    W2 ~ N(0, 1/d_hidden), biases ~ N(0, 0.02^2); all seeded.  Overrides:
+    batch, n, d, d_hidden, clusters, k."""
+    spec = dict(MLP_SPECS[name])
+    spec.update(over)
+    device = torch.device(device)
+    batch, n, d, dh = spec["batch"], spec["n"], spec["d"], spec["d_hidden"]
+    gen = torch.Generator(device=device).manual_seed(seed)
+    x_pre = torch.empty(batch * n, d, dtype=torch.bfloat16, device=device)
+    for b in range(batch):
+        h = _outliers(gen, _clustered(gen, n, d, spec["clusters"], device), device)
+        x_pre[b * n:(b + 1) * n] = h.to(torch.bfloat16)
+    w1 = (torch.randn(dh, d, generator=gen, device=device) / math.sqrt(d)).to(torch.bfloat16)
+    w2 = (torch.randn(d, dh, generator=gen, device=device) / math.sqrt(dh)).to(torch.bfloat16)
+    b1 = 0.02 * torch.randn(dh, generator=gen, device=device)
+    b2 = 0.02 * torch.randn(d, generator=gen, device=device)
+    return MlpInputs(name=name, x_pre=x_pre, resid=x_pre, w1=w1, w2=w2, b1=b1, b2=b2, seqlens=[n] * batch,
+                     k=spec["k"])
+
