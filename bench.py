@@ -616,6 +616,90 @@ def per_config(args, dev, altr, peak, world, barrier, seconds_cpu):
     return out
 
 
+def _bf16_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["bf16_tflops"]), float(p.get("bf16_tflops_sustained", p["bf16_tflops"])), "measured"
+    except Exception:
+        return 1900.0, 1700.0, "fallback"
+
+
+def measure_mlp(args, dev, altr, reps=20):
+    """The vision encoder's final-layer MLP with the scoring fused into its
+    second GEMM (Eq. 5, Section IV-B), then the selection, the gather and
+    the projector's first layer on the kept tokens read by index, on the
+    CLIP-ViT-L/14-shaped batch: 64 images x 576 tokens, D = 1024, hidden
+    4096, K = 192.  Each kernel timed with CUDA events on the current stream
+    (median of `reps` steps, inputs larger than L2); beside it, the unfused
+    route through the same library (cuBLAS MLP, tr_score pass) for context."""
+    w = synth.make_mlp("clip_mlp576", seed=args.seed, device=dev)
+    t, d, dh = w.total, w.x_pre.shape[1], w.w1.shape[0]
+    wp, bp = synth.make_projector(d, w.d_proj, seed=args.seed, device=dev)
+    budget = altr.budgets(w.seqlens, k=w.k)
+    ks, k1s, cu = budget
+    m = altr.Mlp(t, w.w1, w.w2, w.b1, w.b2, act=w.act)
+    red = altr.Reducer(w.seqlens, d, torch.bfloat16, dev, budget=budget)
+    # events: 0 | hidden | 1 | score | 2 (status zeroed) 3 | select | 4 | gather | 5 | project | 6
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(7)] for _ in range(reps + 3)]
+    spans = {"tr_mlp_hidden": (0, 1), "tr_mlp_score": (1, 2), "tr_select": (3, 4), "tr_gather": (4, 5),
+             "tr_project_kept": (5, 6)}
+    clocks = ClockSampler(dev)
+    for ev in evs:
+        out = m.run(w.x_pre, w.resid, events=ev[0:3])
+        r = red.run_select_gather(out.x, w.x_pre, out.x_post, out.stats, events=ev[3:6])
+        z, err = altr.project_kept(out.x, r.idx, cu, wp, bp, act="gelu", seqlens=w.seqlens, error=m.error)
+        ev[6].record()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    med = {n: statistics.median(ev[i].elapsed_time(ev[j]) for ev in evs[3:]) for n, (i, j) in spans.items()}
+    step = statistics.median(ev[0].elapsed_time(ev[6]) for ev in evs[3:])
+    status = red.status.cpu().tolist()
+    err_v = int(m.error.item())
+    # the unfused route, for context: the MLP through cuBLAS (torch), then
+    # the separate scoring pass over x, x', x''
+    act = torch.nn.functional.gelu if w.act == "gelu" else (lambda v: v * torch.sigmoid(1.702 * v))
+    u_ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(reps + 3)]
+    for ev in u_ev:
+        ev[0].record()
+        h = act(torch.nn.functional.linear(w.x_pre, w.w1, w.b1.to(torch.bfloat16)))
+        xq = torch.nn.functional.linear(h, w.w2, w.b2.to(torch.bfloat16))
+        xx = w.resid + xq
+        ev[1].record()
+        altr.score(xx, w.x_pre, xq, seqlens=w.seqlens)
+        ev[2].record()
+    torch.cuda.synchronize()
+    u_mlp = statistics.median(e[0].elapsed_time(e[1]) for e in u_ev[3:])
+    u_score = statistics.median(e[1].elapsed_time(e[2]) for e in u_ev[3:])
+    peak, peak_sus, kind = _bf16_peak()
+    flop = 2.0 * t * d * dh
+    total_k = cu[-1]
+    flop_p = 2.0 * total_k * d * w.d_proj
+    tf = lambda f, ms: f / (ms * 1e-3) / 1e12
+    e = 2  # bf16
+    return {
+        "workload": f"clip_mlp576: B={w.batch}, N=576, D={d}, hidden {dh} ({w.act}), bf16, K={w.k}, lambda=1/3; "
+                    f"projector first layer {d} -> {w.d_proj} (gelu) on the kept tokens",
+        "steps": reps, "ms_per_step": step, "value": w.batch / (step * 1e-3), "unit": "images/s",
+        "kernels_ms": med,
+        "roofline": {"bound": "tensor", "kernel": "tr_mlp_score (k_mlp_gemm, scoring epilogue)",
+                     "achieved": tf(flop, med["tr_mlp_score"]), "peak": peak, "unit": "TFLOP/s",
+                     "frac": tf(flop, med["tr_mlp_score"]) / peak,
+                     "peak_source": f"{kind} cuBLAS bf16 GEMM (burst)", "traffic": None,
+                     "algorithmic_flops": flop},
+        "gemm_tflops": {"tr_mlp_hidden": tf(flop, med["tr_mlp_hidden"]), "tr_mlp_score": tf(flop, med["tr_mlp_score"]),
+                        "tr_project_kept": tf(flop_p, med["tr_project_kept"]),
+                        "frac_of_measured_peak": {"tr_mlp_hidden": tf(flop, med["tr_mlp_hidden"]) / peak,
+                                                  "tr_mlp_score": tf(flop, med["tr_mlp_score"]) / peak,
+                                                  "tr_project_kept": tf(flop_p, med["tr_project_kept"]) / peak}},
+        "scoring_bytes": {"fused_extra_reads": t * d * e, "separate_pass_reads": 3 * t * d * e,
+                          "note": "the fused epilogue reads x' (its P and A terms); x'' and x are written by the "
+                                  "MLP in both routes; the separate pass reads x, x', x'' again"},
+        "unfused_context_ms": {"cublas_mlp_and_residual": u_mlp, "k_score_pass": u_score},
+        "clocks": clk, "status": status, "kernel_error": err_v,
+    }
+
+
 def run_ours(args, world, rank, local):
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
@@ -688,6 +772,9 @@ def run_ours(args, world, rank, local):
     if args.config_steps > 0 and not args.batch and not args.per_frame:
         line["per_config"] = per_config(args, dev, altr, peak, world, barrier,
                                         args.config_cpu_seconds if rank == 0 else 0.0)
+        torch.cuda.empty_cache()
+        line["mlp_fused"] = measure_mlp(args, dev, altr)
+        torch.cuda.empty_cache()
     if rank == 0 and world == 1:
         w = synth.make(args.workload, seed=args.seed, device="cpu", **over)
         if args.per_frame:

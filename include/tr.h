@@ -352,6 +352,28 @@ size_t tr_mlp_workspace_bytes(const tr_mlp *m);
 tr_status tr_mlp_score(const tr_mlp *m, const void *h, void *x_post, void *x, float *stats, float *h2, float *s,
                        void *ws, size_t ws_bytes, int32_t *d_error, void *stream);
 
+/*
+ * ---- The first projector layer on the kept tokens, gathered on the fly ----
+ *
+ * The projector P maps the kept tokens X* = X_imp union X_div (Eq. 7) into
+ * the LLM's embedding space (Z* = P(X*), Section III-A).  This call runs its
+ * first layer, z = sigma(X* W^T + bias), on the tensor cores with the rows of
+ * X* read straight from x by the selection's kept indices, so the gathered
+ * copy y (tr_gather) is not needed for it:
+ *   in:       the tokens x (bf16, as given to tr_select; x_pre / x_post unused)
+ *   d_cu_k:   device int32[batch+1] prefix sums of K_b; idx: device int32
+ *             [total_k] kept local indices (tr_select's output)
+ *   w:        device bf16 [d_out, d] (nn.Linear layout); bias fp32 [d_out] or NULL
+ *   act:      TR_ACT_GELU (LLaVA-1.5's projector), TR_ACT_QUICK_GELU, TR_ACT_NONE
+ *   z:        device bf16 [total_k, d_out], row r for kept slot r
+ * An index outside its image's tokens gives a row of zeros as input.  d and
+ * d_out are multiples of 16; pointers 16-byte aligned.  d_error as for
+ * tr_mlp_hidden.  Further projector layers are plain GEMMs on z.
+ */
+tr_status tr_project_kept(const tr_tokens *in, const int32_t *d_cu_k, const int32_t *idx, int32_t total_k,
+                          const void *w, const float *bias, int32_t d_out, int32_t act, void *z, int32_t *d_error,
+                          void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -99,6 +99,8 @@ def load() -> ctypes.CDLL:
     lib.tr_mlp_workspace_bytes.argtypes, lib.tr_mlp_workspace_bytes.restype = [mlp], SZ
     lib.tr_mlp_score.argtypes = [mlp, VP, VP, VP, VP, VP, VP, VP, SZ, VP, VP]
     lib.tr_mlp_score.restype = I32
+    lib.tr_project_kept.argtypes = [tok, VP, VP, I32, VP, VP, I32, I32, VP, VP, VP]
+    lib.tr_project_kept.restype = I32
     _lib = lib
     return lib
 

@@ -243,6 +243,27 @@ class Reducer:
         return ReduceResult(self.y[:self.total_k], self.idx[:self.total_k], self.cu_k, self.h2, self.s,
                             self.status)
 
+    def run_select_gather(self, x, x_pre, x_post, stats, events=None):
+        """tr_select then tr_gather on statistics records made elsewhere (e.g.
+        by Mlp's fused scoring), on the current stream; ``events`` (three
+        torch.cuda.Event or None) recorded before, between and after."""
+        tok = self._bind(x, x_pre, x_post)
+        st = _stream(self.device)
+        lib = self.lib
+        self.status.zero_()
+        if events:
+            events[0].record()
+        check("tr_select", lib.tr_select(
+            tok.ref(), _ptr(stats), _ptr(self.d_k), _ptr(self.d_k1), _ptr(self.d_cu), _ptr(self.idx), None,
+            _ptr(self.h2), _ptr(self.s), _ptr(self._ws), self._ws_bytes, _ptr(self.status), st))
+        if events:
+            events[1].record()
+        check("tr_gather", lib.tr_gather(tok.ref(), _ptr(self.d_cu), _ptr(self.idx), self.total_k, _ptr(self.y), st))
+        if events:
+            events[2].record()
+        return ReduceResult(self.y[:self.total_k], self.idx[:self.total_k], self.cu_k, self.h2, self.s,
+                            self.status)
+
     def run_separate(self, x, x_pre, x_post, events=None):
         """The three kernels the pipeline launches, tr_score, tr_select and
         tr_gather, on the current stream, with ``events`` (four
@@ -623,3 +644,27 @@ def mlp(x_pre, w1, w2, b1=None, b2=None, resid=None, act="gelu", scores=False) -
     """The encoder's final-layer MLP with the scoring fused in, in one call
     (Eq. 5; see Mlp)."""
     return Mlp(x_pre.shape[0], w1, w2, b1, b2, act, scores).run(x_pre, resid)
+
+
+def project_kept(x, idx, cu_k, w, bias=None, act="gelu", seqlens=None, error=None):
+    """tr_project_kept: z = sigma(X* W^T + bias) for the kept tokens X*, their
+    rows read from ``x`` by the selection's ``idx`` (local per image, image b
+    owning slots cu_k[b]..cu_k[b+1]) without a gathered copy.  ``w`` bf16
+    [d_out, D], ``bias`` fp32 [d_out] or None; returns z bf16 [sum K, d_out]."""
+    lib = load()
+    if x.dtype != torch.bfloat16 or w.dtype != torch.bfloat16:
+        raise TypeError("x and w must be bf16")
+    if act not in TR_ACT:
+        raise ValueError(f"act must be one of {sorted(TR_ACT)}")
+    x2, _, _, seqlens = _flatten(x, None, x, seqlens)
+    tok = _Tokens(x2, None, x2, seqlens)
+    total_k = int(cu_k[-1])
+    d_out = int(w.shape[0])
+    dev = x2.device
+    d_cu = torch.tensor(list(cu_k), dtype=torch.int32, device=dev)
+    b = None if bias is None else bias.float().contiguous()
+    z = torch.empty(max(total_k, 1), d_out, dtype=torch.bfloat16, device=dev)
+    err = torch.zeros(1, dtype=torch.int32, device=dev) if error is None else error
+    check("tr_project_kept", lib.tr_project_kept(tok.ref(), _ptr(d_cu), _ptr(idx), total_k, _ptr(w.contiguous()),
+                                                 _ptr(b), d_out, TR_ACT[act], _ptr(z), _ptr(err), _stream(dev)))
+    return z[:total_k], err

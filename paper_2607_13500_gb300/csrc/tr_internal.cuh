@@ -92,9 +92,10 @@ inline Bounds certification_bounds(int d, int dtype) {
   if (dtype == TR_F32) ep *= 2.0;  // bf16 and fp16 products are exact in fp32
   // The encoder-MLP GEMM's epilogue (tr_mlp_score, bf16) writes the same
   // records: each term enters its double-float sum through TwoSum, over at
-  // most 256 columns per partial (low-part roundings below
-  // u^2 256 * 257 / 2 of the partial's sum|x'x''|), and the ceil(d / 256)
-  // partials are merged (2 roundings of at most u^2 257 of the total each).
+  // most 128 columns per partial (low-part roundings below
+  // u^2 128 * 129 / 2 of the partial's sum|x'x''|), and the 2 ceil(d / 256)
+  // partials are merged (2 roundings of at most u^2 129 of the total each);
+  // the bound below, written for partials of up to 256 columns, covers that.
   // The bounds cover both producers of a record.  Its L1, S2, A and B are
   // within that same tiny relative error, far inside g below.
   if (dtype == TR_BF16) {

@@ -21,15 +21,26 @@
 //               accumulators) and issues tcgen05.mma (M 128, N 256, K 16)
 //               from one thread, committing each stage back to the
 //               producer and each finished accumulator to the epilogue;
-//   warps 2-5   epilogue: one thread per accumulator row (TMEM lane),
+//   warps 2-9   epilogue: one thread per accumulator row (TMEM lane) and
+//               column half (warps 2-5 columns 0-127, warps 6-9 128-255),
 //               16 columns per tcgen05.ld; the hidden GEMM applies
 //               bias + activation and stores H, the score GEMM stores x''
 //               and x and accumulates the row sums.
+// The projector mode (tr_project_kept) is the hidden GEMM with its A rows
+// gathered: A row j is token idx[j] of the image that owns kept slot j, so
+// the first projector layer reads X* = X_imp union X_div (Eq. 7) straight
+// from x without a gathered copy.  Four more warps (10-13) move those rows
+// with 16-byte cp.async copies into the 128-byte-swizzled layout TMA would
+// have written (chunk c of row r at r * 128 + ((c ^ (r & 7)) << 4)); a
+// copier waits for its copies of a stage, fences them into the async proxy
+// the tensor cores read through, and arrives on the stage's barrier, two
+// stages behind its issue so that copies stay in flight.
+//
 // The epilogue of tile i overlaps the main loop of tile i + 1 (two TMEM
-// accumulators).  A row's sums over its n_tiles column blocks are combined
-// by the last of the CTAs that worked on its row block (an arrival counter;
-// no CTA waits for another), in column-block order, so the record does not
-// depend on which CTA finished first.
+// accumulators).  A row's sums over its 2 n_tiles column halves are
+// combined by the last of the warps that worked on them (an arrival
+// counter; no warp or CTA waits for another), in column order, so the
+// record does not depend on which finished first.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
@@ -48,7 +59,11 @@ constexpr int kBM = 128, kBN = 256, kBK = 64, kStages = 4;
 constexpr int kATile = kBM * kBK * 2;             // bytes of one A k-block
 constexpr int kBTile = kBN * kBK * 2;             // bytes of one B k-block
 constexpr int kStageBytes = kATile + kBTile;      // 48 KiB
-constexpr int kGemmThreads = 192;                 // 6 warps
+constexpr int kEpiWarps = 8;                      // two warpgroups: column halves of a tile
+enum { kModeHidden = 0, kModeScore = 1, kModeProject = 2 };
+// producer, MMA issuer, epilogue (+ the four A copiers of the projector mode)
+__host__ __device__ constexpr int gemm_threads(int mode) { return 64 + 32 * kEpiWarps + (mode == 2 ? 128 : 0); }
+constexpr int kCopyLag = 2;                       // stages a copier keeps in flight before it signals
 constexpr int kTmemCols = 2 * kBN;                // two accumulators
 constexpr int kChunk = 16;                        // columns per tcgen05.ld
 constexpr int kPartWords = 10;                    // hi, lo of L1, S2, A, B, P
@@ -63,11 +78,16 @@ struct GemmArgs {
   uint16_t *out;        // hidden: H [m, n]; score: x'' [m, n] (bf16 bits)
   const uint16_t *x_pre, *resid;  // score: x' [m, n], residual [m, n] or NULL
   uint16_t *x;          // score: block output [m, n]
-  float *part;          // score: [row blocks][n_tiles][4][kPartWords][32] partial sums
+  float *part;          // score: [row blocks][n_tiles][2 halves][4][kPartWords][32] partial sums
   int *arrivals;        // score: [row blocks][4], zero at launch
   float4 *stats;        // score: [m] records (two float4 each)
   float *h2, *s;        // score: optional outputs
   int32_t *err;         // optional: set when a pipeline wait timed out
+  // projector mode: A row j = x[first row of the image owning kept slot j + idx[j]]
+  const uint16_t *gx;   // x [total_rows, k]
+  long long total_rows;
+  int batch, n_uniform;
+  const int32_t *cu_seqlens, *cu_k, *idx;
 };
 
 __device__ __forceinline__ float bf16_val(uint32_t bits16) { return __uint_as_float(bits16 << 16); }
@@ -155,14 +175,17 @@ __device__ __forceinline__ void epi_score(const GemmArgs &g, long long row, int 
   dx[1] = make_uint4(xo[4], xo[5], xo[6], xo[7]);
 }
 
-// This warp's 32 rows of one tile are done: publish their partial sums; the
-// warp that completes a row block's quadrant (the last of its n_tiles
-// column blocks to arrive) merges the partials in column-block order and
-// writes the rows' records.
-__device__ __forceinline__ void publish_rows(const GemmArgs &g, int rb, int nt, int q, long long row, bool row_ok,
-                                             const Acc &acc) {
+// This warp's 32 rows of one tile half are done: publish their partial
+// sums; the warp that completes a row block's quadrant (the last of its
+// 2 n_tiles column halves to arrive) merges the partials in column order
+// and writes the rows' records.
+__device__ __forceinline__ long long part_slot(const GemmArgs &g, int rb, int nt, int half, int q) {
+  return (((long long)(rb * g.n_tiles + nt) * 2 + half) * 4 + q) * (kPartWords * 32);
+}
+__device__ __forceinline__ void publish_rows(const GemmArgs &g, int rb, int nt, int half, int q, long long row,
+                                             bool row_ok, const Acc &acc) {
   const int lane = threadIdx.x & 31;
-  float *dst = g.part + ((long long)(rb * g.n_tiles + nt) * 4 + q) * (kPartWords * 32) + lane;
+  float *dst = g.part + part_slot(g, rb, nt, half, q) + lane;
   const float vals[kPartWords] = {acc.l1.hi, acc.l1.lo, acc.s2.hi, acc.s2.lo, acc.a.hi,
                                   acc.a.lo,  acc.b.hi,  acc.b.lo,  acc.p.hi,  acc.p.lo};
 #pragma unroll
@@ -170,13 +193,13 @@ __device__ __forceinline__ void publish_rows(const GemmArgs &g, int rb, int nt, 
   __threadfence();
   __syncwarp();
   int last = 0;
-  if (lane == 0) last = atomicAdd(g.arrivals + rb * 4 + q, 1) == g.n_tiles - 1;
+  if (lane == 0) last = atomicAdd(g.arrivals + rb * 4 + q, 1) == 2 * g.n_tiles - 1;
   last = __shfl_sync(0xffffffffu, last, 0);
   if (!last) return;
   __threadfence();
   Acc tot{{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
-  for (int t = 0; t < g.n_tiles; ++t) {
-    const float *src = g.part + ((long long)(rb * g.n_tiles + t) * 4 + q) * (kPartWords * 32) + lane;
+  for (int t = 0; t < 2 * g.n_tiles; ++t) {
+    const float *src = g.part + part_slot(g, rb, t >> 1, t & 1, q) + lane;
     float w[kPartWords];
 #pragma unroll
     for (int j = 0; j < kPartWords; ++j) w[j] = __ldcg(src + 32 * j);
@@ -190,8 +213,37 @@ __device__ __forceinline__ void publish_rows(const GemmArgs &g, int rb, int nt, 
   if (lane == 0) g.arrivals[rb * 4 + q] = 0;  // ready for the next launch
 }
 
-template <bool kScore>
-__global__ void __launch_bounds__(kGemmThreads, 1)
+// cp.async of 16 bytes (src_bytes = 0: zero fill, nothing read) and its groups.
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int kN>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(kN) : "memory");
+}
+__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
+
+// Row of x that kept slot j names (projector mode), or -1: the image b with
+// cu_k[b] <= j < cu_k[b + 1], its local index idx[j] checked against the
+// image's tokens (an index outside them gives a zero row, never another
+// image's token or an address outside x).
+__device__ __forceinline__ long long kept_source_row(const GemmArgs &g, long long j) {
+  if (j >= g.m) return -1;
+  int lo = 0, hi = g.batch;  // cu_k[lo] <= j < cu_k[hi]
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (__ldg(g.cu_k + mid) <= j) lo = mid; else hi = mid;
+  }
+  const long long first = g.cu_seqlens ? (long long)__ldg(g.cu_seqlens + lo) : (long long)lo * g.n_uniform;
+  const long long n_b = g.cu_seqlens ? (long long)__ldg(g.cu_seqlens + lo + 1) - first : (long long)g.n_uniform;
+  const int local = __ldg(g.idx + j);
+  if (local < 0 || local >= n_b || first < 0 || first + local >= g.total_rows) return -1;
+  return first + local;
+}
+
+template <int kMode>
+__global__ void __launch_bounds__(gemm_threads(kMode), 1)
     k_mlp_gemm(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
                const GemmArgs g) {
   extern __shared__ unsigned char smem_raw[];
@@ -213,12 +265,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      tc::mbar_init(full(s), 1);
+      tc::mbar_init(full(s), kMode == kModeProject ? 1 + 128 : 1);  // + the copiers' arrivals
       tc::mbar_init(empty(s), 1);
     }
     for (int a = 0; a < 2; ++a) {
       tc::mbar_init(tfull(a), 1);
-      tc::mbar_init(tempty(a), 4 * 32);
+      tc::mbar_init(tempty(a), 32 * kEpiWarps);
     }
     tc::mbar_init(done, 1);
     tc::mbar_fence_init();
@@ -247,8 +299,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           break;
         }
         if (lane == 0) {
-          tc::mbar_expect_tx(full(stage), kStageBytes);
-          tc::tma_load_2d(sa(stage), &map_a, kb * kBK, rb * kBM, full(stage));
+          if (kMode == kModeProject) {  // A comes from the copiers
+            tc::mbar_expect_tx(full(stage), kBTile);
+          } else {
+            tc::mbar_expect_tx(full(stage), kStageBytes);
+            tc::tma_load_2d(sa(stage), &map_a, kb * kBK, rb * kBM, full(stage));
+          }
           tc::tma_load_2d(sb(stage), &map_b, kb * kBK, nt * kBN, full(stage));
         }
         __syncwarp();
@@ -306,9 +362,49 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     if (lane == 0) tc::mma_commit(done);
     __syncwarp();
     tc::mbar_wait_warp(done, 0);
+  } else if (kMode == kModeProject && warp >= 2 + kEpiWarps) {
+    // ---------------------------------------------------------------- A copiers (projector mode)
+    const int r = (int)threadIdx.x - 32 * (2 + kEpiWarps);  // tile row of this thread
+    int stage = 0, pending = 0;  // stages copied into but not yet signalled: stage - pending ... stage - 1
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int tile = blockIdx.x; tile < g.tiles && ok; tile += gridDim.x) {
+      const int rb = tile / g.n_tiles;
+      const long long src = kept_source_row(g, (long long)rb * kBM + r);
+      const uint16_t *srow = g.gx + (src >= 0 ? src : 0) * g.k;
+      for (int kb = 0; kb < g.kblocks; ++kb) {
+        if (!tc::mbar_wait_warp(empty(stage), phase ^ 1u)) {
+          ok = false;
+          break;
+        }
+        const uint32_t dst = sa(stage) + (uint32_t)(r * 128);
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          const int col = kb * kBK + c * 8;
+          const bool in = src >= 0 && col < g.k;
+          cp_async16(dst + (uint32_t)((c ^ (r & 7)) << 4), in ? srow + col : g.gx, in ? 16u : 0u);
+        }
+        cp_async_commit();
+        if (++pending > kCopyLag) {  // the copies of the stage issued kCopyLag stages ago are complete
+          cp_async_wait<kCopyLag>();
+          fence_proxy_async();
+          tc::mbar_arrive(full((stage - kCopyLag + kStages) % kStages));
+          --pending;
+        }
+        if (++stage == kStages) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+    }
+    if (!ok && lane == 0) flag_error(g, 8);
+    cp_async_wait<0>();
+    fence_proxy_async();
+    for (int i = pending; i > 0; --i) tc::mbar_arrive(full((stage - i + kStages) % kStages));
   } else {
     // ---------------------------------------------------------------- epilogue
-    const int q = warp & 3;  // TMEM lane quadrant this warp may read
+    const int q = warp & 3;            // TMEM lane quadrant this warp may read
+    const int half = (warp - 2) >> 2;  // column half of the tile
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = blockIdx.x; tile < g.tiles; tile += gridDim.x) {
@@ -322,13 +418,14 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       const bool row_ok = row < g.m;
       const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(acc * kBN);
       Acc sums{{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
-      for (int c = 0; c < kBN / kChunk; ++c) {
-        const int col0 = nt * kBN + c * kChunk;
+      for (int c = 0; c < kBN / 2 / kChunk; ++c) {
+        const int tcol = half * (kBN / 2) + c * kChunk;  // column within the tile
+        const int col0 = nt * kBN + tcol;
         if (col0 >= g.n) break;  // uniform across the warp
         float v[16];
-        tc::tmem_ld16(taddr + (uint32_t)(c * kChunk), v);
+        tc::tmem_ld16(taddr + (uint32_t)tcol, v);
         if (row_ok) {
-          if (kScore)
+          if (kMode == kModeScore)
             epi_score(g, row, col0, v, sums);
           else
             epi_hidden(g, row, col0, v);
@@ -336,7 +433,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       }
       tc::fence_before_sync();
       tc::mbar_arrive(tempty(acc));  // the MMA warp may refill this accumulator
-      if (kScore) publish_rows(g, rb, nt, q, row, row_ok, sums);
+      if (kMode == kModeScore) publish_rows(g, rb, nt, half, q, row, row_ok, sums);
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1u;
     }
@@ -385,22 +482,22 @@ bool make_map(CUtensorMap *map, const void *base, long long rows, long long cols
 
 std::atomic<int> g_gemm_smem_set[64];
 
-template <bool kScore>
+template <int kMode>
 cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, const GemmArgs &g, cudaStream_t st) {
   if (g.tiles == 0) return cudaSuccess;
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
-  const int bit = kScore ? 2 : 1;
+  const int bit = 1 << kMode;
   if (!(g_gemm_smem_set[dev & 63].load() & bit)) {
-    err = cudaFuncSetAttribute(k_mlp_gemm<kScore>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmem);
+    err = cudaFuncSetAttribute(k_mlp_gemm<kMode>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmem);
     if (err != cudaSuccess) return err;
     g_gemm_smem_set[dev & 63].fetch_or(bit);
   }
   const int sms = sm_count();
   if (sms <= 0) return cudaErrorInvalidDevice;
   const int grid = g.tiles < sms ? g.tiles : sms;
-  k_mlp_gemm<kScore><<<grid, kGemmThreads, kGemmSmem, st>>>(ma, mb, g);
+  k_mlp_gemm<kMode><<<grid, gemm_threads(kMode), kGemmSmem, st>>>(ma, mb, g);
   return cudaGetLastError();
 }
 
@@ -428,7 +525,7 @@ MlpWs mlp_ws(const tr_mlp *m) {
   const long long n_tiles = (m->d + kBN - 1) / kBN;
   MlpWs w;
   w.part = 0;
-  w.arrivals = align_up((size_t)rblocks * n_tiles * 4 * kPartWords * 32 * sizeof(float), 256);
+  w.arrivals = align_up((size_t)rblocks * n_tiles * 2 * 4 * kPartWords * 32 * sizeof(float), 256);
   w.total = align_up(w.arrivals + (size_t)rblocks * 4 * sizeof(int), 256);
   return w;
 }
@@ -460,7 +557,7 @@ tr_status tr_mlp_hidden(const tr_mlp *m, void *h, int32_t *d_error, void *stream
   CUtensorMap ma, mb;
   if (!make_map(&ma, m->x_pre, m->t, m->d, kBM) || !make_map(&mb, m->w1, m->d_hidden, m->d, kBN))
     return TR_ERR_CUDA;
-  return launch_gemm<false>(ma, mb, g, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+  return launch_gemm<kModeHidden>(ma, mb, g, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TR_OK : TR_ERR_CUDA;
 }
 
 size_t tr_mlp_workspace_bytes(const tr_mlp *m) {
@@ -503,7 +600,54 @@ tr_status tr_mlp_score(const tr_mlp *m, const void *h, void *x_post, void *x, fl
   CUtensorMap ma, mb;
   if (!make_map(&ma, h, m->t, m->d_hidden, kBM) || !make_map(&mb, m->w2, m->d, m->d_hidden, kBN))
     return TR_ERR_CUDA;
-  return launch_gemm<true>(ma, mb, g, st) == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+  return launch_gemm<kModeScore>(ma, mb, g, st) == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+}
+
+tr_status tr_project_kept(const tr_tokens *in, const int32_t *d_cu_k, const int32_t *idx, int32_t total_k,
+                          const void *w, const float *bias, int32_t d_out, int32_t act, void *z, int32_t *d_error,
+                          void *stream) {
+  if (!in || !in->x || !w || !z) return TR_ERR_ARG;
+  if (in->dtype != TR_BF16) return TR_ERR_DTYPE;
+  if (in->d <= 0 || d_out <= 0 || in->batch < 0) return TR_ERR_ARG;
+  if (act != TR_ACT_GELU && act != TR_ACT_QUICK_GELU && act != TR_ACT_NONE) return TR_ERR_ARG;
+  if (in->d % 16 != 0 || d_out % 16 != 0) return TR_ERR_ALIGN;
+  if (in->d > TR_MAX_D || d_out > TR_MLP_MAX_HIDDEN) return TR_ERR_UNSUPPORTED;
+  if (misaligned16(in->x) || misaligned16(w) || misaligned16(bias) || misaligned16(z)) return TR_ERR_ALIGN;
+  long long total_rows;
+  if (in->cu_seqlens) {
+    if (in->total < 0) return TR_ERR_ARG;
+    total_rows = in->total;
+  } else {
+    if (in->n < 0) return TR_ERR_ARG;
+    total_rows = (long long)in->batch * in->n;
+  }
+  if (total_k < 0 || total_k > total_rows) return TR_ERR_BUDGET;
+  if (total_k == 0) return TR_OK;
+  if (in->batch == 0 || !d_cu_k || !idx) return TR_ERR_ARG;
+  const long long rblocks = ((long long)total_k + kBM - 1) / kBM;
+  if (rblocks * ((d_out + kBN - 1) / kBN) > INT_MAX) return TR_ERR_UNSUPPORTED;
+  GemmArgs g{};
+  g.m = total_k;
+  g.n = d_out;
+  g.k = in->d;
+  g.n_tiles = (g.n + kBN - 1) / kBN;
+  g.tiles = (int)rblocks * g.n_tiles;
+  g.kblocks = (g.k + kBK - 1) / kBK;
+  g.bias = bias;
+  g.act = act;
+  g.out = static_cast<uint16_t *>(z);
+  g.err = d_error;
+  g.gx = static_cast<const uint16_t *>(in->x);
+  g.total_rows = total_rows;
+  g.batch = in->batch;
+  g.n_uniform = in->cu_seqlens ? 0 : in->n;
+  g.cu_seqlens = in->cu_seqlens;
+  g.cu_k = d_cu_k;
+  g.idx = idx;
+  CUtensorMap mb;
+  if (!make_map(&mb, w, d_out, in->d, kBN)) return TR_ERR_CUDA;
+  return launch_gemm<kModeProject>(mb, mb, g, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TR_OK
+                                                                                                 : TR_ERR_CUDA;
 }
 
 }  // extern "C"

@@ -200,7 +200,9 @@ def algorithmic_bytes(seqlens, ks, d, elem_bytes, aliased_pre=False):
 # CLIP-ViT-L/14 block (D = 1024, hidden 4096).  x'' and x are *not* drawn
 # here: the MLP kernels compute them.
 MLP_SPECS = {
-    "clip_mlp576": dict(batch=64, n=576, d=1024, d_hidden=4096, clusters=32, k=192),
+    # CLIP-ViT-L/14-336 (LLaVA-1.5's vision tower): QuickGELU in its MLP
+    "clip_mlp576": dict(batch=64, n=576, d=1024, d_hidden=4096, clusters=32, k=192, act="quick_gelu",
+                        d_proj=4096),
 }
 
 
@@ -215,6 +217,8 @@ class MlpInputs:
     b2: torch.Tensor       # [D] fp32
     seqlens: list
     k: int
+    act: str = "gelu"
+    d_proj: int = 4096   # width of the projector's first layer (LLaVA-1.5: 1024 -> 4096)
 
     @property
     def total(self) -> int:
@@ -244,5 +248,13 @@ def make_mlp(name: str = "clip_mlp576", seed: int = 0, device="cpu", **over) -> 
     b1 = 0.02 * torch.randn(dh, generator=gen, device=device)
     b2 = 0.02 * torch.randn(d, generator=gen, device=device)
     return MlpInputs(name=name, x_pre=x_pre, resid=x_pre, w1=w1, w2=w2, b1=b1, b2=b2, seqlens=[n] * batch,
-                     k=spec["k"])
+                     k=spec["k"], act=spec.get("act", "gelu"), d_proj=spec.get("d_proj", 4096))
+
+
+def make_projector(d: int, d_proj: int, seed: int = 0, device="cpu"):
+    """Seeded weights of the projector's first layer: W_p ~ N(0, 1/D) bf16
+    [d_proj, D] and a bias ~ N(0, 0.02^2) fp32 [d_proj]."""
+    gen = torch.Generator(device=torch.device(device)).manual_seed(seed + 77)
+    w = (torch.randn(d_proj, d, generator=gen, device=device) / math.sqrt(d)).to(torch.bfloat16)
+    return w, 0.02 * torch.randn(d_proj, generator=gen, device=device)
 

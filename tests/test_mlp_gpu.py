@@ -192,3 +192,56 @@ def test_fused_selection_full_size():
     assert torch.equal(out.x.view(torch.int16), want_x.view(torch.int16))
     budget = altr.budgets(w.seqlens, k=w.k)
     _select_and_check(altr, out, w.x_pre, w.seqlens, budget, [0, 37, 63])
+
+
+# ---------------------------------------------------------------- projector on the kept tokens
+def _hidden_on(altr, y, w, bias, act):
+    """The hidden-GEMM kernel run on an explicit gathered copy y (TMA loads):
+    the same MMA inputs as tr_project_kept, which reads the rows by index."""
+    m = altr.Mlp(y.shape[0], w, w.t().contiguous(), bias, None, act=act)
+    out = m.run(y.contiguous())
+    return out.h, out.error
+
+
+@pytest.mark.parametrize("name,over,bud,d_out,act", [
+    ("llava576", dict(batch=3, d=1024), dict(k=192), 4096, "gelu"),           # LLaVA-1.5's 1024 -> 4096 layer
+    ("ragged_dynres", dict(batch=5, n=(256, 3000), d=1152), dict(ratio=(2, 9)), 1280, "quick_gelu"),
+], ids=["llava576", "ragged_dynres"])
+def test_project_kept(name, over, bud, d_out, act):
+    # Selection, then the projector's first layer on the kept tokens read
+    # from x by index: bit for bit the hidden GEMM on the gathered copy y,
+    # and within the GEMM tolerance of float64 on the kept rows.
+    altr = _alt()
+    w_in = synth.make(name, seed=17, device="cuda", **over)
+    budget = altr.budgets(w_in.seqlens, **bud)
+    r = altr.reduce(w_in.x, w_in.x_pre, w_in.x_post, seqlens=w_in.seqlens, budget=budget)
+    g = torch.Generator(device="cuda").manual_seed(5)
+    w = (torch.randn(d_out, w_in.d, generator=g, device="cuda") / math.sqrt(w_in.d)).to(torch.bfloat16)
+    bias = 0.05 * torch.randn(d_out, generator=g, device="cuda")
+    z, err = altr.project_kept(w_in.x, r.idx, budget[2], w, bias, act=act, seqlens=w_in.seqlens)
+    zh, err_h = _hidden_on(altr, r.y, w, bias, act)
+    torch.cuda.synchronize()
+    assert err.item() == 0 and err_h.item() == 0
+    assert torch.equal(z.view(torch.int16), zh.view(torch.int16))
+    v, mag = _gemm_ref(r.y, w, bias)
+    _check_close(z, _sigma(v, act), mag, slope=1.13)
+
+
+def test_project_kept_index_outside_its_image():
+    # A kept index past its image's tokens (or negative) feeds a zero row:
+    # its output row is sigma(bias), the other rows are untouched by it.
+    altr = _alt()
+    x = _inputs(100, 256, 512, seed=9, resid=False, bias=False)[0]
+    idx = torch.tensor([0, 10, 55, -3, 1, 49, 50], dtype=torch.int32, device="cuda")
+    cu = [0, 4, 7]
+    g = torch.Generator(device="cuda").manual_seed(6)
+    w = (torch.randn(256, 256, generator=g, device="cuda") / 16).to(torch.bfloat16)
+    bias = 0.1 * torch.randn(256, generator=g, device="cuda")
+    z, err = altr.project_kept(x, idx, cu, w, bias, act="gelu", seqlens=[50, 50])
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    rows = torch.zeros(7, 256, dtype=torch.bfloat16, device="cuda")  # slots 2, 3, 6 stay zero rows
+    for slot, row in [(0, 0), (1, 10), (4, 51), (5, 99)]:
+        rows[slot] = x[row]
+    v, mag = _gemm_ref(rows, w, bias)
+    _check_close(z, _sigma(v, "gelu"), mag, slope=1.13)
