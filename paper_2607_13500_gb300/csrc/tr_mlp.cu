@@ -95,10 +95,31 @@ __device__ __forceinline__ uint32_t bf16_bits(float v) {  // round to nearest ev
   return static_cast<uint32_t>(__bfloat16_as_ushort(__float2bfloat16_rn(v)));
 }
 
+// erf(z) for z >= 0 by Abramowitz and Stegun, Handbook of Mathematical
+// Functions (1964), formula 7.1.26: 1 - (a1 t + ... + a5 t^5) exp(-z^2) with
+// t = 1 / (1 + p z), |error| <= 1.5e-7; evaluated with the fast exponential
+// and reciprocal intrinsics (a few ulp each), so GELU below stays within
+// ~2e-7 |v| of x Phi(x), far inside the bf16 rounding of its result.
+__device__ __forceinline__ float erf_as(float z) {
+  const float t = __fdividef(1.f, fmaf(0.3275911f, z, 1.f));
+  const float poly =
+      t * fmaf(t, fmaf(t, fmaf(t, fmaf(t, 1.061405429f, -1.453152027f), 1.421413741f), -0.284496736f), 0.254829592f);
+  return 1.f - poly * __expf(-z * z);
+}
+
 __device__ __forceinline__ float activate(float v, int act) {
-  if (act == TR_ACT_GELU) return 0.5f * v * (1.f + erff(v * 0.70710678118654752f));
-  if (act == TR_ACT_QUICK_GELU) return v / (1.f + expf(-1.702f * v));
+  if (act == TR_ACT_GELU) {  // v Phi(v) = v (1 + erf(v / sqrt 2)) / 2
+    const float e = erf_as(fabsf(v) * 0.70710678118654752f);
+    return 0.5f * v * (1.f + copysignf(e, v));
+  }
+  if (act == TR_ACT_QUICK_GELU)  // v sigma(1.702 v); the exponent is capped so the divisor stays finite
+    return __fdividef(v, 1.f + __expf(fminf(-1.702f * v, 80.f)));
   return v;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t *>(&h);
 }
 
 __device__ __forceinline__ void flag_error(const GemmArgs &g, int code) {
@@ -107,16 +128,23 @@ __device__ __forceinline__ void flag_error(const GemmArgs &g, int code) {
 
 // Hidden GEMM epilogue for 16 columns of one row: H = bf16(act(acc + b1)).
 __device__ __forceinline__ void epi_hidden(const GemmArgs &g, long long row, int col0, const float (&v)[16]) {
+  float a[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) a[i] = v[i];
+  if (g.bias) {  // the same 16 values in every lane: four broadcast loads
+    const float4 *bp = reinterpret_cast<const float4 *>(g.bias + col0);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float4 b = __ldg(bp + i);
+      a[4 * i] += b.x;
+      a[4 * i + 1] += b.y;
+      a[4 * i + 2] += b.z;
+      a[4 * i + 3] += b.w;
+    }
+  }
   uint32_t w[8];
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    float a = v[2 * i], b = v[2 * i + 1];
-    if (g.bias) {
-      a += __ldg(g.bias + col0 + 2 * i);
-      b += __ldg(g.bias + col0 + 2 * i + 1);
-    }
-    w[i] = bf16_bits(activate(a, g.act)) | (bf16_bits(activate(b, g.act)) << 16);
-  }
+  for (int i = 0; i < 8; ++i) w[i] = pack_bf16x2(activate(a[2 * i], g.act), activate(a[2 * i + 1], g.act));
   uint4 *dst = reinterpret_cast<uint4 *>(g.out + row * g.n + col0);
   dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
   dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
@@ -447,6 +475,241 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
   }
 }
 
+// ---------------------------------------------------------------- the SM-pair kernel
+// The same GEMM with tcgen05's 2-SM MMA: a cluster of two CTAs shares each
+// 256 x 256 output tile (tile t: row block t / n_tiles of 256 rows).  CTA
+// rank r loads A rows 128 r .. 128 r + 127 of the tile and B rows (output
+// columns) 128 r .. 128 r + 127 into its own shared memory -- 32 KiB per
+// k-block stage, six stages -- and both CTAs' loads complete on the even
+// CTA's stage barrier.  The even CTA alone issues the pair's MMAs (M 256,
+// N 256, K 16), which read both CTAs' stages and write each CTA's 128
+// accumulator rows into its own TMEM; its commits reach the same barriers
+// in both CTAs (multicast).  Each CTA's epilogue drains its own rows and
+// releases the accumulator on the even CTA's barrier.  Per SM a k-block
+// brings 32 KiB of operands for a 128 x 256 x 64 product, against 48 KiB on
+// one SM, so six stages in flight hide the load latency that four did not.
+constexpr int kStagesP = 6;
+constexpr int kHalfTile = 128 * kBK * 2;          // 128 rows of a k-block (A or B)
+constexpr int kStagePBytes = 2 * kHalfTile;       // this CTA's A rows + B rows
+constexpr uint32_t kIdescPair = tc::idesc_bf16(2 * kBM, kBN);
+constexpr size_t kGemmPSmem = (size_t)kStagesP * kStagePBytes + 1024 + 256;
+
+template <int kMode>
+__global__ void __launch_bounds__(gemm_threads(kMode), 1)
+    k_mlp_gemm_pair(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
+                    const GemmArgs g) {
+  extern __shared__ unsigned char smem_raw[];
+  unsigned char *smem = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                                          ~static_cast<uintptr_t>(1023));
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)kStagesP * kStagePBytes);
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * kStagesP + 5);
+  const uint32_t sbase = tc::smem_u32(smem);
+  const uint32_t b0 = tc::smem_u32(bars);
+  auto full = [&](int s) { return b0 + 8u * s; };
+  auto empty = [&](int s) { return b0 + 8u * (kStagesP + s); };
+  auto tfull = [&](int a) { return b0 + 8u * (2 * kStagesP + a); };
+  auto tempty = [&](int a) { return b0 + 8u * (2 * kStagesP + 2 + a); };
+  const uint32_t done = b0 + 8u * (2 * kStagesP + 4);
+  auto sa = [&](int s) { return sbase + (uint32_t)(s * kStagePBytes); };
+  auto sb = [&](int s) { return sbase + (uint32_t)(s * kStagePBytes + kHalfTile); };
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const uint32_t rank = tc::cluster_rank();
+  const bool leader = rank == 0;
+  const int cluster = blockIdx.x >> 1, clusters = gridDim.x >> 1;
+  // operand bytes landing on the even CTA's stage barrier per k-block (both CTAs)
+  constexpr uint32_t kTx = kMode == kModeProject ? 2 * kHalfTile : 2 * kStagePBytes;
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStagesP; ++s) {
+      tc::mbar_init(full(s), kMode == kModeProject ? 1 + 2 * 128 : 1);  // + both CTAs' A copiers
+      tc::mbar_init(empty(s), 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      tc::mbar_init(tfull(a), 1);
+      tc::mbar_init(tempty(a), 2 * kEpiWarps);  // one arrival per epilogue warp of either CTA
+    }
+    tc::mbar_init(done, 1);
+    tc::mbar_fence_init();
+    tc::tma_prefetch_map(&map_a);
+    tc::tma_prefetch_map(&map_b);
+  }
+  if (warp == 1) {
+    tc::tmem_alloc_pair(tc::smem_u32(tmem_slot), kTmemCols);
+    tc::tmem_relinquish_pair();
+  }
+  tc::fence_before_sync();
+  tc::cluster_sync();  // barriers initialised and TMEM allocated in both CTAs
+  tc::fence_after_sync();
+  const uint32_t tmem = *tmem_slot;
+  auto full_even = [&](int s) { return tc::map_shared(full(s), 0); };
+  auto tempty_even = [&](int a) { return tc::map_shared(tempty(a), 0); };
+  const int row_tiles = (g.m + 2 * kBM - 1) / (2 * kBM);
+  const int tiles = row_tiles * g.n_tiles;
+
+  if (warp == 0) {
+    // ---------------------------------------------------------------- TMA producer (both CTAs)
+    int stage = 0;
+    uint32_t phase = 0, filled = 0, last_parity = 0;
+    bool ok = true;
+    for (int tile = cluster; tile < tiles && ok; tile += clusters) {
+      const int rb = tile / g.n_tiles, nt = tile - rb * g.n_tiles;
+      for (int kb = 0; kb < g.kblocks; ++kb) {
+        if (!tc::mbar_wait_warp(empty(stage), phase ^ 1u)) {
+          ok = false;
+          break;
+        }
+        if (lane == 0) {
+          const uint32_t bar = full_even(stage);
+          if (leader) tc::mbar_expect_tx(full(stage), kTx);
+          if (kMode != kModeProject)
+            tc::tma_load_2d_pair(sa(stage), &map_a, kb * kBK, rb * 2 * kBM + (int)rank * kBM, bar);
+          tc::tma_load_2d_pair(sb(stage), &map_b, kb * kBK, nt * kBN + (int)rank * 128, bar);
+        }
+        __syncwarp();
+        filled |= 1u << stage;
+        last_parity = (last_parity & ~(1u << stage)) | (phase << stage);
+        if (++stage == kStagesP) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+    }
+    if (!ok && lane == 0) flag_error(g, 1);
+    // every load of either CTA lands on the even CTA's barriers: it waits for
+    // them before the final cluster barrier, so no CTA exits with loads in flight
+    if (leader)
+      for (int s = 0; s < kStagesP; ++s)
+        if (filled & (1u << s)) tc::mbar_wait_warp(full(s), (last_parity >> s) & 1u);
+  } else if (warp == 1) {
+    // ---------------------------------------------------------------- MMA issuer (even CTA)
+    if (leader) {
+      int stage = 0, acc = 0;
+      uint32_t phase = 0, acc_phase = 0;
+      bool ok = true;
+      for (int tile = cluster; tile < tiles && ok; tile += clusters) {
+        if (!tc::mbar_wait_warp(tempty(acc), acc_phase ^ 1u)) {
+          ok = false;
+          break;
+        }
+        tc::fence_after_sync();
+        const uint32_t d = tmem + (uint32_t)(acc * kBN);
+        for (int kb = 0; kb < g.kblocks; ++kb) {
+          if (!tc::mbar_wait_warp(full(stage), phase)) {
+            ok = false;
+            break;
+          }
+          tc::fence_after_sync();
+          if (lane == 0) {
+            const uint64_t da = tc::sw128_desc(sa(stage)), db = tc::sw128_desc(sb(stage));
+#pragma unroll
+            for (int k = 0; k < kBK / 16; ++k)
+              tc::mma_bf16_pair(d, da + 2u * k, db + 2u * k, kIdescPair, (kb | k) != 0);
+            tc::mma_commit_pair(empty(stage), 0x3);  // both CTAs' stage is free once these MMAs read it
+          }
+          __syncwarp();
+          if (++stage == kStagesP) {
+            stage = 0;
+            phase ^= 1u;
+          }
+        }
+        if (!ok) break;
+        if (lane == 0) tc::mma_commit_pair(tfull(acc), 0x3);
+        __syncwarp();
+        acc ^= 1;
+        if (acc == 0) acc_phase ^= 1u;
+      }
+      if (!ok && lane == 0) flag_error(g, 2);
+      if (lane == 0) tc::mma_commit_pair(done, 0x3);
+      __syncwarp();
+    }
+    tc::mbar_wait_warp(done, 0);  // every pair MMA has completed (both CTAs' TMEM)
+  } else if (kMode == kModeProject && warp >= 2 + kEpiWarps) {
+    // ---------------------------------------------------------------- A copiers (projector mode)
+    const int r = (int)threadIdx.x - 32 * (2 + kEpiWarps);
+    int stage = 0, pending = 0;
+    uint32_t phase = 0;
+    bool ok = true;
+    for (int tile = cluster; tile < tiles && ok; tile += clusters) {
+      const int rb = tile / g.n_tiles;
+      const long long src = kept_source_row(g, (long long)rb * 2 * kBM + (long long)rank * kBM + r);
+      const uint16_t *srow = g.gx + (src >= 0 ? src : 0) * g.k;
+      for (int kb = 0; kb < g.kblocks; ++kb) {
+        if (!tc::mbar_wait_warp(empty(stage), phase ^ 1u)) {
+          ok = false;
+          break;
+        }
+        const uint32_t dst = sa(stage) + (uint32_t)(r * 128);
+#pragma unroll
+        for (int c = 0; c < 8; ++c) {
+          const int col = kb * kBK + c * 8;
+          const bool in = src >= 0 && col < g.k;
+          cp_async16(dst + (uint32_t)((c ^ (r & 7)) << 4), in ? srow + col : g.gx, in ? 16u : 0u);
+        }
+        cp_async_commit();
+        if (++pending > kCopyLag) {
+          cp_async_wait<kCopyLag>();
+          fence_proxy_async();
+          tc::mbar_arrive_cluster(full_even((stage - kCopyLag + kStagesP) % kStagesP));
+          --pending;
+        }
+        if (++stage == kStagesP) {
+          stage = 0;
+          phase ^= 1u;
+        }
+      }
+    }
+    if (!ok && lane == 0) flag_error(g, 8);
+    cp_async_wait<0>();
+    fence_proxy_async();
+    for (int i = pending; i > 0; --i) tc::mbar_arrive_cluster(full_even((stage - i + kStagesP) % kStagesP));
+  } else {
+    // ---------------------------------------------------------------- epilogue (both CTAs)
+    const int q = warp & 3;
+    const int half = (warp - 2) >> 2;
+    int acc = 0;
+    uint32_t acc_phase = 0;
+    for (int tile = cluster; tile < tiles; tile += clusters) {
+      const int rb = tile / g.n_tiles, nt = tile - rb * g.n_tiles;
+      if (!tc::mbar_wait_warp(tfull(acc), acc_phase)) {
+        if (lane == 0) flag_error(g, 4);
+        break;
+      }
+      tc::fence_after_sync();
+      const int rb128 = 2 * rb + (int)rank;  // this CTA's 128-row block
+      const long long row = (long long)rb128 * kBM + 32 * q + lane;
+      const bool row_ok = row < g.m;
+      const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(acc * kBN);
+      Acc sums{{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
+      for (int c = 0; c < kBN / 2 / kChunk; ++c) {
+        const int tcol = half * (kBN / 2) + c * kChunk;
+        const int col0 = nt * kBN + tcol;
+        if (col0 >= g.n) break;
+        float v[16];
+        tc::tmem_ld16(taddr + (uint32_t)tcol, v);
+        if (row_ok) {
+          if (kMode == kModeScore)
+            epi_score(g, row, col0, v, sums);
+          else
+            epi_hidden(g, row, col0, v);
+        }
+      }
+      tc::fence_before_sync();
+      __syncwarp();
+      if (lane == 0) tc::mbar_arrive_cluster(tempty_even(acc));  // this warp is done with the accumulator
+      if (kMode == kModeScore && rb128 * kBM < g.m) publish_rows(g, rb128, nt, half, q, row, row_ok, sums);
+      acc ^= 1;
+      if (acc == 0) acc_phase ^= 1u;
+    }
+  }
+
+  tc::fence_before_sync();
+  tc::cluster_sync();  // neither CTA leaves while the other may still signal its barriers
+  if (warp == 1) {
+    tc::fence_after_sync();
+    tc::tmem_dealloc_pair(tmem, kTmemCols);
+  }
+}
+
 // ---------------------------------------------------------------- host side
 using EncodeTiled = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
@@ -482,15 +745,16 @@ bool make_map(CUtensorMap *map, const void *base, long long rows, long long cols
 
 std::atomic<int> g_gemm_smem_set[64];
 
+std::atomic<int> g_pair_smem_set[64];
+std::atomic<int> g_pair_clusters[64][3];
+
 template <int kMode>
-cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, const GemmArgs &g, cudaStream_t st) {
-  if (g.tiles == 0) return cudaSuccess;
-  int dev = 0;
-  cudaError_t err = cudaGetDevice(&dev);
-  if (err != cudaSuccess) return err;
+cudaError_t launch_single(const CUtensorMap &ma, const CUtensorMap &mb, const GemmArgs &g, cudaStream_t st,
+                          int dev) {
   const int bit = 1 << kMode;
   if (!(g_gemm_smem_set[dev & 63].load() & bit)) {
-    err = cudaFuncSetAttribute(k_mlp_gemm<kMode>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmem);
+    cudaError_t err =
+        cudaFuncSetAttribute(k_mlp_gemm<kMode>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kGemmSmem);
     if (err != cudaSuccess) return err;
     g_gemm_smem_set[dev & 63].fetch_or(bit);
   }
@@ -499,6 +763,55 @@ cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, const Gemm
   const int grid = g.tiles < sms ? g.tiles : sms;
   k_mlp_gemm<kMode><<<grid, gemm_threads(kMode), kGemmSmem, st>>>(ma, mb, g);
   return cudaGetLastError();
+}
+
+template <int kMode>
+cudaError_t launch_pair(const CUtensorMap &ma, const CUtensorMap &mb, const GemmArgs &g, cudaStream_t st, int dev) {
+  const int bit = 1 << kMode;
+  cudaLaunchConfig_t cfg = {};
+  cfg.blockDim = dim3(gemm_threads(kMode));
+  cfg.dynamicSmemBytes = kGemmPSmem;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  if (!(g_pair_smem_set[dev & 63].load() & bit)) {
+    cudaError_t err = cudaFuncSetAttribute(k_mlp_gemm_pair<kMode>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                           (int)kGemmPSmem);
+    if (err != cudaSuccess) return err;
+    int clusters = 0;
+    cfg.gridDim = dim3(2 * 64);
+    err = cudaOccupancyMaxActiveClusters(&clusters, k_mlp_gemm_pair<kMode>, &cfg);
+    if (err != cudaSuccess) return err;
+    if (clusters <= 0) return cudaErrorInvalidConfiguration;
+    g_pair_clusters[dev & 63][kMode].store(clusters);
+    g_pair_smem_set[dev & 63].fetch_or(bit);
+  }
+  const int row_tiles = (g.m + 2 * kBM - 1) / (2 * kBM);
+  const long long tiles = (long long)row_tiles * g.n_tiles;
+  const int max_clusters = g_pair_clusters[dev & 63][kMode].load();
+  const int clusters = tiles < max_clusters ? (int)tiles : max_clusters;
+  cfg.gridDim = dim3(2 * clusters);
+  return cudaLaunchKernelEx(&cfg, k_mlp_gemm_pair<kMode>, ma, mb, g);
+}
+
+// Batches of more than one 128-row block run on SM pairs (2-SM MMA); a
+// single row block on one SM.  The B operand's TMA box follows: 128 rows
+// per CTA in a pair, the whole 256-row tile on one SM.
+inline bool use_pair(int m) { return m > kBM; }
+inline int b_box_rows(int m) { return use_pair(m) ? 128 : kBN; }
+
+template <int kMode>
+cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, const GemmArgs &g, cudaStream_t st) {
+  if (g.tiles == 0) return cudaSuccess;
+  int dev = 0;
+  cudaError_t err = cudaGetDevice(&dev);
+  if (err != cudaSuccess) return err;
+  return use_pair(g.m) ? launch_pair<kMode>(ma, mb, g, st, dev) : launch_single<kMode>(ma, mb, g, st, dev);
 }
 
 bool misaligned16(const void *p) { return p && (reinterpret_cast<uintptr_t>(p) & 15u) != 0; }
@@ -555,7 +868,7 @@ tr_status tr_mlp_hidden(const tr_mlp *m, void *h, int32_t *d_error, void *stream
   g.out = static_cast<uint16_t *>(h);
   g.err = d_error;
   CUtensorMap ma, mb;
-  if (!make_map(&ma, m->x_pre, m->t, m->d, kBM) || !make_map(&mb, m->w1, m->d_hidden, m->d, kBN))
+  if (!make_map(&ma, m->x_pre, m->t, m->d, kBM) || !make_map(&mb, m->w1, m->d_hidden, m->d, b_box_rows(g.m)))
     return TR_ERR_CUDA;
   return launch_gemm<kModeHidden>(ma, mb, g, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TR_OK : TR_ERR_CUDA;
 }
@@ -598,7 +911,7 @@ tr_status tr_mlp_score(const tr_mlp *m, const void *h, void *x_post, void *x, fl
   g.s = s;
   g.err = d_error;
   CUtensorMap ma, mb;
-  if (!make_map(&ma, h, m->t, m->d_hidden, kBM) || !make_map(&mb, m->w2, m->d, m->d_hidden, kBN))
+  if (!make_map(&ma, h, m->t, m->d_hidden, kBM) || !make_map(&mb, m->w2, m->d, m->d_hidden, b_box_rows(g.m)))
     return TR_ERR_CUDA;
   return launch_gemm<kModeScore>(ma, mb, g, st) == cudaSuccess ? TR_OK : TR_ERR_CUDA;
 }
@@ -645,7 +958,7 @@ tr_status tr_project_kept(const tr_tokens *in, const int32_t *d_cu_k, const int3
   g.cu_k = d_cu_k;
   g.idx = idx;
   CUtensorMap mb;
-  if (!make_map(&mb, w, d_out, in->d, kBN)) return TR_ERR_CUDA;
+  if (!make_map(&mb, w, d_out, in->d, b_box_rows(g.m))) return TR_ERR_CUDA;
   return launch_gemm<kModeProject>(mb, mb, g, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TR_OK
                                                                                                  : TR_ERR_CUDA;
 }
