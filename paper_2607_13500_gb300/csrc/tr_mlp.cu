@@ -68,7 +68,11 @@ constexpr int kTmemCols = 2 * kBN;                // two accumulators
 constexpr int kChunk = 16;                        // columns per tcgen05.ld
 constexpr int kPartWords = 10;                    // hi, lo of L1, S2, A, B, P
 constexpr uint32_t kIdesc = tc::idesc_bf16(kBM, kBN);
-constexpr size_t kGemmSmem = (size_t)kStages * kStageBytes + 1024 + 256;
+// Per epilogue warp, a 32-row x 64-column bf16 output block staged for a TMA
+// store (hidden and projector modes), 128-byte rows in the swizzled layout.
+constexpr int kStageOut = 32 * 128;
+constexpr int kStageOutAll = kEpiWarps * kStageOut;  // 32 KiB
+constexpr size_t kGemmSmem = (size_t)kStages * kStageBytes + kStageOutAll + 1024 + 256;
 
 struct GemmArgs {
   int m, n, k;          // C[m, n] = A[m, k] B[n, k]^T
@@ -91,9 +95,6 @@ struct GemmArgs {
 };
 
 __device__ __forceinline__ float bf16_val(uint32_t bits16) { return __uint_as_float(bits16 << 16); }
-__device__ __forceinline__ uint32_t bf16_bits(float v) {  // round to nearest even
-  return static_cast<uint32_t>(__bfloat16_as_ushort(__float2bfloat16_rn(v)));
-}
 
 // erf(z) for z >= 0 by Abramowitz and Stegun, Handbook of Mathematical
 // Functions (1964), formula 7.1.26: 1 - (a1 t + ... + a5 t^5) exp(-z^2) with
@@ -150,50 +151,66 @@ __device__ __forceinline__ void epi_hidden(const GemmArgs &g, long long row, int
   dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
 }
 
+// The 16 columns of x' and of the residual that the score epilogue of one
+// chunk reads, loaded one chunk ahead of their use.
+struct ScoreIn {
+  uint4 p0, p1, r0, r1;
+};
+__device__ __forceinline__ void load_score_in(const GemmArgs &g, long long row, int col0, ScoreIn &in) {
+  const long long base = row * g.n + col0;
+  const uint4 *pp = reinterpret_cast<const uint4 *>(g.x_pre + base);
+  in.p0 = __ldg(pp);
+  in.p1 = __ldg(pp + 1);
+  if (g.resid) {
+    const uint4 *rp = reinterpret_cast<const uint4 *>(g.resid + base);
+    in.r0 = __ldg(rp);
+    in.r1 = __ldg(rp + 1);
+  } else {
+    in.r0 = in.r1 = make_uint4(0u, 0u, 0u, 0u);
+  }
+}
+
 // Score GEMM epilogue for 16 columns of one row: x'' = bf16(acc + b2),
 // x = bf16(resid + x''), both stored; the five sums take the stored values
 // (products and squares of bf16 values are exact in fp32; each term enters
 // its double-float sum through TwoSum).
 __device__ __forceinline__ void epi_score(const GemmArgs &g, long long row, int col0, const float (&v)[16],
-                                          Acc &acc) {
+                                          const ScoreIn &in, Acc &acc) {
   const long long base = row * g.n + col0;
-  const uint4 *pp = reinterpret_cast<const uint4 *>(g.x_pre + base);
-  const uint4 p0 = __ldg(pp), p1 = __ldg(pp + 1);
-  uint4 r0 = make_uint4(0u, 0u, 0u, 0u), r1 = r0;
-  if (g.resid) {
-    const uint4 *rp = reinterpret_cast<const uint4 *>(g.resid + base);
-    r0 = __ldg(rp);
-    r1 = __ldg(rp + 1);
+  const uint32_t pw[8] = {in.p0.x, in.p0.y, in.p0.z, in.p0.w, in.p1.x, in.p1.y, in.p1.z, in.p1.w};
+  const uint32_t rw[8] = {in.r0.x, in.r0.y, in.r0.z, in.r0.w, in.r1.x, in.r1.y, in.r1.z, in.r1.w};
+  float a[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) a[i] = v[i];
+  if (g.bias) {
+    const float4 *bp = reinterpret_cast<const float4 *>(g.bias + col0);
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float4 b = __ldg(bp + i);
+      a[4 * i] += b.x;
+      a[4 * i + 1] += b.y;
+      a[4 * i + 2] += b.z;
+      a[4 * i + 3] += b.w;
+    }
   }
-  const uint32_t pw[8] = {p0.x, p0.y, p0.z, p0.w, p1.x, p1.y, p1.z, p1.w};
-  const uint32_t rw[8] = {r0.x, r0.y, r0.z, r0.w, r1.x, r1.y, r1.z, r1.w};
   uint32_t qo[8], xo[8];
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
-    uint32_t qb[2], xb[2];
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-      const int c = 2 * i + h;
-      float a = v[c];
-      if (g.bias) a += __ldg(g.bias + col0 + c);
-      qb[h] = bf16_bits(a);
-      const float q = bf16_val(qb[h]);                         // x''
-      const float xp = bf16_val(h ? pw[i] >> 16 : pw[i] & 0xffffu);  // x'
-      float xv = q;                                            // x = resid + x'' (or x'')
-      if (g.resid) {
-        xb[h] = bf16_bits(bf16_val(h ? rw[i] >> 16 : rw[i] & 0xffffu) + q);
-        xv = bf16_val(xb[h]);
-      } else {
-        xb[h] = qb[h];
-      }
-      df_add(acc.l1, fabsf(xv));
-      df_add(acc.s2, xv * xv);
-      df_add(acc.a, xp * xp);
-      df_add(acc.b, q * q);
-      df_add(acc.p, xp * q);
-    }
-    qo[i] = qb[0] | (qb[1] << 16);
-    xo[i] = xb[0] | (xb[1] << 16);
+    qo[i] = pack_bf16x2(a[2 * i], a[2 * i + 1]);  // x''
+    const float q0 = bf16_val(qo[i] & 0xffffu), q1 = bf16_val(qo[i] >> 16);
+    xo[i] = g.resid ? pack_bf16x2(bf16_val(rw[i] & 0xffffu) + q0, bf16_val(rw[i] >> 16) + q1) : qo[i];
+    const float x0 = bf16_val(xo[i] & 0xffffu), x1 = bf16_val(xo[i] >> 16);
+    const float p0 = bf16_val(pw[i] & 0xffffu), p1 = bf16_val(pw[i] >> 16);  // x'
+    df_add(acc.l1, fabsf(x0));
+    df_add(acc.l1, fabsf(x1));
+    df_add(acc.s2, x0 * x0);
+    df_add(acc.s2, x1 * x1);
+    df_add(acc.a, p0 * p0);
+    df_add(acc.a, p1 * p1);
+    df_add(acc.b, q0 * q0);
+    df_add(acc.b, q1 * q1);
+    df_add(acc.p, p0 * q0);
+    df_add(acc.p, p1 * q1);
   }
   uint4 *dq = reinterpret_cast<uint4 *>(g.out + base);
   dq[0] = make_uint4(qo[0], qo[1], qo[2], qo[3]);
@@ -201,6 +218,123 @@ __device__ __forceinline__ void epi_score(const GemmArgs &g, long long row, int 
   uint4 *dx = reinterpret_cast<uint4 *>(g.x + base);
   dx[0] = make_uint4(xo[0], xo[1], xo[2], xo[3]);
   dx[1] = make_uint4(xo[4], xo[5], xo[6], xo[7]);
+}
+
+// One accumulator tile's worth of this warp's epilogue: the 8 chunks of 16
+// columns of its column half, each chunk's TMEM load (and, for the score
+// epilogue, its x' and residual loads) issued while the chunk before it is
+// processed.
+// Hidden / projector epilogue of one tile half for this warp: 8 chunks of
+// 16 columns, H = bf16(act(acc + bias)), staged per 64 columns in this
+// warp's 32 x 64 swizzled block (unit u of row r at r * 128 +
+// ((u ^ (r & 7)) << 4): the 32 lanes' 16-byte writes fall in distinct banks)
+// and written by one TMA store per 64 columns, so global memory sees whole
+// 128-byte row segments instead of one 32-byte piece per row and lane.  The
+// next chunk's TMEM load and bias are in flight while a chunk is processed;
+// a block is rewritten only after its previous store has read it.  Rows and
+// columns past the output are computed from zero operands and clipped by
+// the store.
+__device__ __forceinline__ void drain_tile_store(const GemmArgs &g, const CUtensorMap *map_out, uint32_t buf,
+                                                 uint32_t taddr, int half, int nt, long long row0) {
+  constexpr int kChunks = kBN / 2 / kChunk;
+  const int lane = threadIdx.x & 31;
+  const int col_first = nt * kBN + half * (kBN / 2);
+  int chunks = 0;
+  while (chunks < kChunks && col_first + chunks * kChunk < g.n) ++chunks;
+  if (chunks == 0) return;
+  uint32_t cur[16], nxt[16];
+  float4 bc[4], bn[4];
+  auto load_bias = [&](int col0, float4 (&b)[4]) {
+    if (g.bias) {
+      const float4 *bp = reinterpret_cast<const float4 *>(g.bias + col0);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) b[i] = __ldg(bp + i);
+    } else {
+#pragma unroll
+      for (int i = 0; i < 4; ++i) b[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  };
+  tc::tmem_ld16_issue(taddr + (uint32_t)(half * (kBN / 2)), cur);
+  load_bias(col_first, bc);
+  tc::tmem_ld_wait(cur);
+  const uint32_t rowbuf = buf + (uint32_t)(lane * 128);
+  for (int c = 0; c < chunks; ++c) {
+    const int col0 = col_first + c * kChunk;
+    const bool more = c + 1 < chunks;
+    if (more) {
+      tc::tmem_ld16_issue(taddr + (uint32_t)(half * (kBN / 2) + (c + 1) * kChunk), nxt);
+      load_bias(col0 + kChunk, bn);
+    }
+    const float bias[16] = {bc[0].x, bc[0].y, bc[0].z, bc[0].w, bc[1].x, bc[1].y, bc[1].z, bc[1].w,
+                            bc[2].x, bc[2].y, bc[2].z, bc[2].w, bc[3].x, bc[3].y, bc[3].z, bc[3].w};
+    uint32_t w[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      w[i] = pack_bf16x2(activate(__uint_as_float(cur[2 * i]) + bias[2 * i], g.act),
+                         activate(__uint_as_float(cur[2 * i + 1]) + bias[2 * i + 1], g.act));
+    if ((c & 3) == 0 && c > 0) {  // the block's previous store must have read it
+      if (lane == 0) tc::bulk_wait_read();
+      __syncwarp();
+    }
+    const int u = 2 * (c & 3);
+    tc::st_shared_v4(rowbuf + (uint32_t)((u ^ (lane & 7)) << 4), w[0], w[1], w[2], w[3]);
+    tc::st_shared_v4(rowbuf + (uint32_t)(((u + 1) ^ (lane & 7)) << 4), w[4], w[5], w[6], w[7]);
+    if ((c & 3) == 3 || !more) {  // a 64-column block is complete: one TMA store for the warp's 32 rows
+      tc::fence_async_shared();
+      __syncwarp();
+      if (lane == 0 && row0 < g.m) {  // a block wholly past the last row is not stored
+        tc::tma_store_2d(map_out, col_first + 64 * (c >> 2), (int)row0, buf);
+        tc::bulk_commit();
+      }
+    }
+    if (more) {
+      tc::tmem_ld_wait(nxt);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) cur[i] = nxt[i];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) bc[i] = bn[i];
+    }
+  }
+  if (lane == 0) tc::bulk_wait_read();  // the block may be rewritten by the next tile
+  __syncwarp();
+}
+
+template <int kMode>
+__device__ __forceinline__ void drain_tile(const GemmArgs &g, uint32_t taddr, int half, int nt, long long row,
+                                           bool row_ok, Acc &sums) {
+  constexpr int kChunks = kBN / 2 / kChunk;
+  int chunks = 0;  // chunks of this half inside the output (uniform across the warp)
+  while (chunks < kChunks && nt * kBN + half * (kBN / 2) + chunks * kChunk < g.n) ++chunks;
+  if (chunks == 0) return;
+  uint32_t cur[16], nxt[16];
+  ScoreIn in_cur{}, in_nxt{};
+  const int col_first = nt * kBN + half * (kBN / 2);
+  tc::tmem_ld16_issue(taddr + (uint32_t)(half * (kBN / 2)), cur);
+  if (kMode == kModeScore && row_ok) load_score_in(g, row, col_first, in_cur);
+  tc::tmem_ld_wait(cur);
+  for (int c = 0; c < chunks; ++c) {
+    const int col0 = col_first + c * kChunk;
+    const bool more = c + 1 < chunks;
+    if (more) {
+      tc::tmem_ld16_issue(taddr + (uint32_t)(half * (kBN / 2) + (c + 1) * kChunk), nxt);
+      if (kMode == kModeScore && row_ok) load_score_in(g, row, col0 + kChunk, in_nxt);
+    }
+    if (row_ok) {
+      float v[16];
+#pragma unroll
+      for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(cur[i]);
+      if (kMode == kModeScore)
+        epi_score(g, row, col0, v, in_cur, sums);
+      else
+        epi_hidden(g, row, col0, v);
+    }
+    if (more) {
+      tc::tmem_ld_wait(nxt);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) cur[i] = nxt[i];
+      in_cur = in_nxt;
+    }
+  }
 }
 
 // This warp's 32 rows of one tile half are done: publish their partial
@@ -273,12 +407,13 @@ __device__ __forceinline__ long long kept_source_row(const GemmArgs &g, long lon
 template <int kMode>
 __global__ void __launch_bounds__(gemm_threads(kMode), 1)
     k_mlp_gemm(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
-               const GemmArgs g) {
+               const __grid_constant__ CUtensorMap map_out, const GemmArgs g) {
   extern __shared__ unsigned char smem_raw[];
   // stage tiles at a 1024-byte boundary (the swizzle atom), barriers after them
   unsigned char *smem = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                           ~static_cast<uintptr_t>(1023));
-  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)kStages * kStageBytes);
+  const uint32_t out_stage = tc::smem_u32(smem + (size_t)kStages * kStageBytes);  // epilogue staging
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)kStages * kStageBytes + kStageOutAll);
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * kStages + 5);
   const uint32_t sbase = tc::smem_u32(smem);
   const uint32_t b0 = tc::smem_u32(bars);
@@ -446,25 +581,18 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
       const bool row_ok = row < g.m;
       const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(acc * kBN);
       Acc sums{{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
-      for (int c = 0; c < kBN / 2 / kChunk; ++c) {
-        const int tcol = half * (kBN / 2) + c * kChunk;  // column within the tile
-        const int col0 = nt * kBN + tcol;
-        if (col0 >= g.n) break;  // uniform across the warp
-        float v[16];
-        tc::tmem_ld16(taddr + (uint32_t)tcol, v);
-        if (row_ok) {
-          if (kMode == kModeScore)
-            epi_score(g, row, col0, v, sums);
-          else
-            epi_hidden(g, row, col0, v);
-        }
-      }
+      if (kMode == kModeScore)
+        drain_tile<kMode>(g, taddr, half, nt, row, row_ok, sums);
+      else
+        drain_tile_store(g, &map_out, out_stage + (uint32_t)((warp - 2) * kStageOut), taddr, half, nt,
+                         row - lane);
       tc::fence_before_sync();
       tc::mbar_arrive(tempty(acc));  // the MMA warp may refill this accumulator
       if (kMode == kModeScore) publish_rows(g, rb, nt, half, q, row, row_ok, sums);
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1u;
     }
+    if (kMode != kModeScore && lane == 0) tc::bulk_wait();  // this warp's output stores have completed
   }
 
   tc::fence_before_sync();
@@ -492,16 +620,17 @@ constexpr int kStagesP = 6;
 constexpr int kHalfTile = 128 * kBK * 2;          // 128 rows of a k-block (A or B)
 constexpr int kStagePBytes = 2 * kHalfTile;       // this CTA's A rows + B rows
 constexpr uint32_t kIdescPair = tc::idesc_bf16(2 * kBM, kBN);
-constexpr size_t kGemmPSmem = (size_t)kStagesP * kStagePBytes + 1024 + 256;
+constexpr size_t kGemmPSmem = (size_t)kStagesP * kStagePBytes + kStageOutAll + 1024 + 256;
 
 template <int kMode>
 __global__ void __launch_bounds__(gemm_threads(kMode), 1)
     k_mlp_gemm_pair(const __grid_constant__ CUtensorMap map_a, const __grid_constant__ CUtensorMap map_b,
-                    const GemmArgs g) {
+                    const __grid_constant__ CUtensorMap map_out, const GemmArgs g) {
   extern __shared__ unsigned char smem_raw[];
   unsigned char *smem = reinterpret_cast<unsigned char *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                           ~static_cast<uintptr_t>(1023));
-  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)kStagesP * kStagePBytes);
+  const uint32_t out_stage = tc::smem_u32(smem + (size_t)kStagesP * kStagePBytes);  // epilogue staging
+  uint64_t *bars = reinterpret_cast<uint64_t *>(smem + (size_t)kStagesP * kStagePBytes + kStageOutAll);
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(bars + 2 * kStagesP + 5);
   const uint32_t sbase = tc::smem_u32(smem);
   const uint32_t b0 = tc::smem_u32(bars);
@@ -680,19 +809,11 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
       const bool row_ok = row < g.m;
       const uint32_t taddr = tmem + ((uint32_t)(32 * q) << 16) + (uint32_t)(acc * kBN);
       Acc sums{{0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}, {0.f, 0.f}};
-      for (int c = 0; c < kBN / 2 / kChunk; ++c) {
-        const int tcol = half * (kBN / 2) + c * kChunk;
-        const int col0 = nt * kBN + tcol;
-        if (col0 >= g.n) break;
-        float v[16];
-        tc::tmem_ld16(taddr + (uint32_t)tcol, v);
-        if (row_ok) {
-          if (kMode == kModeScore)
-            epi_score(g, row, col0, v, sums);
-          else
-            epi_hidden(g, row, col0, v);
-        }
-      }
+      if (kMode == kModeScore)
+        drain_tile<kMode>(g, taddr, half, nt, row, row_ok, sums);
+      else
+        drain_tile_store(g, &map_out, out_stage + (uint32_t)((warp - 2) * kStageOut), taddr, half, nt,
+                         row - lane);
       tc::fence_before_sync();
       __syncwarp();
       if (lane == 0) tc::mbar_arrive_cluster(tempty_even(acc));  // this warp is done with the accumulator
@@ -700,6 +821,7 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
       acc ^= 1;
       if (acc == 0) acc_phase ^= 1u;
     }
+    if (kMode != kModeScore && lane == 0) tc::bulk_wait();  // this warp's output stores have completed
   }
 
   tc::fence_before_sync();
@@ -749,8 +871,8 @@ std::atomic<int> g_pair_smem_set[64];
 std::atomic<int> g_pair_clusters[64][3];
 
 template <int kMode>
-cudaError_t launch_single(const CUtensorMap &ma, const CUtensorMap &mb, const GemmArgs &g, cudaStream_t st,
-                          int dev) {
+cudaError_t launch_single(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &mo, const GemmArgs &g,
+                          cudaStream_t st, int dev) {
   const int bit = 1 << kMode;
   if (!(g_gemm_smem_set[dev & 63].load() & bit)) {
     cudaError_t err =
@@ -761,12 +883,13 @@ cudaError_t launch_single(const CUtensorMap &ma, const CUtensorMap &mb, const Ge
   const int sms = sm_count();
   if (sms <= 0) return cudaErrorInvalidDevice;
   const int grid = g.tiles < sms ? g.tiles : sms;
-  k_mlp_gemm<kMode><<<grid, gemm_threads(kMode), kGemmSmem, st>>>(ma, mb, g);
+  k_mlp_gemm<kMode><<<grid, gemm_threads(kMode), kGemmSmem, st>>>(ma, mb, mo, g);
   return cudaGetLastError();
 }
 
 template <int kMode>
-cudaError_t launch_pair(const CUtensorMap &ma, const CUtensorMap &mb, const GemmArgs &g, cudaStream_t st, int dev) {
+cudaError_t launch_pair(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &mo, const GemmArgs &g,
+                        cudaStream_t st, int dev) {
   const int bit = 1 << kMode;
   cudaLaunchConfig_t cfg = {};
   cfg.blockDim = dim3(gemm_threads(kMode));
@@ -796,7 +919,7 @@ cudaError_t launch_pair(const CUtensorMap &ma, const CUtensorMap &mb, const Gemm
   const int max_clusters = g_pair_clusters[dev & 63][kMode].load();
   const int clusters = tiles < max_clusters ? (int)tiles : max_clusters;
   cfg.gridDim = dim3(2 * clusters);
-  return cudaLaunchKernelEx(&cfg, k_mlp_gemm_pair<kMode>, ma, mb, g);
+  return cudaLaunchKernelEx(&cfg, k_mlp_gemm_pair<kMode>, ma, mb, mo, g);
 }
 
 // Batches of more than one 128-row block run on SM pairs (2-SM MMA); a
@@ -806,12 +929,13 @@ inline bool use_pair(int m) { return m > kBM; }
 inline int b_box_rows(int m) { return use_pair(m) ? 128 : kBN; }
 
 template <int kMode>
-cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, const GemmArgs &g, cudaStream_t st) {
+cudaError_t launch_gemm(const CUtensorMap &ma, const CUtensorMap &mb, const CUtensorMap &mo, const GemmArgs &g,
+                        cudaStream_t st) {
   if (g.tiles == 0) return cudaSuccess;
   int dev = 0;
   cudaError_t err = cudaGetDevice(&dev);
   if (err != cudaSuccess) return err;
-  return use_pair(g.m) ? launch_pair<kMode>(ma, mb, g, st, dev) : launch_single<kMode>(ma, mb, g, st, dev);
+  return use_pair(g.m) ? launch_pair<kMode>(ma, mb, mo, g, st, dev) : launch_single<kMode>(ma, mb, mo, g, st, dev);
 }
 
 bool misaligned16(const void *p) { return p && (reinterpret_cast<uintptr_t>(p) & 15u) != 0; }
@@ -867,10 +991,12 @@ tr_status tr_mlp_hidden(const tr_mlp *m, void *h, int32_t *d_error, void *stream
   g.act = m->act;
   g.out = static_cast<uint16_t *>(h);
   g.err = d_error;
-  CUtensorMap ma, mb;
-  if (!make_map(&ma, m->x_pre, m->t, m->d, kBM) || !make_map(&mb, m->w1, m->d_hidden, m->d, b_box_rows(g.m)))
+  CUtensorMap ma, mb, mo;
+  if (!make_map(&ma, m->x_pre, m->t, m->d, kBM) || !make_map(&mb, m->w1, m->d_hidden, m->d, b_box_rows(g.m)) ||
+      !make_map(&mo, h, m->t, m->d_hidden, 32))
     return TR_ERR_CUDA;
-  return launch_gemm<kModeHidden>(ma, mb, g, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+  return launch_gemm<kModeHidden>(ma, mb, mo, g, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TR_OK
+                                                                                                    : TR_ERR_CUDA;
 }
 
 size_t tr_mlp_workspace_bytes(const tr_mlp *m) {
@@ -913,7 +1039,7 @@ tr_status tr_mlp_score(const tr_mlp *m, const void *h, void *x_post, void *x, fl
   CUtensorMap ma, mb;
   if (!make_map(&ma, h, m->t, m->d_hidden, kBM) || !make_map(&mb, m->w2, m->d, m->d_hidden, b_box_rows(g.m)))
     return TR_ERR_CUDA;
-  return launch_gemm<kModeScore>(ma, mb, g, st) == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+  return launch_gemm<kModeScore>(ma, mb, mb, g, st) == cudaSuccess ? TR_OK : TR_ERR_CUDA;  // no output map
 }
 
 tr_status tr_project_kept(const tr_tokens *in, const int32_t *d_cu_k, const int32_t *idx, int32_t total_k,
@@ -957,10 +1083,10 @@ tr_status tr_project_kept(const tr_tokens *in, const int32_t *d_cu_k, const int3
   g.cu_seqlens = in->cu_seqlens;
   g.cu_k = d_cu_k;
   g.idx = idx;
-  CUtensorMap mb;
-  if (!make_map(&mb, w, d_out, in->d, b_box_rows(g.m))) return TR_ERR_CUDA;
-  return launch_gemm<kModeProject>(mb, mb, g, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TR_OK
-                                                                                                 : TR_ERR_CUDA;
+  CUtensorMap mb, mo;
+  if (!make_map(&mb, w, d_out, in->d, b_box_rows(g.m)) || !make_map(&mo, z, total_k, d_out, 32)) return TR_ERR_CUDA;
+  return launch_gemm<kModeProject>(mb, mb, mo, g, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TR_OK
+                                                                                                     : TR_ERR_CUDA;
 }
 
 }  // extern "C"
