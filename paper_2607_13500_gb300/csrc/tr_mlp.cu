@@ -31,10 +31,12 @@
 // the first projector layer reads X* = X_imp union X_div (Eq. 7) straight
 // from x without a gathered copy.  Four more warps (10-13) move those rows
 // with 16-byte cp.async copies into the 128-byte-swizzled layout TMA would
-// have written (chunk c of row r at r * 128 + ((c ^ (r & 7)) << 4)); a
-// copier waits for its copies of a stage, fences them into the async proxy
-// the tensor cores read through, and arrives on the stage's barrier, two
-// stages behind its issue so that copies stay in flight.
+// have written (chunk c of row r at r * 128 + ((c ^ (r & 7)) << 4)), eight
+// threads to a row so that each warp copy reads whole 128-byte segments; a
+// copier waits for its copies of a stage and fences them into the async
+// proxy the tensor cores read through, and once its whole warp has, one lane
+// arrives on the stage's barrier -- some stages behind the issue, so that
+// copies stay in flight.
 //
 // The epilogue of tile i overlaps the main loop of tile i + 1 (two TMEM
 // accumulators).  A row's sums over its 2 n_tiles column halves are
@@ -63,7 +65,12 @@ constexpr int kEpiWarps = 8;                      // two warpgroups: column halv
 enum { kModeHidden = 0, kModeScore = 1, kModeProject = 2 };
 // producer, MMA issuer, epilogue (+ the four A copiers of the projector mode)
 __host__ __device__ constexpr int gemm_threads(int mode) { return 64 + 32 * kEpiWarps + (mode == 2 ? 128 : 0); }
-constexpr int kCopyLag = 2;                       // stages a copier keeps in flight before it signals
+// Stages a copier keeps in flight before it signals the oldest: two fewer
+// than the ring holds (a copier issues stage s + lag only after the MMAs have
+// released that slot, i.e. consumed stage s + lag - stages < s, which it has
+// already signalled).
+constexpr int kCopyLag = 2;     // one SM: 4-stage ring
+constexpr int kCopyLagP = 4;    // SM pair: 6-stage ring
 constexpr int kTmemCols = 2 * kBN;                // two accumulators
 constexpr int kChunk = 16;                        // columns per tcgen05.ld
 constexpr int kPartWords = 10;                    // hi, lo of L1, S2, A, B, P
@@ -428,7 +435,7 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      tc::mbar_init(full(s), kMode == kModeProject ? 1 + 128 : 1);  // + the copiers' arrivals
+      tc::mbar_init(full(s), kMode == kModeProject ? 1 + 4 : 1);  // + one arrival per copier warp
       tc::mbar_init(empty(s), 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -527,31 +534,35 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
     tc::mbar_wait_warp(done, 0);
   } else if (kMode == kModeProject && warp >= 2 + kEpiWarps) {
     // ---------------------------------------------------------------- A copiers (projector mode)
-    const int r = (int)threadIdx.x - 32 * (2 + kEpiWarps);  // tile row of this thread
+    const int t = (int)threadIdx.x - 32 * (2 + kEpiWarps);
+    const int c = t & 7;  // this thread's 16-byte unit of each row's 128-byte k-block segment
     int stage = 0, pending = 0;  // stages copied into but not yet signalled: stage - pending ... stage - 1
     uint32_t phase = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < g.tiles && ok; tile += gridDim.x) {
       const int rb = tile / g.n_tiles;
-      const long long src = kept_source_row(g, (long long)rb * kBM + r);
-      const uint16_t *srow = g.gx + (src >= 0 ? src : 0) * g.k;
+      long long src[8];  // rows (t >> 3) + 16 i of the tile: 8 threads per row, whole 128-byte segments per warp
+#pragma unroll
+      for (int i = 0; i < 8; ++i) src[i] = kept_source_row(g, (long long)rb * kBM + (t >> 3) + 16 * i);
       for (int kb = 0; kb < g.kblocks; ++kb) {
         if (!tc::mbar_wait_warp(empty(stage), phase ^ 1u)) {
           ok = false;
           break;
         }
-        const uint32_t dst = sa(stage) + (uint32_t)(r * 128);
+        const int col = kb * kBK + c * 8;
 #pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          const int col = kb * kBK + c * 8;
-          const bool in = src >= 0 && col < g.k;
-          cp_async16(dst + (uint32_t)((c ^ (r & 7)) << 4), in ? srow + col : g.gx, in ? 16u : 0u);
+        for (int i = 0; i < 8; ++i) {
+          const int r = (t >> 3) + 16 * i;
+          const bool in = src[i] >= 0 && col < g.k;
+          cp_async16(sa(stage) + (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4)), in ? g.gx + src[i] * g.k + col : g.gx,
+                     in ? 16u : 0u);
         }
         cp_async_commit();
         if (++pending > kCopyLag) {  // the copies of the stage issued kCopyLag stages ago are complete
           cp_async_wait<kCopyLag>();
           fence_proxy_async();
-          tc::mbar_arrive(full((stage - kCopyLag + kStages) % kStages));
+          __syncwarp();  // the warp's copies of that stage are complete and fenced: one arrival
+          if (lane == 0) tc::mbar_arrive(full((stage - kCopyLag + kStages) % kStages));
           --pending;
         }
         if (++stage == kStages) {
@@ -563,7 +574,9 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
     if (!ok && lane == 0) flag_error(g, 8);
     cp_async_wait<0>();
     fence_proxy_async();
-    for (int i = pending; i > 0; --i) tc::mbar_arrive(full((stage - i + kStages) % kStages));
+    __syncwarp();
+    if (lane == 0)
+      for (int i = pending; i > 0; --i) tc::mbar_arrive(full((stage - i + kStages) % kStages));
   } else {
     // ---------------------------------------------------------------- epilogue
     const int q = warp & 3;            // TMEM lane quadrant this warp may read
@@ -617,6 +630,7 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
 // brings 32 KiB of operands for a 128 x 256 x 64 product, against 48 KiB on
 // one SM, so six stages in flight hide the load latency that four did not.
 constexpr int kStagesP = 6;
+static_assert(kCopyLagP < kStagesP && kCopyLag < kStages, "a copier must signal a stage before it needs its slot again");
 constexpr int kHalfTile = 128 * kBK * 2;          // 128 rows of a k-block (A or B)
 constexpr int kStagePBytes = 2 * kHalfTile;       // this CTA's A rows + B rows
 constexpr uint32_t kIdescPair = tc::idesc_bf16(2 * kBM, kBN);
@@ -650,7 +664,7 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
   constexpr uint32_t kTx = kMode == kModeProject ? 2 * kHalfTile : 2 * kStagePBytes;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStagesP; ++s) {
-      tc::mbar_init(full(s), kMode == kModeProject ? 1 + 2 * 128 : 1);  // + both CTAs' A copiers
+      tc::mbar_init(full(s), kMode == kModeProject ? 1 + 2 * 4 : 1);  // + both CTAs' copier warps
       tc::mbar_init(empty(s), 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -754,31 +768,36 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
     tc::mbar_wait_warp(done, 0);  // every pair MMA has completed (both CTAs' TMEM)
   } else if (kMode == kModeProject && warp >= 2 + kEpiWarps) {
     // ---------------------------------------------------------------- A copiers (projector mode)
-    const int r = (int)threadIdx.x - 32 * (2 + kEpiWarps);
+    const int t = (int)threadIdx.x - 32 * (2 + kEpiWarps);
+    const int c = t & 7;  // as in the one-SM kernel: 8 threads per row
     int stage = 0, pending = 0;
     uint32_t phase = 0;
     bool ok = true;
     for (int tile = cluster; tile < tiles && ok; tile += clusters) {
       const int rb = tile / g.n_tiles;
-      const long long src = kept_source_row(g, (long long)rb * 2 * kBM + (long long)rank * kBM + r);
-      const uint16_t *srow = g.gx + (src >= 0 ? src : 0) * g.k;
+      long long src[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+        src[i] = kept_source_row(g, (long long)rb * 2 * kBM + (long long)rank * kBM + (t >> 3) + 16 * i);
       for (int kb = 0; kb < g.kblocks; ++kb) {
         if (!tc::mbar_wait_warp(empty(stage), phase ^ 1u)) {
           ok = false;
           break;
         }
-        const uint32_t dst = sa(stage) + (uint32_t)(r * 128);
+        const int col = kb * kBK + c * 8;
 #pragma unroll
-        for (int c = 0; c < 8; ++c) {
-          const int col = kb * kBK + c * 8;
-          const bool in = src >= 0 && col < g.k;
-          cp_async16(dst + (uint32_t)((c ^ (r & 7)) << 4), in ? srow + col : g.gx, in ? 16u : 0u);
+        for (int i = 0; i < 8; ++i) {
+          const int r = (t >> 3) + 16 * i;
+          const bool in = src[i] >= 0 && col < g.k;
+          cp_async16(sa(stage) + (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4)), in ? g.gx + src[i] * g.k + col : g.gx,
+                     in ? 16u : 0u);
         }
         cp_async_commit();
-        if (++pending > kCopyLag) {
-          cp_async_wait<kCopyLag>();
+        if (++pending > kCopyLagP) {
+          cp_async_wait<kCopyLagP>();
           fence_proxy_async();
-          tc::mbar_arrive_cluster(full_even((stage - kCopyLag + kStagesP) % kStagesP));
+          __syncwarp();
+          if (lane == 0) tc::mbar_arrive_cluster(full_even((stage - kCopyLagP + kStagesP) % kStagesP));
           --pending;
         }
         if (++stage == kStagesP) {
@@ -790,7 +809,9 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
     if (!ok && lane == 0) flag_error(g, 8);
     cp_async_wait<0>();
     fence_proxy_async();
-    for (int i = pending; i > 0; --i) tc::mbar_arrive_cluster(full_even((stage - i + kStagesP) % kStagesP));
+    __syncwarp();
+    if (lane == 0)
+      for (int i = pending; i > 0; --i) tc::mbar_arrive_cluster(full_even((stage - i + kStagesP) % kStagesP));
   } else {
     // ---------------------------------------------------------------- epilogue (both CTAs)
     const int q = warp & 3;
