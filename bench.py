@@ -81,6 +81,9 @@ def _args():
                     help="pipeline steps timed for each workload of the per_config block (0: no per_config block)")
     ap.add_argument("--config-cpu-seconds", type=float, default=3.0,
                     help="CPU oracle seconds per per_config workload")
+    ap.add_argument("--mlp-only", action="store_true",
+                    help="time only the fused encoder-MLP path (clip_mlp576; --batch sets the images, --steps "
+                         "the timed repetitions) and print its entry")
     a = ap.parse_args()
     if a.warmup < 3:
         ap.error("--warmup must be at least 3")
@@ -625,7 +628,7 @@ def _bf16_peak():
         return 1900.0, 1700.0, "fallback"
 
 
-def measure_mlp(args, dev, altr, reps=20):
+def measure_mlp(args, dev, altr, reps=20, batch=None):
     """The vision encoder's final-layer MLP with the scoring fused into its
     second GEMM (Eq. 5, Section IV-B), then the selection, the gather and
     the projector's first layer on the kept tokens read by index, on the
@@ -633,7 +636,7 @@ def measure_mlp(args, dev, altr, reps=20):
     4096, K = 192.  Each kernel timed with CUDA events on the current stream
     (median of `reps` steps, inputs larger than L2); beside it, the unfused
     route through the same library (cuBLAS MLP, tr_score pass) for context."""
-    w = synth.make_mlp("clip_mlp576", seed=args.seed, device=dev)
+    w = synth.make_mlp("clip_mlp576", seed=args.seed, device=dev, **({"batch": batch} if batch else {}))
     t, d, dh = w.total, w.x_pre.shape[1], w.w1.shape[0]
     wp, bp = synth.make_projector(d, w.d_proj, seed=args.seed, device=dev)
     budget = altr.budgets(w.seqlens, k=w.k)
@@ -788,11 +791,23 @@ def run_ours(args, world, rank, local):
         torch.distributed.destroy_process_group()
 
 
+def run_mlp_only(args):
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    from paper_2607_13500_gb300 import _build
+    _build.build()
+    import paper_2607_13500_gb300 as altr
+    print(json.dumps({"mlp_fused": measure_mlp(args, dev, altr, reps=args.steps, batch=args.batch)}), flush=True)
+
+
 def main():
     args = _args()
     world, rank, local = _dist()
     if args.impl == "reference":
         run_reference(args, world, rank)
+        return
+    if args.mlp_only:
+        run_mlp_only(args)
         return
     run_ours(args, world, rank, local)
 

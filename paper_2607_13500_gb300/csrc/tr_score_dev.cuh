@@ -218,7 +218,8 @@ __device__ __forceinline__ void accumulate_round(const uint4 *__restrict__ rx, c
 // Partial sums of chunks [c0, c1) of one row, read straight from global
 // memory in rounds of kB chunks per lane and stream.  When the row's chunks
 // are a multiple of 32 (every lane has the same count) the last round is cut
-// to the chunks that remain (6, 4 or 2 per lane), so no lane works on padding.
+// to the chunks that remain (6, 4 or 2 per lane, fewer than a full round), so
+// no lane works on padding.
 template <int kDt>
 __device__ __forceinline__ void accumulate_global(const uint4 *__restrict__ rx, const uint4 *__restrict__ rp,
                                                   const uint4 *__restrict__ rq, int c0, int c1, Acc &acc,
@@ -230,9 +231,9 @@ __device__ __forceinline__ void accumulate_global(const uint4 *__restrict__ rx, 
   for (; base + 32 * kB <= c1; base += 32 * kB) accumulate_round<kDt, kB, false>(rx, rp, rq, base, c1, acc, acc2, lane);
   const int rest = c1 - base;
   if (rest > 0) {
-    if (kB == 8 && rest == 32 * 6)
+    if (kB > 6 && rest == 32 * 6)
       accumulate_round<kDt, 6, false>(rx, rp, rq, base, c1, acc, acc2, lane);
-    else if (kB == 8 && rest == 32 * 4)
+    else if (kB > 4 && rest == 32 * 4)
       accumulate_round<kDt, 4, false>(rx, rp, rq, base, c1, acc, acc2, lane);
     else if (rest == 32 * 2)
       accumulate_round<kDt, 2, false>(rx, rp, rq, base, c1, acc, acc2, lane);
