@@ -316,7 +316,7 @@ def run_reference(args, world, rank):
 # ---------------------------------------------------------------- traffic from the committed ncu summary
 def _score_source_hash():
     h = hashlib.sha256()
-    for f in ("tr_score.cu", "tr_score_dev.cuh", "tr_df.cuh", "tr_internal.cuh"):
+    for f in ("tr_score.cu", "tr_score_dev.cuh", "tr_record.cuh", "tr_df.cuh", "tr_internal.cuh"):
         h.update(open(os.path.join(ROOT, "paper_2607_13500_gb300", "csrc", f), "rb").read())
     return h.hexdigest()[:16]
 
