@@ -42,6 +42,10 @@ struct ExactRec {
   uint32_t flags_l;  // kRecNonFiniteX | kRecOverflowL, valid once L1, S2 are filled
   uint32_t flags_s;  // kRecNonFiniteS | kRecOverflowS, valid once P, A, B are filled
   uint32_t pad;
+  // The keys R and s recomputed in double-float from error-free sums
+  // (hi + lo each; see the select kernel's double-float tier), within the
+  // Bounds::df_* bounds of the true keys.
+  float r_hi, r_lo, s_hi, s_lo;
 };
 static_assert(sizeof(ExactRec) % 16 == 0, "ExactRec records keep 16-byte alignment");
 
@@ -72,6 +76,10 @@ struct Bounds {
   // with directed rounding:  R >= R32 * r_lo,  R <= R32 * r_hi,
   // |s - s32| <= s_abs + s_rel |s32|
   float r_lo, r_hi, s_abs, s_rel;
+  // Keys recomputed by the select kernel's double-float tier (R_df, s_df):
+  // |R_df - R| <= df_r R_df,  |s_df - s| <= df_s_abs + df_s_rel |s_df|
+  // (fp32, rounded outward).
+  float df_r, df_s_abs, df_s_rel;
 };
 
 inline Bounds certification_bounds(int d, int dtype) {
@@ -121,6 +129,29 @@ inline Bounds certification_bounds(int d, int dtype) {
   b.r_hi = (float)((1.0 / (1.0 - b.rho_r)) * (1.0 + 0x1p-22));
   b.s_abs = (float)(b.es_abs * (1.0 + 0x1p-22));
   b.s_rel = (float)(b.es_rel * (1.0 + 0x1p-22));
+  // Double-float tier.  A group of at least 128 threads recomputes a row:
+  // each thread adds its k terms per sum (k = its 16-byte chunks times the
+  // elements per chunk, doubled for fp32, whose squares and products enter as
+  // TwoProd pairs) into a double-float by TwoSum, so hi + (the exact errors)
+  // is the exact partial sum and only the low part's additions round: at most
+  // k^2 u^2 of the sum of |terms| T.  Merging two partials (TwoSum of the high
+  // parts, two low-part additions) rounds by at most (2 j + 1) u^2 T at a
+  // merge whose inputs carry low parts below j u T: the five shuffle levels
+  // inside a warp add at most (10 k + 35) u^2 T, and merging at most 16 warp
+  // partials in turn at most 15 (2 k + 43) u^2 T; in all
+  // (k^2 + 40 k + 680) u^2 T <= 4 (k + 16)^2 u^2 T.  For L1, S2, A, B, T is
+  // the sum itself; for P, T = sum |x'x''| <= sqrt(A B).  Keys then: R from
+  // L1^2 / S2 within (1 + e)^2 / (1 - e) (1 + 2^-40) of the truth, s within
+  // e + |s| (e + 2^-40), the double-float operations' 2^-40 covering their
+  // own roundings.
+  const int per_chunk_df = 16 / elem_bytes(dtype);
+  const double chunks_df = (double)((d / per_chunk_df + 127) / 128);
+  const double k_df = chunks_df * per_chunk_df * (dtype == TR_F32 ? 2.0 : 1.0);
+  const double e_df = 4.0 * (k_df + 16.0) * (k_df + 16.0) * u * u;
+  const double r_df = (1.0 + e_df) * (1.0 + e_df) / (1.0 - e_df) * (1.0 + 0x1p-40) - 1.0;
+  b.df_r = (float)(1.05 * r_df / (1.0 - r_df));  // relative to R_df
+  b.df_s_abs = (float)(1.05 * e_df / (1.0 - e_df) + 0x1p-60);
+  b.df_s_rel = (float)(1.05 * (e_df + 0x1p-40));
   return b;
 }
 

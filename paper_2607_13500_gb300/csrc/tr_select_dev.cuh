@@ -17,10 +17,13 @@
 // suffices to test adjacent pairs.  Only decisions matter: the cut at K1 for
 // Stage I and the neighbourhood of each stride position for Stage II.  The
 // tokens of an uncertain run (a maximal stretch of uncertain cuts around a
-// decision) are recomputed exactly -- their five sums as integers, from the
-// input bits -- and ranked by exact rational comparison (cross products of
-// big integers), ties to the lower index.  Rows whose fp32 sums left the
-// error model (non-finite, overflowed, tiny) are recomputed exactly up front.
+// decision) are recomputed in double-float from error-free sums first; when
+// those keys separate every pair of the run (any run that is not an exact
+// tie, in practice) they rank it.  Otherwise the run is recomputed exactly
+// -- its five sums as integers, from the input bits -- and ranked by exact
+// rational comparison (cross products of big integers), ties to the lower
+// index.  Rows whose fp32 sums left the error model (non-finite, overflowed,
+// tiny) are recomputed exactly up front.
 #pragma once
 
 #include <cfloat>
@@ -41,6 +44,8 @@ enum : uint8_t {
   F_NEEDL = 16,  // exact L1, S2 requested
   F_NEEDS = 32,  // exact P, A, B requested
   F_RUN = 64,    // lies in an uncertain run around a stride position
+  F_DF = 128,    // with F_NEED*: the double-float tier may settle it; alone: it did
+                 // (the row's ExactRec holds the current stage's double-float key)
 };
 
 // ---------------------------------------------------------------- float keys
@@ -112,20 +117,23 @@ __device__ __forceinline__ df::F2 fx_f2(const Fx &x) {
 
 // Keys of a row settled exactly: the same double-float evaluation as the
 // score pass, from the exact sums (truncated to 64 bits), rounded once.
-__device__ __forceinline__ float exact_r_key(const ExactRec &r) {
+// Out of line, like every path that only near-ties and extreme rows take:
+// the select kernel is bound by instruction fetch, so the common path's
+// code is kept compact.
+__device__ __noinline__ float exact_r_key(const ExactRec &r) {
   if (r.flags_l & kRecNonFiniteX) return 0.f;
   if (r.l1.n == 0) return 1.f;
   const Fx l1 = big_fx(r.l1), s2 = big_fx(r.s2);
   const df::F2 L = fx_f2(l1), S = fx_f2(s2);
   return ldexpf(df::round(df::div(df::mul(L, L), S)), 2 * (l1.e + 63) - (s2.e + 63));
 }
-__device__ __forceinline__ float exact_h2(const ExactRec &r) {
+__device__ __noinline__ float exact_h2(const ExactRec &r) {
   if (r.flags_l & kRecNonFiniteX) return -INFINITY;
   if (r.l1.n == 0) return 0.f;
   const Fx l1 = big_fx(r.l1), s2 = big_fx(r.s2);
   return 2.f * fx_log(l1) - fx_log(s2);
 }
-__device__ __forceinline__ float exact_s_key(const ExactRec &r) {
+__device__ __noinline__ float exact_s_key(const ExactRec &r) {
   if (r.flags_s & kRecNonFiniteS) return 2.f;
   if (r.a.n == 0 || r.b.n == 0 || r.p.n == 0) return 0.f;
   const Fx p = big_fx(r.p), a = big_fx(r.a), b = big_fx(r.b);
@@ -613,13 +621,232 @@ __device__ __forceinline__ void exact_row_any(const SelectArgs &a, long long row
   }
 }
 
-// Recomputes the rows whose flags request it and records what is now exact.
-// The pending rows are listed first (a block-wide vote skips everything when
+// ---------------------------------------------------------------- double-float tier
+// A near-tie is almost never an exact tie: the fp32 keys' bound (about
+// 2^-22) is what leaves it open.  Before recomputing a row exactly, the
+// select kernel recomputes its sums with error-free transformations -- every
+// term, exact in fp32 (|x|, and squares and products of bf16 / fp16 values;
+// fp32 squares and products as TwoProd pairs), enters a double-float by
+// TwoSum -- and keeps the keys R and s as double-floats within Bounds::df_*
+// (about 2^-32 relative or tighter).  A run whose rows these keys separate
+// pairwise is ranked by them; one they do not separate (an exact tie, or
+// closer than the bound) is recomputed exactly.  A row whose values could
+// make a term inexact (a non-finite value, a square or product that would
+// leave the normal fp32 range) or whose sums leave [kTiny, kHuge] is not
+// handled here: it goes to the exact path.
+
+// Runs longer than this skip the tier: long runs are exact ties in practice.
+constexpr int kDfRunMax = 32;
+
+// Value of element i of a 16-byte chunk as fp32 (exact for all three types).
+template <int kDt>
+__device__ __forceinline__ void unpack_f32(const uint4 &v, float *out) {
+  const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+  if (kDt == TR_BF16) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      out[2 * i] = __uint_as_float(w[i] << 16);
+      out[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+    }
+  } else if (kDt == TR_F16) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const uint32_t h = (w[i >> 1] >> (16 * (i & 1))) & 0xffffu;
+      const uint32_t sg = (h & 0x8000u) << 16, ex = (h >> 10) & 0x1fu, mant = h & 0x3ffu;
+      float f;
+      if (ex == 0x1fu)
+        f = __uint_as_float(sg | 0x7f800000u | (mant << 13));
+      else if (ex == 0u)
+        f = __uint_as_float(sg | __float_as_uint(__uint2float_rn(mant) * 0x1p-24f));
+      else
+        f = __uint_as_float(sg | ((ex + 112u) << 23) | (mant << 13));
+      out[i] = f;
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) out[i] = __uint_as_float(w[i]);
+  }
+}
+
+// A value whose square (and whose products with other such values) is an
+// exact normal fp32 number or zero: 0, or 2^-50 <= |v| <= 2^50.
+__device__ __forceinline__ bool df_value_ok(float v) {
+  const float m = fabsf(v);
+  return m == 0.f || (m >= 0x1p-50f && m <= 0x1p+50f);
+}
+
+// hi + lo += t with hi + (exact errors) the exact running sum.
+__device__ __forceinline__ void df_term(float &hi, float &lo, float t) {
+  const df::F2 r = df::two_sum(hi, t);
+  hi = r.h;
+  lo = __fadd_rn(lo, r.l);
+}
+__device__ __forceinline__ void df_join(float &hi, float &lo, float h2, float l2) {
+  const df::F2 r = df::two_sum(hi, h2);
+  hi = r.h;
+  lo = __fadd_rn(__fadd_rn(lo, l2), r.l);
+}
+__device__ __forceinline__ void df_warp_join(float &hi, float &lo) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float h2 = __shfl_xor_sync(0xffffffffu, hi, o), l2 = __shfl_xor_sync(0xffffffffu, lo, o);
+    df_join(hi, lo, h2, l2);
+  }
+}
+
+struct PartDf {
+  float h[kWarps * 3], l[kWarps * 3];
+  int ok[4];  // per group: the row's keys were written
+};
+
+// Double-float keys of one row (mode 0: R from L1, S2 of x; mode 1: s from
+// A, B, P of x', x'') by a group of warps; writes rec->r_* or rec->s_* and
+// returns true, uniformly across the group, or false when the row is not
+// eligible (nothing written).
+template <int kDt>
+__device__ bool df_row_block(const SelectArgs &a, long long row, int mode, ExactRec *rec, PartDf &part,
+                             const Group &g) {
+  constexpr int kPer = kDt == TR_F32 ? 4 : 8;  // elements per 16-byte chunk
+  constexpr int kLoads = 4;                    // chunks per stream in flight per thread
+  const int nchunks = a.d / kPer;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  bool ok = true;
+  float h0 = 0.f, l0 = 0.f, h1 = 0.f, l1 = 0.f, h2 = 0.f, l2 = 0.f;
+  const uint4 *p0 = static_cast<const uint4 *>(mode == 0 ? a.x : (a.x_pre ? a.x_pre : a.x)) + row * nchunks;
+  const uint4 *p1 = static_cast<const uint4 *>(a.x_post) + row * nchunks;
+  for (int c0 = g.tid(); c0 < nchunks; c0 += kLoads * g.size) {
+    uint4 u0[kLoads], u1[kLoads];
+#pragma unroll
+    for (int j = 0; j < kLoads; ++j) {  // every load of the round first
+      const int c = c0 + j * g.size;
+      if (c < nchunks) {
+        u0[j] = __ldg(p0 + c);
+        if (mode != 0) u1[j] = __ldg(p1 + c);
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < kLoads; ++j) {
+      if (c0 + j * g.size >= nchunks) break;
+      float v0[kPer], v1[kPer];
+      unpack_f32<kDt>(u0[j], v0);
+      if (mode == 0) {
+#pragma unroll
+        for (int i = 0; i < kPer; ++i) {
+          const float x = v0[i];
+          ok &= df_value_ok(x);
+          df_term(h0, l0, fabsf(x));
+          if (kDt == TR_F32) {
+            const df::F2 q = df::two_prod(x, x);
+            df_term(h1, l1, q.h);
+            l1 = __fadd_rn(l1, q.l);
+          } else {
+            df_term(h1, l1, __fmul_rn(x, x));
+          }
+        }
+      } else {
+        unpack_f32<kDt>(u1[j], v1);
+#pragma unroll
+        for (int i = 0; i < kPer; ++i) {
+          const float p = v0[i], q = v1[i];
+          ok &= df_value_ok(p) && df_value_ok(q);
+          if (kDt == TR_F32) {
+            const df::F2 pp2 = df::two_prod(p, p), qq2 = df::two_prod(q, q), pq2 = df::two_prod(p, q);
+            df_term(h0, l0, pp2.h);
+            l0 = __fadd_rn(l0, pp2.l);
+            df_term(h1, l1, qq2.h);
+            l1 = __fadd_rn(l1, qq2.l);
+            df_term(h2, l2, pq2.h);
+            l2 = __fadd_rn(l2, pq2.l);
+          } else {
+            df_term(h0, l0, __fmul_rn(p, p));
+            df_term(h1, l1, __fmul_rn(q, q));
+            df_term(h2, l2, __fmul_rn(p, q));
+          }
+        }
+      }
+    }
+  }
+  if (!g.all(ok)) return false;
+  df_warp_join(h0, l0);
+  df_warp_join(h1, l1);
+  if (mode != 0) df_warp_join(h2, l2);
+  if (lane == 0) {
+    part.h[warp * 3 + 0] = h0;
+    part.l[warp * 3 + 0] = l0;
+    part.h[warp * 3 + 1] = h1;
+    part.l[warp * 3 + 1] = l1;
+    part.h[warp * 3 + 2] = h2;
+    part.l[warp * 3 + 2] = l2;
+  }
+  g.sync();
+  const int gi = g.bar - 1;
+  if (g.tid() == 0) {
+    // the group's first thread merges the warps' partials in turn
+    const int w0 = g.first >> 5, nw = g.size >> 5;
+    float s[3][2];
+#pragma unroll
+    for (int j = 0; j < 3; ++j) {
+      float h = part.h[w0 * 3 + j], l = part.l[w0 * 3 + j];
+      for (int w = w0 + 1; w < w0 + nw; ++w) df_join(h, l, part.h[w * 3 + j], part.l[w * 3 + j]);
+      const df::F2 n = df::two_sum(h, l);
+      s[j][0] = n.h;
+      s[j][1] = n.l;
+    }
+    bool fine;
+    if (mode == 0) {
+      const df::F2 L1{s[0][0], s[0][1]}, S2{s[1][0], s[1][1]};
+      fine = S2.h >= kTiny && S2.h <= kHuge;
+      if (fine) {
+        const df::F2 r = df::div(df::mul(L1, L1), S2);
+        rec->r_hi = r.h;
+        rec->r_lo = r.l;
+      }
+    } else {
+      const df::F2 A{s[0][0], s[0][1]}, B{s[1][0], s[1][1]}, P{s[2][0], s[2][1]};
+      fine = A.h >= kTiny && A.h <= kHuge && B.h >= kTiny && B.h <= kHuge;
+      if (fine) {
+        const df::F2 v = df::div(P, df::mul(df::sqrt(A), df::sqrt(B)));
+        rec->s_hi = v.h;
+        rec->s_lo = v.l;
+      }
+    }
+    part.ok[gi] = fine ? 1 : 0;
+  }
+  g.sync();
+  return part.ok[gi] != 0;
+}
+
+// +1 / -1 when the double-float keys order row a above / below row b for
+// certain, 0 when their bounds overlap.
+__device__ __forceinline__ int df_cmp_r(const ExactRec &ra, const ExactRec &rb, const Bounds &bd) {
+  const float ah = ra.r_hi, bh = rb.r_hi;
+  const float d = __fadd_rn(__fsub_rn(ah, bh), __fsub_rn(ra.r_lo, rb.r_lo));
+  const float m = bd.df_r * (fabsf(ah) + fabsf(bh));
+  return d > m ? 1 : (d < -m ? -1 : 0);
+}
+__device__ __forceinline__ int df_cmp_s(const ExactRec &ra, const ExactRec &rb, const Bounds &bd) {
+  const float ah = ra.s_hi, bh = rb.s_hi;
+  const float d = __fadd_rn(__fsub_rn(ah, bh), __fsub_rn(ra.s_lo, rb.s_lo));
+  const float m = 2.f * bd.df_s_abs + bd.df_s_rel * (fabsf(ah) + fabsf(bh));
+  return d > m ? 1 : (d < -m ? -1 : 0);
+}
+
+__device__ __forceinline__ bool df_row_any(const SelectArgs &a, long long row, int mode, ExactRec *rec, PartDf &part,
+                                           const Group &g) {
+  return a.dtype == TR_BF16  ? df_row_block<TR_BF16>(a, row, mode, rec, part, g)
+         : a.dtype == TR_F16 ? df_row_block<TR_F16>(a, row, mode, rec, part, g)
+                             : df_row_block<TR_F32>(a, row, mode, rec, part, g);
+}
+
+// Recomputes the rows whose flags request it: by the double-float tier where
+// F_DF allows it and the row qualifies (F_DF stays set), else exactly (F_XL,
+// F_XS).  The pending rows are listed first (a block-wide vote skips everything when
 // none is); then up to four rows at a time are handled by groups of warps.
 constexpr int kPendCap = 512;
 __device__ __noinline__ void refine_listed(const SelectArgs &a, long long off, int n, uint8_t *fl, ExactRec *rec,
                                            const bool primary) {
   __shared__ Part128 part;
+  __shared__ PartDf pdf;
   __shared__ int plist[kPendCap];
   __shared__ int pcount;
   for (;;) {
@@ -644,11 +871,22 @@ __device__ __noinline__ void refine_listed(const SelectArgs &a, long long off, i
         const int row = plist[base + gi];
         const uint8_t fr = fl[row];
         const float *st = a.stats + (off + row) * TR_STATS_WORDS;
-        if (fr & F_NEEDL) exact_row_any(a, off + row, 0, st, rec + row, part, g);
-        if (fr & F_NEEDS) exact_row_any(a, off + row, 1, st, rec + row, part, g);
+        bool dl = false, ds = false;  // settled by the double-float tier
+        if (fr & F_NEEDL) {
+          if (fr & F_DF) dl = df_row_any(a, off + row, 0, rec + row, pdf, g);
+          if (!dl) exact_row_any(a, off + row, 0, st, rec + row, part, g);
+        }
+        if (fr & F_NEEDS) {
+          if (fr & F_DF) ds = df_row_any(a, off + row, 1, rec + row, pdf, g);
+          if (!ds) exact_row_any(a, off + row, 1, st, rec + row, part, g);
+        }
         if (g.tid() == 0) {
-          fl[row] = (uint8_t)((fr & ~(F_NEEDL | F_NEEDS)) | ((fr & F_NEEDL) ? F_XL : 0) | ((fr & F_NEEDS) ? F_XS : 0));
-          if (a.status && primary) atomicAdd(&a.status[2], 1);
+          uint8_t f = (uint8_t)(fr & ~(F_NEEDL | F_NEEDS | F_DF));
+          if (fr & F_NEEDL) f |= dl ? F_DF : F_XL;
+          if (fr & F_NEEDS) f |= ds ? F_DF : F_XS;
+          fl[row] = f;
+          const bool exact = ((fr & F_NEEDL) && !dl) || ((fr & F_NEEDS) && !ds);
+          if (exact && a.status && primary) atomicAdd(&a.status[2], 1);
         }
       }
       __syncthreads();
@@ -839,6 +1077,7 @@ __device__ __noinline__ uint16_t *radix_sort(const uint32_t *key, uint16_t *a, u
   uint32_t *h = hist + warp * 256;
   const unsigned lt = (1u << lane) - 1u;
   if (m < 2) return a;
+#pragma unroll 1
   for (int shift = 0; shift < 32; shift += 8) {
     for (int d = lane; d < 256; d += 32) h[d] = 0u;
     if (tid == 0) skip = 0;
@@ -949,6 +1188,35 @@ __device__ void bitonic_regs(unsigned long long (&v)[E], unsigned long long *scr
       }
     }
   }
+}
+
+// Ascending order of the m <= kSelectThreads rows listed in a by their
+// composite keys (distinct), by counting: thread i places row a[i] at the
+// number of listed rows with a smaller key.  m^2 comparisons spread over m
+// threads and two block barriers: cheaper than a bitonic network for the
+// short lists it takes (see kCountSortMax).  scratch: m 64-bit words,
+// 16-byte aligned.
+constexpr int kCountSortMax = 128;
+__device__ void sort_count(const uint32_t *key, uint16_t *a, int m, unsigned long long *scratch) {
+  const int tid = threadIdx.x;
+  unsigned long long c = 0;
+  if (tid < m) {
+    c = ((unsigned long long)key[a[tid]] << 16) | a[tid];
+    scratch[tid] = c;
+  }
+  if (tid == m && (m & 1)) scratch[m] = ~0ull;  // pads the last pair; never below c
+  __syncthreads();
+  if (tid < m) {
+    const ulonglong2 *s2 = reinterpret_cast<const ulonglong2 *>(scratch);
+    int rank = 0;
+#pragma unroll 4
+    for (int j = 0; j < (m + 1) >> 1; ++j) {
+      const ulonglong2 v = s2[j];
+      rank += (v.x < c) + (v.y < c);
+    }
+    a[rank] = (uint16_t)(c & 0xffffu);  // every read of a[] preceded the barrier
+  }
+  __syncthreads();
 }
 
 template <int E>
@@ -1201,7 +1469,10 @@ __device__ uint16_t *sort_rows(const uint32_t *key, uint16_t *a, uint16_t *b, ui
   unsigned long long *scratch = reinterpret_cast<unsigned long long *>(hist);
   if (m <= kSelectThreads) {
     __syncthreads();  // hist may still be read by the caller's previous step
-    sort_small<1>(key, a, m, scratch);
+    if (m <= kCountSortMax)
+      sort_count(key, a, m, scratch);
+    else
+      sort_small<1>(key, a, m, scratch);
     return a;
   }
   if (uint16_t *o = bucket_sort(key, a, b, m, hist, complemented)) return o;
@@ -1237,6 +1508,7 @@ __device__ uint32_t select_rank(const uint32_t *key, int n, int r, uint32_t *his
   uint32_t pre = 0u, mask = 0u;
   int rr = r;
   __syncthreads();  // hist may still be read by the caller's previous step
+#pragma unroll 1
   for (int shift = 24; shift >= 0; shift -= 8) {
     uint32_t *h = hist + warp * 256;
     for (int d = lane; d < 256; d += 32) h[d] = 0u;
@@ -1430,9 +1702,10 @@ __device__ __forceinline__ void settle_unreliable(const SelectArgs &a, ImageCtx 
 
 }
 
-// 2. Stage I: top-K1 by R (equivalently H2), descending, lower index first.
-//    Marks X_imp (F_IMP) in the flags.
-__device__ __forceinline__ void stage_one(const SelectArgs &a, ImageCtx &c) {
+// Stage I when the K1-th and (K1+1)-th keys are not certainly ordered (t1:
+// the K1-th key).  Out of line: only images with a near-tie at the cut come
+// here.
+__device__ __noinline__ void resolve_cut(const SelectArgs &a, const ImageCtx c, const uint32_t t1) {
   __shared__ int sh_lo, sh_hi;
   const int tid = threadIdx.x;
   const int nthr = blockDim.x;
@@ -1446,6 +1719,141 @@ __device__ __forceinline__ void stage_one(const SelectArgs &a, ImageCtx &c) {
   uint8_t *fl = c.fl;
   ExactRec *rec = c.rec;
   const bool primary = c.primary;
+  const int k1 = c.k1;
+  // Uncertain cut: only the order near it matters.  The rows whose R32
+  // lies within a relative kCutWindow of the K1-th one (far wider than
+  // the certification band) are listed and sorted; when the uncertain
+  // run around the cut ends inside that list, every row with a smaller
+  // key (larger R) precedes it in the full order and is certainly kept,
+  // every row with a larger key certainly not.  Otherwise (or when the
+  // window holds too many rows) all n rows are sorted.
+  const float r1 = unord32(~t1);
+  const uint32_t kw_lo = ~ord32(r1 * (1.f + kCutWindow)), kw_hi = ~ord32(r1 * (1.f - kCutWindow));
+  const bool windowed = isfinite(r1) && r1 > 0.f;  // uniform
+  const uint16_t *ord = nullptr;
+  int base = 0, len = 0;  // ord[q] sits at position base + q of the full order
+  if (windowed) {
+    const int per = (n + nthr - 1) / nthr;
+    const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
+    int c_in = 0, c_lt = 0;
+    for (int i = i0; i < i1; ++i) {
+      const uint32_t k = key[i];
+      c_in += k >= kw_lo && k <= kw_hi;
+      c_lt += k < kw_lo;
+    }
+    // one scan of both counts (each total is at most n < 2^16)
+    int both = 0;
+    int pos = block_exclusive_scan(c_in | (c_lt << 16), &both) & 0xffff;
+    const int n_in = both & 0xffff, n_lt = both >> 16;
+    if (n_in <= 2 * kSelectThreads) {  // uniform
+      for (int i = i0; i < i1; ++i) {
+        const uint32_t k = key[i];
+        if (k >= kw_lo && k <= kw_hi) ib[pos++] = (uint16_t)i;
+      }
+      __syncthreads();
+      unsigned long long *scratch = reinterpret_cast<unsigned long long *>(hist);
+      if (n_in <= kCountSortMax)
+        sort_count(key, ib, n_in, scratch);
+      else if (n_in <= kSelectThreads)
+        sort_small<1>(key, ib, n_in, scratch);
+      else
+        sort_small<2>(key, ib, n_in, scratch);
+      ord = ib;
+      base = n_lt;
+      len = n_in;
+    }
+  }
+  for (int attempt = 0; attempt < 2; ++attempt) {
+    if (!ord) {
+      ord = sort_rows(key, ia, ib, bid, n, hist, true);
+      base = 0;
+      len = n;
+    }
+    const bool whole = base == 0 && len == n;
+    if (tid == 0) {
+      int lo = k1 - base, hi = k1 - base;
+      bool escaped = lo < 1 || lo >= len;
+      if (!escaped && !cert_r(key, ord, lo, a.bounds)) {
+        --lo;
+        while (lo > 0 && !cert_r(key, ord, lo, a.bounds)) --lo;
+        ++hi;
+        while (hi < len && !cert_r(key, ord, hi, a.bounds)) ++hi;
+        escaped = !whole && (lo == 0 || hi == len);  // the run may go on outside the list
+      }
+      sh_lo = escaped ? -1 : lo;
+      sh_hi = hi;
+    }
+    __syncthreads();
+    if (sh_lo >= 0) break;
+    ord = nullptr;  // the window was not enough: sort everything
+  }
+  const int lo = sh_lo, hi = sh_hi;
+  if (base > 0)
+    for (int i = tid; i < n; i += nthr)
+      if (key[i] < kw_lo) fl[i] |= F_IMP;
+  for (int q = tid; q < lo; q += nthr) fl[ord[q]] |= F_IMP;
+  if (hi > lo) {
+    // The run's rows: double-float keys first (short runs), and exact
+    // sums when those do not separate every pair or a row has them already.
+    const uint8_t want = hi - lo <= kDfRunMax ? (uint8_t)(F_NEEDL | F_DF) : (uint8_t)F_NEEDL;
+    for (int q = lo + tid; q < hi; q += nthr) {
+      const int r = ord[q];
+      if (!(fl[r] & F_XL)) fl[r] |= want;
+    }
+    __syncthreads();
+    refine_pending(a, off, n, fl, rec, primary);
+    __syncthreads();
+    bool open = false;
+    for (int q = lo + tid; q < hi && !open; q += nthr) {
+      const int r = ord[q];
+      open = (fl[r] & F_XL) != 0;
+      for (int q2 = q + 1; q2 < hi && !open; ++q2) {
+        const int r2 = ord[q2];
+        open = (fl[r2] & F_XL) || df_cmp_r(rec[r2], rec[r], a.bounds) == 0;
+      }
+    }
+    if (__syncthreads_or(open)) {
+      for (int q = lo + tid; q < hi; q += nthr) {
+        const int r = ord[q];
+        if (!(fl[r] & F_XL)) fl[r] = (uint8_t)((fl[r] & ~F_DF) | F_NEEDL);
+      }
+      __syncthreads();
+      refine_pending(a, off, n, fl, rec, primary);
+      __syncthreads();
+    }
+    for (int q = lo + tid; q < hi; q += nthr) {
+      const int r = ord[q];
+      const bool exact = (fl[r] & F_XL) != 0;  // then every row of the run is
+      const bool ovf = exact && (rec[r].flags_l & kRecOverflowL);
+      int rank = 0;
+      for (int q2 = lo; q2 < hi; ++q2) {
+        if (q2 == q) continue;
+        const int r2 = ord[q2];
+        int c;
+        if (!exact)
+          c = df_cmp_r(rec[r2], rec[r], a.bounds);  // never 0 here
+        else if (ovf || (rec[r2].flags_l & kRecOverflowL))
+          c = q2 < q ? 1 : -1;  // no exact value: keep the float order
+        else
+          c = cmp_r(rec[r2], rec[r]);
+        if (c > 0 || (c == 0 && r2 < r)) ++rank;
+      }
+      if (base + lo + rank < k1) fl[r] |= F_IMP;
+    }
+  }
+  __syncthreads();
+}
+
+// 2. Stage I: top-K1 by R (equivalently H2), descending, lower index first.
+//    Marks X_imp (F_IMP) in the flags.
+__device__ __forceinline__ void stage_one(const SelectArgs &a, ImageCtx &c) {
+  const int tid = threadIdx.x;
+  const int nthr = blockDim.x;
+  const int n = c.n;
+  uint32_t *key = c.key;
+  uint32_t *hist = c.hist;
+  uint8_t *fl = c.fl;
+  ExactRec *rec = c.rec;
   const int k1 = c.k1;
   const bool need_r = c.need_r;
   if (need_r) {
@@ -1467,107 +1875,12 @@ __device__ __forceinline__ void stage_one(const SelectArgs &a, ImageCtx &c) {
         if (key[i] <= t1) fl[i] |= F_IMP;
       __syncthreads();
     } else {
-      // Uncertain cut: only the order near it matters.  The rows whose R32
-      // lies within a relative kCutWindow of the K1-th one (far wider than
-      // the certification band) are listed and sorted; when the uncertain
-      // run around the cut ends inside that list, every row with a smaller
-      // key (larger R) precedes it in the full order and is certainly kept,
-      // every row with a larger key certainly not.  Otherwise (or when the
-      // window holds too many rows) all n rows are sorted.
-      const float r1 = unord32(~t1);
-      const uint32_t kw_lo = ~ord32(r1 * (1.f + kCutWindow)), kw_hi = ~ord32(r1 * (1.f - kCutWindow));
-      const bool windowed = isfinite(r1) && r1 > 0.f;  // uniform
-      const uint16_t *ord = nullptr;
-      int base = 0, len = 0;  // ord[q] sits at position base + q of the full order
-      if (windowed) {
-        const int per = (n + nthr - 1) / nthr;
-        const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
-        int c_in = 0, c_lt = 0;
-        for (int i = i0; i < i1; ++i) {
-          const uint32_t k = key[i];
-          c_in += k >= kw_lo && k <= kw_hi;
-          c_lt += k < kw_lo;
-        }
-        int n_in = 0, n_lt = 0;
-        int pos = block_exclusive_scan(c_in, &n_in);
-        block_exclusive_scan(c_lt, &n_lt);
-        if (n_in <= 2 * kSelectThreads) {  // uniform
-          for (int i = i0; i < i1; ++i) {
-            const uint32_t k = key[i];
-            if (k >= kw_lo && k <= kw_hi) ib[pos++] = (uint16_t)i;
-          }
-          __syncthreads();
-          unsigned long long *scratch = reinterpret_cast<unsigned long long *>(hist);
-          if (n_in <= kSelectThreads)
-            sort_small<1>(key, ib, n_in, scratch);
-          else
-            sort_small<2>(key, ib, n_in, scratch);
-          ord = ib;
-          base = n_lt;
-          len = n_in;
-        }
-      }
-      for (int attempt = 0; attempt < 2; ++attempt) {
-        if (!ord) {
-          ord = sort_rows(key, ia, ib, bid, n, hist, true);
-          base = 0;
-          len = n;
-        }
-        const bool whole = base == 0 && len == n;
-        if (tid == 0) {
-          int lo = k1 - base, hi = k1 - base;
-          bool escaped = lo < 1 || lo >= len;
-          if (!escaped && !cert_r(key, ord, lo, a.bounds)) {
-            --lo;
-            while (lo > 0 && !cert_r(key, ord, lo, a.bounds)) --lo;
-            ++hi;
-            while (hi < len && !cert_r(key, ord, hi, a.bounds)) ++hi;
-            escaped = !whole && (lo == 0 || hi == len);  // the run may go on outside the list
-          }
-          sh_lo = escaped ? -1 : lo;
-          sh_hi = hi;
-        }
-        __syncthreads();
-        if (sh_lo >= 0) break;
-        ord = nullptr;  // the window was not enough: sort everything
-      }
-      const int lo = sh_lo, hi = sh_hi;
-      if (base > 0)
-        for (int i = tid; i < n; i += nthr)
-          if (key[i] < kw_lo) fl[i] |= F_IMP;
-      for (int q = tid; q < lo; q += nthr) fl[ord[q]] |= F_IMP;
-      if (hi > lo) {
-        for (int q = lo + tid; q < hi; q += nthr) {
-          const int r = ord[q];
-          if (!(fl[r] & F_XL)) fl[r] |= F_NEEDL;
-        }
-        __syncthreads();
-        refine_pending(a, off, n, fl, rec, primary);
-        __syncthreads();
-        for (int q = lo + tid; q < hi; q += nthr) {
-          const int r = ord[q];
-          const bool ovf = rec[r].flags_l & kRecOverflowL;
-          int rank = 0;
-          for (int q2 = lo; q2 < hi; ++q2) {
-            if (q2 == q) continue;
-            const int r2 = ord[q2];
-            int c;
-            if (ovf || (rec[r2].flags_l & kRecOverflowL))
-              c = q2 < q ? 1 : -1;  // no exact value: keep the float order
-            else
-              c = cmp_r(rec[r2], rec[r]);
-            if (c > 0 || (c == 0 && r2 < r)) ++rank;
-          }
-          if (base + lo + rank < k1) fl[r] |= F_IMP;
-        }
-      }
-      __syncthreads();
+      resolve_cut(a, c, t1);
     }
   } else if (k1 == n) {
     for (int i = tid; i < n; i += nthr) fl[i] |= F_IMP;
     __syncthreads();
   }
-
 }
 
 // 3a. Consistency keys ord32(s32) of every row (stage I's keys are no
@@ -1591,7 +1904,11 @@ __device__ __forceinline__ void consistency_keys(const SelectArgs &a, ImageCtx &
 #pragma unroll
     for (int u = 0; u < kKeyIlp; ++u) {
       const int i = i0 + u * nthr;
-      if (i < n) key[i] = ord32((fl[i] & F_XS) ? exact_s_key(rec[i]) : sv[u]);
+      if (i < n) {
+        const uint8_t f = fl[i];
+        key[i] = ord32((f & F_XS) ? exact_s_key(rec[i]) : sv[u]);
+        fl[i] = (uint8_t)(f & ~F_DF);  // a stage-I double-float key is not an s key
+      }
     }
   }
 }
@@ -1613,9 +1930,12 @@ __device__ __forceinline__ int list_rows(ImageCtx &c, uint16_t *dst, const bool 
   return m;
 }
 
-// 3b. Stage II along ord, X_rem sorted by s (m rows): the stride picks
-//     (F_DIV), with uncertain neighbourhoods settled exactly.
-__device__ __forceinline__ void stage_two_picks(const SelectArgs &a, ImageCtx &c, const uint16_t *ord, const int m) {
+// Stage II's uncertain neighbourhoods (rows flagged F_RUN): each run is
+// ranked by double-float keys or, failing those, exactly, and the stride
+// picks inside it are marked.  Out of line: only images with a near-tie at a
+// pick come here.
+__device__ __noinline__ void rank_pick_runs(const SelectArgs &a, const ImageCtx c, const uint16_t *ord, const int m,
+                                            const int t) {
   const int tid = threadIdx.x;
   const int nthr = blockDim.x;
   const int n = c.n;
@@ -1625,7 +1945,73 @@ __device__ __forceinline__ void stage_two_picks(const SelectArgs &a, ImageCtx &c
   ExactRec *rec = c.rec;
   const bool primary = c.primary;
   const int k2 = c.k2;
+  refine_pending(a, off, n, fl, rec, primary);
+  __syncthreads();
+  // A run whose double-float keys leave a pair unseparated (or with a row
+  // that has exact sums) is recomputed exactly as a whole.
+  bool open = false;
+  for (int q = tid; q < m; q += nthr) {
+    const int r = ord[q];
+    if (!(fl[r] & F_RUN) || (fl[r] & F_XS)) continue;
+    int lo = q;
+    while (lo > 0 && !cert_s(key, ord, lo, a.bounds)) --lo;
+    int hi = q + 1;
+    while (hi < m && !cert_s(key, ord, hi, a.bounds)) ++hi;
+    bool undecided = false;
+    for (int q2 = lo; q2 < hi && !undecided; ++q2) {
+      if (q2 == q) continue;
+      const int r2 = ord[q2];
+      undecided = (fl[r2] & F_XS) || df_cmp_s(rec[r2], rec[r], a.bounds) == 0;
+    }
+    if (undecided) {
+      open = true;
+      for (int q2 = lo; q2 < hi; ++q2) {
+        const int r2 = ord[q2];
+        if (!(fl[r2] & F_XS)) fl[r2] = (uint8_t)((fl[r2] & ~F_DF) | F_NEEDS);
+      }
+    }
+  }
+  if (__syncthreads_or(open)) {
+    refine_pending(a, off, n, fl, rec, primary);
+    __syncthreads();
+  }
+  for (int q = tid; q < m; q += nthr) {
+    const int r = ord[q];
+    if (!(fl[r] & F_RUN)) continue;
+    int lo = q;
+    while (lo > 0 && !cert_s(key, ord, lo, a.bounds)) --lo;
+    int hi = q + 1;
+    while (hi < m && !cert_s(key, ord, hi, a.bounds)) ++hi;
+    const bool exact = (fl[r] & F_XS) != 0;  // then every row of the run is
+    const bool ovf = exact && (rec[r].flags_s & kRecOverflowS);
+    int rank = 0;
+    for (int q2 = lo; q2 < hi; ++q2) {
+      if (q2 == q) continue;
+      const int r2 = ord[q2];
+      int c;
+      if (!exact)
+        c = df_cmp_s(rec[r2], rec[r], a.bounds);  // never 0 here
+      else if (ovf || (rec[r2].flags_s & kRecOverflowS))
+        c = q2 < q ? -1 : 1;
+      else
+        c = cmp_s(rec[r2], rec[r]);
+      if (c < 0 || (c == 0 && r2 < r)) ++rank;
+    }
+    if (is_pick(lo + rank, m, k2, t, a.stride_interval)) fl[r] |= F_DIV;
+  }
+  __syncthreads();
+}
+
+// 3b. Stage II along ord, X_rem sorted by s (m rows): the stride picks
+//     (F_DIV), with uncertain neighbourhoods settled exactly.
+__device__ __forceinline__ void stage_two_picks(const SelectArgs &a, ImageCtx &c, const uint16_t *ord, const int m) {
+  const int tid = threadIdx.x;
+  const int nthr = blockDim.x;
+  uint32_t *key = c.key;
+  uint8_t *fl = c.fl;
+  const int k2 = c.k2;
   const int t = max(1, m / k2);
+  bool marked = false;  // some pick's neighbourhood is uncertain
   for (int j = tid; j < k2; j += nthr) {
     const int p = pick_position(j, m, k2, t, a.stride_interval);
     const bool c0 = p == 0 || cert_s(key, ord, p, a.bounds);
@@ -1638,37 +2024,16 @@ __device__ __forceinline__ void stage_two_picks(const SelectArgs &a, ImageCtx &c
       int hi = p + 1;
       while (hi < m && !cert_s(key, ord, hi, a.bounds)) ++hi;
       // Threads whose runs coincide write the same bits: the races are benign.
+      // Short runs try the double-float keys first.
+      const uint8_t want = hi - lo <= kDfRunMax ? (uint8_t)(F_NEEDS | F_DF) : (uint8_t)F_NEEDS;
       for (int q = lo; q < hi; ++q) {
         const int r = ord[q];
-        fl[r] |= (uint8_t)(F_RUN | ((fl[r] & F_XS) ? 0 : F_NEEDS));
+        fl[r] |= (uint8_t)(F_RUN | ((fl[r] & F_XS) ? 0 : want));
       }
+      marked = true;
     }
   }
-  __syncthreads();
-  refine_pending(a, off, n, fl, rec, primary);
-  __syncthreads();
-  for (int q = tid; q < m; q += nthr) {
-    const int r = ord[q];
-    if (!(fl[r] & F_RUN)) continue;
-    int lo = q;
-    while (lo > 0 && !cert_s(key, ord, lo, a.bounds)) --lo;
-    int hi = q + 1;
-    while (hi < m && !cert_s(key, ord, hi, a.bounds)) ++hi;
-    const bool ovf = rec[r].flags_s & kRecOverflowS;
-    int rank = 0;
-    for (int q2 = lo; q2 < hi; ++q2) {
-      if (q2 == q) continue;
-      const int r2 = ord[q2];
-      int c;
-      if (ovf || (rec[r2].flags_s & kRecOverflowS))
-        c = q2 < q ? -1 : 1;
-      else
-        c = cmp_s(rec[r2], rec[r]);
-      if (c < 0 || (c == 0 && r2 < r)) ++rank;
-    }
-    if (is_pick(lo + rank, m, k2, t, a.stride_interval)) fl[r] |= F_DIV;
-  }
-  __syncthreads();
+  if (__syncthreads_or(marked)) rank_pick_runs(a, c, ord, m, t);  // else every pick is certain
 }
 
 // 4. X* = X_imp union X_div in ascending token order (Eq. 7), plus outputs;

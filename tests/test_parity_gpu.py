@@ -632,6 +632,60 @@ def test_exact_sums_past_the_window():
         check_reduce(x, xp, xq, [n], ([k], [k1], [0, k]))
 
 
+def _near_tie_triples(groups, d, dtype, seed):
+    """Rows in triples whose keys R and s differ by about 2^-25 inside a
+    triple (inside the fp32 keys' certification band, so every triple is an
+    uncertain run) and by about 2^-17 between triples (certain in fp32).
+    Two channels of x set R: a coarse one (two mantissa steps of 2^-3 per
+    triple, in a shuffled triple order) and a fine one (one step of 2^-10 per
+    member); two channels of x'' set s the same way against x' = 4 there.
+    The rows are shuffled so that index order and key order differ."""
+    g = torch.Generator().manual_seed(seed)
+    n = 3 * groups
+    base = torch.randn(d, generator=g)
+    base_p = torch.randn(d, generator=g)
+    base_q = 0.5 * base_p + 0.5 * torch.randn(d, generator=g)
+    x, xp, xq = base.repeat(n, 1), base_p.repeat(n, 1), base_q.repeat(n, 1)
+    coarse_r = torch.randperm(groups, generator=g)
+    coarse_s = torch.randperm(groups, generator=g)
+    for i in range(n):
+        grp, mem = divmod(i, 3)
+        x[i, 11] = 2.0 ** -3 * (1 + 2 * int(coarse_r[grp]) / 128)
+        x[i, 517] = 2.0 ** -10 * (1 + mem / 128)
+        xq[i, 23] = 2.0 ** -3 * (1 + 2 * int(coarse_s[grp]) / 128)
+        xq[i, 700] = 2.0 ** -10 * (1 + ((mem + grp) % 3) / 128)
+    xp[:, 23] = 4.0
+    xp[:, 700] = 4.0
+    perm = torch.randperm(n, generator=g)
+    return x[perm].to(dtype), xp[perm].to(dtype), xq[perm].to(dtype), perm, coarse_r, coarse_s
+
+
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32], ids=["bf16", "f32"])
+def test_near_ties_beyond_fp32(dtype):
+    # Every triple is an uncertain run of the fp32 keys; the double-float
+    # keys separate its rows, so the selection needs no exact sums
+    # (status[2] == 0) and still matches the oracle's exact decisions, at the
+    # importance cut (K1 = 31 splits a triple) and at the stride picks.
+    x, xp, xq, *_ = _near_tie_triples(32, 1024, dtype, 31)
+    n = x.shape[0]
+    for k, k1 in [(40, 31), (60, 0), (45, 16)]:
+        st = check_reduce(x, xp, xq, [n], ([k], [k1], [0, k]))
+        assert st[2] == 0, st
+    # exact ties inside two triples (two rows equal in x, two in x''): the
+    # triple that the importance cut K1 = 31 splits (the 11th from the top
+    # by R) and the triple with the smallest s (the first stride pick) fall
+    # back to exact sums, every other run stays with the double-float keys
+    x, xp, xq, perm, cr, cs = _near_tie_triples(32, 1024, dtype, 32)
+    where = torch.argsort(perm)  # where[i]: the shuffled place of row i
+    gr = int((cr == 32 - 11).nonzero())
+    gs = int((cs == 0).nonzero())
+    x[where[3 * gr + 1]] = x[where[3 * gr]]
+    xq[where[3 * gs + 1]] = xq[where[3 * gs]]
+    for k, k1 in [(40, 31), (60, 0)]:
+        st = check_reduce(x, xp, xq, [n], ([k], [k1], [0, k]))
+        assert 0 < st[2] <= 6, st
+
+
 def test_fp32_wide_range():
     n, d = 300, 1024
     g = torch.Generator().manual_seed(5)
