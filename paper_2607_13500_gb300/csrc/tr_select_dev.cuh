@@ -61,7 +61,8 @@ __device__ __forceinline__ float key_r(const float *st) { return __ldcg(st + 6);
 __device__ __forceinline__ float key_s(const float *st) { return __ldcg(st + 7); }
 // Both keys in one 8-byte load (records are 32-byte aligned).
 __device__ __forceinline__ float2 key_rs(const float *st) { return __ldcg(reinterpret_cast<const float2 *>(st + 6)); }
-constexpr int kKeyIlp = 4;  // rows whose keys a thread loads before it uses any
+constexpr int kKeyIlp = 8;  // rows whose keys a thread loads before it uses any
+constexpr int kRowIlp = 4;  // rows a thread takes at a time in the shared-memory row passes
 
 // ---- a Big truncated to a 64-bit mantissa: value in [m 2^e, (m + 1) 2^e) ----
 // Integer-only (the GPU's fp64 rate is far too low for this path).
@@ -513,8 +514,8 @@ struct Group {
 // 16-byte chunks t, t + size, ...), in three 128-bit windows; false
 // (uniformly across the group) when a term does not fit its window.
 template <int kDt>
-__device__ bool exact_row_block(const SelectArgs &a, long long row, int mode, const float *st, ExactRec *rec,
-                                Part128 &part, const Group &g) {
+__device__ __noinline__ bool exact_row_block(const SelectArgs &a, long long row, int mode, const float *st,
+                                             ExactRec *rec, Part128 &part, const Group g) {
   constexpr int kPer = kDt == TR_F32 ? 4 : 8;  // elements per 16-byte chunk
   const int nchunks = a.d / kPer;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -704,8 +705,8 @@ struct PartDf {
 // returns true, uniformly across the group, or false when the row is not
 // eligible (nothing written).
 template <int kDt>
-__device__ bool df_row_block(const SelectArgs &a, long long row, int mode, ExactRec *rec, PartDf &part,
-                             const Group &g) {
+__device__ __noinline__ bool df_row_block(const SelectArgs &a, long long row, int mode, ExactRec *rec, PartDf &part,
+                                          const Group g) {
   constexpr int kPer = kDt == TR_F32 ? 4 : 8;  // elements per 16-byte chunk
   constexpr int kLoads = 4;                    // chunks per stream in flight per thread
   const int nchunks = a.d / kPer;
@@ -843,10 +844,47 @@ __device__ __forceinline__ bool df_row_any(const SelectArgs &a, long long row, i
 // F_XS).  The pending rows are listed first (a block-wide vote skips everything when
 // none is); then up to four rows at a time are handled by groups of warps.
 constexpr int kPendCap = 512;
-__device__ __noinline__ void refine_listed(const SelectArgs &a, long long off, int n, uint8_t *fl, ExactRec *rec,
-                                           const bool primary) {
+// Recomputes the rows list[0..cnt) (local indices, cnt <= kPendCap) as
+// their flags request, up to four rows at a time by groups of warps.
+// Called by the whole block; ends with a block barrier.
+__device__ __noinline__ void refine_list(const SelectArgs &a, long long off, const int *list, const int cnt,
+                                         uint8_t *fl, ExactRec *rec, const bool primary) {
   __shared__ Part128 part;
   __shared__ PartDf pdf;
+  const int groups = cnt >= 4 ? 4 : (cnt >= 2 ? 2 : 1);
+  const int gsize = (int)blockDim.x / groups;
+  const int gi = (int)threadIdx.x / gsize;
+  const Group g{gi * gsize, gsize, 1 + gi};
+  for (int base = 0; base < cnt; base += groups) {
+    if (base + gi < cnt) {
+      const int row = list[base + gi];
+      const uint8_t fr = fl[row];
+      const float *st = a.stats + (off + row) * TR_STATS_WORDS;
+      bool dl = false, ds = false;  // settled by the double-float tier
+      if (fr & F_NEEDL) {
+        if (fr & F_DF) dl = df_row_any(a, off + row, 0, rec + row, pdf, g);
+        if (!dl) exact_row_any(a, off + row, 0, st, rec + row, part, g);
+      }
+      if (fr & F_NEEDS) {
+        if (fr & F_DF) ds = df_row_any(a, off + row, 1, rec + row, pdf, g);
+        if (!ds) exact_row_any(a, off + row, 1, st, rec + row, part, g);
+      }
+      if (g.tid() == 0 && (fr & (F_NEEDL | F_NEEDS))) {  // a listed row may request nothing
+        uint8_t f = (uint8_t)(fr & ~(F_NEEDL | F_NEEDS | F_DF));
+        if (fr & F_NEEDL) f |= dl ? F_DF : F_XL;
+        if (fr & F_NEEDS) f |= ds ? F_DF : F_XS;
+        fl[row] = f;
+        const bool exact = ((fr & F_NEEDL) && !dl) || ((fr & F_NEEDS) && !ds);
+        if (exact && a.status && primary) atomicAdd(&a.status[2], 1);
+      }
+    }
+    __syncthreads();
+  }
+}
+
+// Every row of the image whose flags request it, listed from the flags.
+__device__ __noinline__ void refine_listed(const SelectArgs &a, long long off, int n, uint8_t *fl, ExactRec *rec,
+                                           const bool primary) {
   __shared__ int plist[kPendCap];
   __shared__ int pcount;
   for (;;) {
@@ -861,36 +899,7 @@ __device__ __noinline__ void refine_listed(const SelectArgs &a, long long off, i
     __syncthreads();
     const int total = pcount;
     if (total == 0) break;
-    const int cnt = min(total, kPendCap);
-    const int groups = cnt >= 4 ? 4 : (cnt >= 2 ? 2 : 1);
-    const int gsize = (int)blockDim.x / groups;
-    const int gi = (int)threadIdx.x / gsize;
-    const Group g{gi * gsize, gsize, 1 + gi};
-    for (int base = 0; base < cnt; base += groups) {
-      if (base + gi < cnt) {
-        const int row = plist[base + gi];
-        const uint8_t fr = fl[row];
-        const float *st = a.stats + (off + row) * TR_STATS_WORDS;
-        bool dl = false, ds = false;  // settled by the double-float tier
-        if (fr & F_NEEDL) {
-          if (fr & F_DF) dl = df_row_any(a, off + row, 0, rec + row, pdf, g);
-          if (!dl) exact_row_any(a, off + row, 0, st, rec + row, part, g);
-        }
-        if (fr & F_NEEDS) {
-          if (fr & F_DF) ds = df_row_any(a, off + row, 1, rec + row, pdf, g);
-          if (!ds) exact_row_any(a, off + row, 1, st, rec + row, part, g);
-        }
-        if (g.tid() == 0) {
-          uint8_t f = (uint8_t)(fr & ~(F_NEEDL | F_NEEDS | F_DF));
-          if (fr & F_NEEDL) f |= dl ? F_DF : F_XL;
-          if (fr & F_NEEDS) f |= ds ? F_DF : F_XS;
-          fl[row] = f;
-          const bool exact = ((fr & F_NEEDL) && !dl) || ((fr & F_NEEDS) && !ds);
-          if (exact && a.status && primary) atomicAdd(&a.status[2], 1);
-        }
-      }
-      __syncthreads();
-    }
+    refine_list(a, off, plist, min(total, kPendCap), fl, rec, primary);
     if (total <= kPendCap) break;  // otherwise list the rows still pending
   }
 }
@@ -1366,27 +1375,39 @@ __device__ __noinline__ uint16_t *sample_sort(const uint32_t *key, uint16_t *a, 
 // and each row's final place is its bucket's start plus the number of
 // bucket members with a smaller (key, row), counted by one thread per row
 // (buckets hold about one row on the workloads here, at most kBucketMax).
-// Returns a, holding the order, or nullptr, having changed nothing, when
-// some bucket would hold more than kBucketMax rows (ties, or keys crowded
-// together), a key encodes NaN, or the keys span no usable range: the caller
-// then takes another sort.  hist: at least nb words.
+// Returns a, holding the order, or nullptr, having changed nothing but the
+// scratch bid (each position's bucket), when some bucket would hold more
+// than kBucketMax rows (ties, or keys crowded together), a key encodes NaN,
+// or the keys span no usable range: the caller then takes another sort.
+// hist: at least nb words.
 constexpr int kBucketMax = 32;
 constexpr int kBuckets = 4096;
 __device__ __forceinline__ float key_value(uint32_t k, bool complemented) {
   return complemented ? -unord32(~k) : unord32(k);
 }
-__device__ uint16_t *bucket_sort(const uint32_t *key, uint16_t *a, uint16_t *b, int m, uint32_t *hist,
+__device__ uint16_t *bucket_sort(const uint32_t *key, uint16_t *a, uint16_t *b, uint16_t *bid, int m, uint32_t *hist,
                                  bool complemented) {
   __shared__ float sh_min[kWarps], sh_max[kWarps];
   __shared__ int sh_big;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nthr = blockDim.x;
+  // Every pass over the rows takes kRowIlp of them per thread at a time,
+  // their loads first, so that the shared-memory latencies overlap.
   float vmin = INFINITY, vmax = -INFINITY;
   bool nan = false;
-  for (int q = tid; q < m; q += blockDim.x) {
-    const float v = key_value(key[a[q]], complemented);
-    vmin = fminf(vmin, v);
-    vmax = fmaxf(vmax, v);
-    nan |= v != v;
+  for (int q0 = tid; q0 < m; q0 += kRowIlp * nthr) {
+    uint16_t r[kRowIlp];
+    uint32_t k[kRowIlp];
+#pragma unroll
+    for (int u = 0; u < kRowIlp; ++u) r[u] = a[min(q0 + u * nthr, m - 1)];  // repeats are harmless here
+#pragma unroll
+    for (int u = 0; u < kRowIlp; ++u) k[u] = key[r[u]];
+#pragma unroll
+    for (int u = 0; u < kRowIlp; ++u) {
+      const float v = key_value(k[u], complemented);
+      vmin = fminf(vmin, v);
+      vmax = fmaxf(vmax, v);
+      nan |= v != v;
+    }
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -1399,7 +1420,7 @@ __device__ uint16_t *bucket_sort(const uint32_t *key, uint16_t *a, uint16_t *b, 
   }
   int nb = 64;
   while (nb < m && nb < kBuckets) nb <<= 1;
-  for (int c = tid; c < nb; c += blockDim.x) hist[c] = 0u;
+  for (int c = tid; c < nb; c += nthr) hist[c] = 0u;
   if (tid == 0) sh_big = 0;
   __syncthreads();
   if (__syncthreads_or(nan)) return nullptr;  // uniform; NaN has no place in a linear bucket map
@@ -1414,10 +1435,27 @@ __device__ uint16_t *bucket_sort(const uint32_t *key, uint16_t *a, uint16_t *b, 
   if (!(span > 0.f) || !isfinite(span) || !isfinite(scale)) return nullptr;  // uniform: all equal or no usable range
   // bucket of a value: floor((v - vmin) * scale), monotone in v, clamped to the last bucket
   auto bucket = [&](float v) { return min(nb - 1, (int)((v - vmin) * scale)); };
-  for (int q = tid; q < m; q += blockDim.x) atomicAdd(&hist[bucket(key_value(key[a[q]], complemented))], 1u);
+  // counts per bucket; each position's bucket is kept in bid for the scatter
+  for (int q0 = tid; q0 < m; q0 += kRowIlp * nthr) {
+    uint16_t r[kRowIlp];
+    uint32_t k[kRowIlp];
+#pragma unroll
+    for (int u = 0; u < kRowIlp; ++u) r[u] = a[min(q0 + u * nthr, m - 1)];
+#pragma unroll
+    for (int u = 0; u < kRowIlp; ++u) k[u] = key[r[u]];
+#pragma unroll
+    for (int u = 0; u < kRowIlp; ++u) {
+      const int q = q0 + u * nthr;
+      if (q < m) {
+        const int c = bucket(key_value(k[u], complemented));
+        bid[q] = (uint16_t)c;
+        atomicAdd(&hist[c], 1u);
+      }
+    }
+  }
   __syncthreads();
   // exclusive scan of the bucket counts (each thread a contiguous stretch) and the largest count
-  const int per = (nb + blockDim.x - 1) / blockDim.x;
+  const int per = (nb + nthr - 1) / nthr;
   const int c0 = min(nb, tid * per), c1 = min(nb, c0 + per);
   int run = 0, big = 0;
   for (int c = c0; c < c1; ++c) {
@@ -1434,24 +1472,54 @@ __device__ uint16_t *bucket_sort(const uint32_t *key, uint16_t *a, uint16_t *b, 
     base += cnt;
   }
   __syncthreads();
-  for (int q = tid; q < m; q += blockDim.x) {
-    const uint16_t row = a[q];
-    b[atomicAdd(&hist[bucket(key_value(key[row], complemented))], 1u)] = row;
+  for (int q0 = tid; q0 < m; q0 += kRowIlp * nthr) {
+    uint16_t r[kRowIlp], c[kRowIlp];
+    uint32_t pos[kRowIlp];
+#pragma unroll
+    for (int u = 0; u < kRowIlp; ++u) {
+      const int q = min(q0 + u * nthr, m - 1);
+      r[u] = a[q];
+      c[u] = bid[q];
+    }
+#pragma unroll
+    for (int u = 0; u < kRowIlp; ++u)
+      if (q0 + u * nthr < m) pos[u] = atomicAdd(&hist[c[u]], 1u);
+#pragma unroll
+    for (int u = 0; u < kRowIlp; ++u)
+      if (q0 + u * nthr < m) b[pos[u]] = r[u];
   }
   __syncthreads();
-  // hist[c] is now the end of bucket c, so bucket c spans [hist[c - 1], hist[c])
-  for (int q = tid; q < m; q += blockDim.x) {
-    const uint16_t row = b[q];
-    const uint32_t kr = key[row];
-    const int c = bucket(key_value(kr, complemented));
-    const int lo = c ? (int)hist[c - 1] : 0, hi = (int)hist[c];
-    const unsigned long long kk = ((unsigned long long)kr << 16) | row;
-    int rank = 0;
-    for (int j = lo; j < hi; ++j) {
-      const uint16_t r2 = b[j];
-      rank += (((unsigned long long)key[r2] << 16) | r2) < kk;
+  // hist[c] is now the end of bucket c, so bucket c spans [hist[c - 1], hist[c]);
+  // a row's place is its bucket's start plus the members with a smaller composite key
+  for (int q0 = tid; q0 < m; q0 += kRowIlp * nthr) {
+    uint16_t row[kRowIlp];
+    uint32_t kr[kRowIlp];
+    int lo[kRowIlp], hi[kRowIlp];
+#pragma unroll
+    for (int u = 0; u < kRowIlp; ++u) row[u] = b[min(q0 + u * nthr, m - 1)];
+#pragma unroll
+    for (int u = 0; u < kRowIlp; ++u) kr[u] = key[row[u]];
+#pragma unroll
+    for (int u = 0; u < kRowIlp; ++u) {
+      const int c = bucket(key_value(kr[u], complemented));
+      lo[u] = c ? (int)hist[c - 1] : 0;
+      hi[u] = (int)hist[c];
     }
-    a[lo + rank] = row;
+#pragma unroll
+    for (int u = 0; u < kRowIlp; ++u) {
+      int rank = 0;
+      if (hi[u] - lo[u] > 1) {
+        const unsigned long long kk = ((unsigned long long)kr[u] << 16) | row[u];
+        for (int j = lo[u]; j < hi[u]; ++j) {
+          const uint16_t r2 = b[j];
+          rank += (((unsigned long long)key[r2] << 16) | r2) < kk;
+        }
+      }
+      lo[u] += rank;
+    }
+#pragma unroll
+    for (int u = 0; u < kRowIlp; ++u)
+      if (q0 + u * nthr < m) a[lo[u]] = row[u];
   }
   __syncthreads();
   return a;
@@ -1475,7 +1543,7 @@ __device__ uint16_t *sort_rows(const uint32_t *key, uint16_t *a, uint16_t *b, ui
       sort_small<1>(key, a, m, scratch);
     return a;
   }
-  if (uint16_t *o = bucket_sort(key, a, b, m, hist, complemented)) return o;
+  if (uint16_t *o = bucket_sort(key, a, b, bid, m, hist, complemented)) return o;
   if (m <= 2 * kSelectThreads) {
     __syncthreads();
     sort_small<2>(key, a, m, scratch);
@@ -1513,9 +1581,13 @@ __device__ uint32_t select_rank(const uint32_t *key, int n, int r, uint32_t *his
     uint32_t *h = hist + warp * 256;
     for (int d = lane; d < 256; d += 32) h[d] = 0u;
     __syncwarp();
-    for (int i = tid; i < n; i += blockDim.x) {
-      const uint32_t k = key[i];
-      if ((k & mask) == pre) atomicAdd(&h[(k >> shift) & 0xffu], 1u);
+    for (int i0 = tid; i0 < n; i0 += kRowIlp * blockDim.x) {
+      uint32_t k[kRowIlp];
+#pragma unroll
+      for (int u = 0; u < kRowIlp; ++u) k[u] = key[min(i0 + u * (int)blockDim.x, n - 1)];
+#pragma unroll
+      for (int u = 0; u < kRowIlp; ++u)
+        if (i0 + u * (int)blockDim.x < n && (k[u] & mask) == pre) atomicAdd(&h[(k[u] >> shift) & 0xffu], 1u);
     }
     __syncthreads();
     if (tid < 256) {  // column tid: only this thread reads or writes it here
@@ -1605,6 +1677,17 @@ __device__ __forceinline__ bool is_pick(int q, int m, int k2, int t, bool interv
 // (replicas that run the same deterministic selection write nothing).
 // The state of one image's selection in a CTA: where its rows are, its
 // budgets and the CTA's shared-memory arrays (layout in select_smem_bytes).
+// The uncertain runs of one image's decisions, kept so that their rows are
+// recomputed and ranked without passes over every row: a run is a stretch
+// [lo, hi) of sorted positions, packed (lo << 16) | hi.
+constexpr int kMaxRuns = 128;
+struct RunList {
+  uint32_t run[kMaxRuns];
+  int count, rows, longest;  // runs recorded (may exceed kMaxRuns), their rows, the longest
+  int npend, npend2;         // rows listed for the first and second recomputation
+  int list[kPendCap];
+};
+
 struct ImageCtx {
   long long off;
   int n, k, k1, k2, ko;
@@ -1614,6 +1697,7 @@ struct ImageCtx {
   uint8_t *fl;
   const float *st;
   ExactRec *rec;
+  RunList *runs;  // block-shared
 };
 
 // Sets up c for image b; false when there is nothing to select (an invalid
@@ -1799,9 +1883,13 @@ __device__ __noinline__ void resolve_cut(const SelectArgs &a, const ImageCtx c, 
     for (int q = lo + tid; q < hi; q += nthr) {
       const int r = ord[q];
       if (!(fl[r] & F_XL)) fl[r] |= want;
+      if (hi - lo <= kPendCap) c.runs->list[q - lo] = r;  // rows with nothing requested are left alone
     }
     __syncthreads();
-    refine_pending(a, off, n, fl, rec, primary);
+    if (hi - lo <= kPendCap)
+      refine_list(a, off, c.runs->list, hi - lo, fl, rec, primary);
+    else
+      refine_pending(a, off, n, fl, rec, primary);
     __syncthreads();
     bool open = false;
     for (int q = lo + tid; q < hi && !open; q += nthr) {
@@ -1818,7 +1906,10 @@ __device__ __noinline__ void resolve_cut(const SelectArgs &a, const ImageCtx c, 
         if (!(fl[r] & F_XL)) fl[r] = (uint8_t)((fl[r] & ~F_DF) | F_NEEDL);
       }
       __syncthreads();
-      refine_pending(a, off, n, fl, rec, primary);
+      if (hi - lo <= kPendCap)
+        refine_list(a, off, c.runs->list, hi - lo, fl, rec, primary);
+      else
+        refine_pending(a, off, n, fl, rec, primary);
       __syncthreads();
     }
     for (int q = lo + tid; q < hi; q += nthr) {
@@ -1871,8 +1962,19 @@ __device__ __forceinline__ void stage_one(const SelectArgs &a, ImageCtx &c) {
       settled = cert_r_val(unord32(~t1), unord32(~t2), a.bounds);
     }
     if (settled) {
-      for (int i = tid; i < n; i += nthr)
-        if (key[i] <= t1) fl[i] |= F_IMP;
+      for (int i0 = tid; i0 < n; i0 += kRowIlp * nthr) {
+        uint32_t k[kRowIlp];
+        uint8_t f[kRowIlp];
+#pragma unroll
+        for (int u = 0; u < kRowIlp; ++u) {
+          const int i = min(i0 + u * nthr, n - 1);
+          k[u] = key[i];
+          f[u] = fl[i];
+        }
+#pragma unroll
+        for (int u = 0; u < kRowIlp; ++u)
+          if (i0 + u * nthr < n && k[u] <= t1) fl[i0 + u * nthr] = (uint8_t)(f[u] | F_IMP);
+      }
       __syncthreads();
     } else {
       resolve_cut(a, c, t1);
@@ -1913,19 +2015,38 @@ __device__ __forceinline__ void consistency_keys(const SelectArgs &a, ImageCtx &
   }
 }
 
+// Row passes in index order give each thread a contiguous stretch of rows,
+// a multiple of 4 long (at most 32), whose flags it loads as 32-bit words
+// before using any (the flags array is 16-byte aligned).
+constexpr int kStretchWords = 8;
+static_assert(TR_MAX_N <= 4 * kStretchWords * kSelectThreads, "a stretch holds at most 32 rows");
+__device__ __forceinline__ int stretch_rows(int n) { return 4 * ((n + 4 * kSelectThreads - 1) / (4 * kSelectThreads)); }
+__device__ __forceinline__ void load_stretch(const uint8_t *fl, int i0, int i1, uint32_t (&w)[kStretchWords]) {
+  const uint32_t *fw = reinterpret_cast<const uint32_t *>(fl + i0);
+#pragma unroll
+  for (int j = 0; j < kStretchWords; ++j) w[j] = i0 + 4 * j < i1 ? fw[j] : 0u;
+}
+__device__ __forceinline__ uint8_t stretch_flag(const uint32_t (&w)[kStretchWords], int j) {
+  return (uint8_t)((w[j >> 2] >> (8 * (j & 3))) & 0xffu);
+}
+
 // The rows of the image (all, or those outside X_imp) in ascending index
 // order -- the stable sort's tie order -- into dst; returns their number.
 __device__ __forceinline__ int list_rows(ImageCtx &c, uint16_t *dst, const bool skip_imp) {
-  const int tid = threadIdx.x, nthr = blockDim.x, n = c.n;
-  const uint8_t *fl = c.fl;
-  const int per = (n + nthr - 1) / nthr;
+  const int tid = threadIdx.x, n = c.n;
+  const int per = stretch_rows(n);
   const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
+  uint32_t w[kStretchWords];
+  load_stretch(c.fl, i0, i1, w);
   int cnt = 0;
-  for (int i = i0; i < i1; ++i) cnt += !(skip_imp && (fl[i] & F_IMP));
+#pragma unroll
+  for (int j = 0; j < 4 * kStretchWords; ++j)
+    if (i0 + j < i1) cnt += !(skip_imp && (stretch_flag(w, j) & F_IMP));
   int m = 0;
   int pos = block_exclusive_scan(cnt, &m);
-  for (int i = i0; i < i1; ++i)
-    if (!(skip_imp && (fl[i] & F_IMP))) dst[pos++] = (uint16_t)i;
+#pragma unroll
+  for (int j = 0; j < 4 * kStretchWords; ++j)
+    if (i0 + j < i1 && !(skip_imp && (stretch_flag(w, j) & F_IMP))) dst[pos++] = (uint16_t)(i0 + j);
   __syncthreads();
   return m;
 }
@@ -1933,9 +2054,11 @@ __device__ __forceinline__ int list_rows(ImageCtx &c, uint16_t *dst, const bool 
 // Stage II's uncertain neighbourhoods (rows flagged F_RUN): each run is
 // ranked by double-float keys or, failing those, exactly, and the stride
 // picks inside it are marked.  Out of line: only images with a near-tie at a
-// pick come here.
-__device__ __noinline__ void rank_pick_runs(const SelectArgs &a, const ImageCtx c, const uint16_t *ord, const int m,
-                                            const int t) {
+// pick come here.  This version passes over every sorted position; the one
+// below works from the recorded runs and takes over when they are few and
+// short.
+__device__ __noinline__ void rank_pick_runs_all(const SelectArgs &a, const ImageCtx c, const uint16_t *ord,
+                                                const int m, const int t) {
   const int tid = threadIdx.x;
   const int nthr = blockDim.x;
   const int n = c.n;
@@ -2002,6 +2125,82 @@ __device__ __noinline__ void rank_pick_runs(const SelectArgs &a, const ImageCtx 
   __syncthreads();
 }
 
+// The recorded runs: their rows are listed directly (no pass over all
+// positions), recomputed, checked pairwise and ranked, one thread per run.
+__device__ __noinline__ void rank_pick_runs(const SelectArgs &a, const ImageCtx c, const uint16_t *ord, const int m,
+                                            const int t) {
+  RunList &rl = *c.runs;
+  const int nruns = rl.count;
+  if (nruns > kMaxRuns || rl.rows > kPendCap || rl.longest > kDfRunMax) {  // uniform
+    rank_pick_runs_all(a, c, ord, m, t);
+    return;
+  }
+  const int tid = threadIdx.x, nthr = blockDim.x;
+  uint8_t *fl = c.fl;
+  ExactRec *rec = c.rec;
+  const int k2 = c.k2;
+  // 1. the runs' rows that request a recomputation (double-float first)
+  for (int r = tid; r < nruns; r += nthr) {
+    const int lo = (int)(rl.run[r] >> 16), hi = (int)(rl.run[r] & 0xffffu);
+    for (int q = lo; q < hi; ++q) {
+      const int row = ord[q];
+      if (fl[row] & F_NEEDS) rl.list[atomicAdd(&rl.npend, 1)] = row;
+    }
+  }
+  __syncthreads();
+  if (rl.npend) refine_list(a, c.off, rl.list, rl.npend, fl, rec, c.primary);
+  // 2. a run whose double-float keys leave a pair unseparated (or with a
+  //    row that has exact sums) is recomputed exactly as a whole
+  for (int r = tid; r < nruns; r += nthr) {
+    const int lo = (int)(rl.run[r] >> 16), hi = (int)(rl.run[r] & 0xffffu);
+    bool undecided = false;
+    for (int q = lo; q < hi && !undecided; ++q) {
+      const int r1 = ord[q];
+      undecided = (fl[r1] & F_XS) != 0;
+      for (int q2 = q + 1; q2 < hi && !undecided; ++q2) {
+        const int r2 = ord[q2];
+        undecided = (fl[r2] & F_XS) || df_cmp_s(rec[r2], rec[r1], a.bounds) == 0;
+      }
+    }
+    if (undecided) {
+      for (int q = lo; q < hi; ++q) {
+        const int row = ord[q];
+        if (!(fl[row] & F_XS)) {
+          fl[row] = (uint8_t)((fl[row] & ~F_DF) | F_NEEDS);
+          rl.list[atomicAdd(&rl.npend2, 1)] = row;
+        }
+      }
+    }
+  }
+  __syncthreads();
+  if (rl.npend2) refine_list(a, c.off, rl.list, rl.npend2, fl, rec, c.primary);
+  // 3. ranks inside each run (every row of a run is double-float, or every
+  //    row exact), and the picks among them
+  for (int r = tid; r < nruns; r += nthr) {
+    const int lo = (int)(rl.run[r] >> 16), hi = (int)(rl.run[r] & 0xffffu);
+    for (int q = lo; q < hi; ++q) {
+      const int row = ord[q];
+      const bool exact = (fl[row] & F_XS) != 0;
+      const bool ovf = exact && (rec[row].flags_s & kRecOverflowS);
+      int rank = 0;
+      for (int q2 = lo; q2 < hi; ++q2) {
+        if (q2 == q) continue;
+        const int r2 = ord[q2];
+        int cmp;
+        if (!exact)
+          cmp = df_cmp_s(rec[r2], rec[row], a.bounds);  // never 0 here
+        else if (ovf || (rec[r2].flags_s & kRecOverflowS))
+          cmp = q2 < q ? -1 : 1;
+        else
+          cmp = cmp_s(rec[r2], rec[row]);
+        if (cmp < 0 || (cmp == 0 && r2 < row)) ++rank;
+      }
+      if (is_pick(lo + rank, m, k2, t, a.stride_interval)) fl[row] |= F_DIV;
+    }
+  }
+  __syncthreads();
+}
+
 // 3b. Stage II along ord, X_rem sorted by s (m rows): the stride picks
 //     (F_DIV), with uncertain neighbourhoods settled exactly.
 __device__ __forceinline__ void stage_two_picks(const SelectArgs &a, ImageCtx &c, const uint16_t *ord, const int m) {
@@ -2031,6 +2230,14 @@ __device__ __forceinline__ void stage_two_picks(const SelectArgs &a, ImageCtx &c
         fl[r] |= (uint8_t)(F_RUN | ((fl[r] & F_XS) ? 0 : want));
       }
       marked = true;
+      // every pick inside a run finds the same run; the first one records it
+      if (j == 0 || pick_position(j - 1, m, k2, t, a.stride_interval) < lo) {
+        RunList &rl = *c.runs;
+        const int slot = atomicAdd(&rl.count, 1);
+        if (slot < kMaxRuns) rl.run[slot] = ((uint32_t)lo << 16) | (uint32_t)hi;
+        atomicAdd(&rl.rows, hi - lo);
+        atomicMax(&rl.longest, hi - lo);
+      }
     }
   }
   if (__syncthreads_or(marked)) rank_pick_runs(a, c, ord, m, t);  // else every pick is certain
@@ -2038,24 +2245,48 @@ __device__ __forceinline__ void stage_two_picks(const SelectArgs &a, ImageCtx &c
 
 // 4. X* = X_imp union X_div in ascending token order (Eq. 7), plus outputs;
 //    the kept local indices are also left in ia (kept_rows).
+// The optional outputs of a row settled exactly (flags f): exact H2 and s,
+// and the non-finite / overflow counts.  Out of line: few rows have them.
+__device__ __noinline__ void emit_exact(const SelectArgs &a, const ExactRec &r, long long row, uint8_t f) {
+  int nonfinite = 0, overflow = 0;
+  if (f & F_XL) {
+    nonfinite |= (r.flags_l & kRecNonFiniteX) != 0;
+    overflow |= (r.flags_l & kRecOverflowL) != 0;
+    if (a.h2 && !(r.flags_l & kRecOverflowL)) a.h2[row] = exact_h2(r);
+  }
+  if (f & F_XS) {
+    nonfinite |= (r.flags_s & kRecNonFiniteS) != 0;
+    overflow |= (r.flags_s & kRecOverflowS) != 0;
+    if (a.s && !(r.flags_s & kRecOverflowS)) a.s[row] = (r.flags_s & kRecNonFiniteS) ? INFINITY : exact_s_key(r);
+  }
+  if (a.status) {
+    if (nonfinite) atomicAdd(&a.status[0], 1);
+    if (overflow) atomicAdd(&a.status[1], 1);
+  }
+}
+
 __device__ __forceinline__ void emit_outputs(const SelectArgs &a, ImageCtx &c) {
   const int tid = threadIdx.x;
-  const int nthr = blockDim.x;
   const int n = c.n;
   const long long off = c.off;
   uint16_t *ia = c.ia;
-  uint8_t *fl = c.fl;
-  ExactRec *rec = c.rec;
   const bool primary = c.primary;
   const int k = c.k, ko = c.ko;
-  const int per = (n + nthr - 1) / nthr;
+  const int per = stretch_rows(n);
   const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
+  uint32_t w[kStretchWords];
+  load_stretch(c.fl, i0, i1, w);
   int cnt = 0;
-  for (int i = i0; i < i1; ++i) cnt += (fl[i] & (F_IMP | F_DIV)) != 0;
+#pragma unroll
+  for (int j = 0; j < 4 * kStretchWords; ++j)
+    if (i0 + j < i1) cnt += (stretch_flag(w, j) & (F_IMP | F_DIV)) != 0;
   int kept_total = 0;
   int pos = ko + block_exclusive_scan(cnt, &kept_total);
-  for (int i = i0; i < i1; ++i) {
-    const uint8_t f = fl[i];
+#pragma unroll
+  for (int j = 0; j < 4 * kStretchWords; ++j) {
+    const int i = i0 + j;
+    if (i >= i1) break;
+    const uint8_t f = stretch_flag(w, j);
     if ((f & (F_IMP | F_DIV)) && pos < ko + k) {  // never write past this image's slots
       if (primary) a.idx[pos] = i;
       ia[pos - ko] = (uint16_t)i;
@@ -2063,25 +2294,7 @@ __device__ __forceinline__ void emit_outputs(const SelectArgs &a, ImageCtx &c) {
     }
     if (!primary) continue;
     if (a.role) a.role[off + i] = (f & F_IMP) ? 1 : ((f & F_DIV) ? 2 : 0);
-    int nonfinite = 0, overflow = 0;
-    if (f & F_XL) {
-      const ExactRec &r = rec[i];
-      nonfinite |= (r.flags_l & kRecNonFiniteX) != 0;
-      overflow |= (r.flags_l & kRecOverflowL) != 0;
-      if (a.h2 && !(r.flags_l & kRecOverflowL))
-        a.h2[off + i] = exact_h2(r);
-    }
-    if (f & F_XS) {
-      const ExactRec &r = rec[i];
-      nonfinite |= (r.flags_s & kRecNonFiniteS) != 0;
-      overflow |= (r.flags_s & kRecOverflowS) != 0;
-      if (a.s && !(r.flags_s & kRecOverflowS))
-        a.s[off + i] = (r.flags_s & kRecNonFiniteS) ? INFINITY : exact_s_key(r);
-    }
-    if (a.status) {
-      if (nonfinite) atomicAdd(&a.status[0], 1);
-      if (overflow) atomicAdd(&a.status[1], 1);
-    }
+    if (f & (F_XL | F_XS)) emit_exact(a, c.rec[i], off + i, f);
   }
   if (tid == 0 && kept_total != k && a.status && primary) atomicAdd(&a.status[3], 1);
   __syncthreads();
@@ -2089,11 +2302,17 @@ __device__ __forceinline__ void emit_outputs(const SelectArgs &a, ImageCtx &c) {
 
 // The selection of image b by one CTA (Algorithm 1 with exact decisions).
 __device__ void select_image(const SelectArgs &a, const int b, unsigned char *smem, const bool primary = true) {
+  __shared__ RunList runs;
   ImageCtx c;
   if (!image_ctx(a, b, smem, primary, c)) return;
+  c.runs = &runs;
   settle_unreliable(a, c, true, true);
   stage_one(a, c);
   if (c.need_s) {
+    if (threadIdx.x == 0) {  // read after the barriers of the listing and the sort
+      runs.count = runs.rows = runs.longest = 0;
+      runs.npend = runs.npend2 = 0;
+    }
     consistency_keys(a, c);
     const int m = list_rows(c, c.ia, true);
     const uint16_t *ord = sort_rows(c.key, c.ia, c.ib, c.bid, m, c.hist, false);
