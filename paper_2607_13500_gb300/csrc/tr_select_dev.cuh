@@ -61,8 +61,7 @@ __device__ __forceinline__ float key_r(const float *st) { return __ldcg(st + 6);
 __device__ __forceinline__ float key_s(const float *st) { return __ldcg(st + 7); }
 // Both keys in one 8-byte load (records are 32-byte aligned).
 __device__ __forceinline__ float2 key_rs(const float *st) { return __ldcg(reinterpret_cast<const float2 *>(st + 6)); }
-constexpr int kKeyIlp = 8;  // rows whose keys a thread loads before it uses any
-constexpr int kRowIlp = 4;  // rows a thread takes at a time in the shared-memory row passes
+constexpr int kKeyIlp = 4;  // rows whose keys a thread loads before it uses any
 
 // ---- a Big truncated to a 64-bit mantissa: value in [m 2^e, (m + 1) 2^e) ----
 // Integer-only (the GPU's fp64 rate is far too low for this path).
@@ -1375,39 +1374,27 @@ __device__ __noinline__ uint16_t *sample_sort(const uint32_t *key, uint16_t *a, 
 // and each row's final place is its bucket's start plus the number of
 // bucket members with a smaller (key, row), counted by one thread per row
 // (buckets hold about one row on the workloads here, at most kBucketMax).
-// Returns a, holding the order, or nullptr, having changed nothing but the
-// scratch bid (each position's bucket), when some bucket would hold more
-// than kBucketMax rows (ties, or keys crowded together), a key encodes NaN,
-// or the keys span no usable range: the caller then takes another sort.
-// hist: at least nb words.
+// Returns a, holding the order, or nullptr, having changed nothing, when
+// some bucket would hold more than kBucketMax rows (ties, or keys crowded
+// together), a key encodes NaN, or the keys span no usable range: the caller
+// then takes another sort.  hist: at least nb words.
 constexpr int kBucketMax = 32;
 constexpr int kBuckets = 4096;
 __device__ __forceinline__ float key_value(uint32_t k, bool complemented) {
   return complemented ? -unord32(~k) : unord32(k);
 }
-__device__ uint16_t *bucket_sort(const uint32_t *key, uint16_t *a, uint16_t *b, uint16_t *bid, int m, uint32_t *hist,
+__device__ uint16_t *bucket_sort(const uint32_t *key, uint16_t *a, uint16_t *b, int m, uint32_t *hist,
                                  bool complemented) {
   __shared__ float sh_min[kWarps], sh_max[kWarps];
   __shared__ int sh_big;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nthr = blockDim.x;
-  // Every pass over the rows takes kRowIlp of them per thread at a time,
-  // their loads first, so that the shared-memory latencies overlap.
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   float vmin = INFINITY, vmax = -INFINITY;
   bool nan = false;
-  for (int q0 = tid; q0 < m; q0 += kRowIlp * nthr) {
-    uint16_t r[kRowIlp];
-    uint32_t k[kRowIlp];
-#pragma unroll
-    for (int u = 0; u < kRowIlp; ++u) r[u] = a[min(q0 + u * nthr, m - 1)];  // repeats are harmless here
-#pragma unroll
-    for (int u = 0; u < kRowIlp; ++u) k[u] = key[r[u]];
-#pragma unroll
-    for (int u = 0; u < kRowIlp; ++u) {
-      const float v = key_value(k[u], complemented);
-      vmin = fminf(vmin, v);
-      vmax = fmaxf(vmax, v);
-      nan |= v != v;
-    }
+  for (int q = tid; q < m; q += blockDim.x) {
+    const float v = key_value(key[a[q]], complemented);
+    vmin = fminf(vmin, v);
+    vmax = fmaxf(vmax, v);
+    nan |= v != v;
   }
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
@@ -1420,7 +1407,7 @@ __device__ uint16_t *bucket_sort(const uint32_t *key, uint16_t *a, uint16_t *b, 
   }
   int nb = 64;
   while (nb < m && nb < kBuckets) nb <<= 1;
-  for (int c = tid; c < nb; c += nthr) hist[c] = 0u;
+  for (int c = tid; c < nb; c += blockDim.x) hist[c] = 0u;
   if (tid == 0) sh_big = 0;
   __syncthreads();
   if (__syncthreads_or(nan)) return nullptr;  // uniform; NaN has no place in a linear bucket map
@@ -1435,27 +1422,10 @@ __device__ uint16_t *bucket_sort(const uint32_t *key, uint16_t *a, uint16_t *b, 
   if (!(span > 0.f) || !isfinite(span) || !isfinite(scale)) return nullptr;  // uniform: all equal or no usable range
   // bucket of a value: floor((v - vmin) * scale), monotone in v, clamped to the last bucket
   auto bucket = [&](float v) { return min(nb - 1, (int)((v - vmin) * scale)); };
-  // counts per bucket; each position's bucket is kept in bid for the scatter
-  for (int q0 = tid; q0 < m; q0 += kRowIlp * nthr) {
-    uint16_t r[kRowIlp];
-    uint32_t k[kRowIlp];
-#pragma unroll
-    for (int u = 0; u < kRowIlp; ++u) r[u] = a[min(q0 + u * nthr, m - 1)];
-#pragma unroll
-    for (int u = 0; u < kRowIlp; ++u) k[u] = key[r[u]];
-#pragma unroll
-    for (int u = 0; u < kRowIlp; ++u) {
-      const int q = q0 + u * nthr;
-      if (q < m) {
-        const int c = bucket(key_value(k[u], complemented));
-        bid[q] = (uint16_t)c;
-        atomicAdd(&hist[c], 1u);
-      }
-    }
-  }
+  for (int q = tid; q < m; q += blockDim.x) atomicAdd(&hist[bucket(key_value(key[a[q]], complemented))], 1u);
   __syncthreads();
   // exclusive scan of the bucket counts (each thread a contiguous stretch) and the largest count
-  const int per = (nb + nthr - 1) / nthr;
+  const int per = (nb + blockDim.x - 1) / blockDim.x;
   const int c0 = min(nb, tid * per), c1 = min(nb, c0 + per);
   int run = 0, big = 0;
   for (int c = c0; c < c1; ++c) {
@@ -1472,54 +1442,24 @@ __device__ uint16_t *bucket_sort(const uint32_t *key, uint16_t *a, uint16_t *b, 
     base += cnt;
   }
   __syncthreads();
-  for (int q0 = tid; q0 < m; q0 += kRowIlp * nthr) {
-    uint16_t r[kRowIlp], c[kRowIlp];
-    uint32_t pos[kRowIlp];
-#pragma unroll
-    for (int u = 0; u < kRowIlp; ++u) {
-      const int q = min(q0 + u * nthr, m - 1);
-      r[u] = a[q];
-      c[u] = bid[q];
-    }
-#pragma unroll
-    for (int u = 0; u < kRowIlp; ++u)
-      if (q0 + u * nthr < m) pos[u] = atomicAdd(&hist[c[u]], 1u);
-#pragma unroll
-    for (int u = 0; u < kRowIlp; ++u)
-      if (q0 + u * nthr < m) b[pos[u]] = r[u];
+  for (int q = tid; q < m; q += blockDim.x) {
+    const uint16_t row = a[q];
+    b[atomicAdd(&hist[bucket(key_value(key[row], complemented))], 1u)] = row;
   }
   __syncthreads();
-  // hist[c] is now the end of bucket c, so bucket c spans [hist[c - 1], hist[c]);
-  // a row's place is its bucket's start plus the members with a smaller composite key
-  for (int q0 = tid; q0 < m; q0 += kRowIlp * nthr) {
-    uint16_t row[kRowIlp];
-    uint32_t kr[kRowIlp];
-    int lo[kRowIlp], hi[kRowIlp];
-#pragma unroll
-    for (int u = 0; u < kRowIlp; ++u) row[u] = b[min(q0 + u * nthr, m - 1)];
-#pragma unroll
-    for (int u = 0; u < kRowIlp; ++u) kr[u] = key[row[u]];
-#pragma unroll
-    for (int u = 0; u < kRowIlp; ++u) {
-      const int c = bucket(key_value(kr[u], complemented));
-      lo[u] = c ? (int)hist[c - 1] : 0;
-      hi[u] = (int)hist[c];
+  // hist[c] is now the end of bucket c, so bucket c spans [hist[c - 1], hist[c])
+  for (int q = tid; q < m; q += blockDim.x) {
+    const uint16_t row = b[q];
+    const uint32_t kr = key[row];
+    const int c = bucket(key_value(kr, complemented));
+    const int lo = c ? (int)hist[c - 1] : 0, hi = (int)hist[c];
+    const unsigned long long kk = ((unsigned long long)kr << 16) | row;
+    int rank = 0;
+    for (int j = lo; j < hi; ++j) {
+      const uint16_t r2 = b[j];
+      rank += (((unsigned long long)key[r2] << 16) | r2) < kk;
     }
-#pragma unroll
-    for (int u = 0; u < kRowIlp; ++u) {
-      int rank = 0;
-      if (hi[u] - lo[u] > 1) {
-        const unsigned long long kk = ((unsigned long long)kr[u] << 16) | row[u];
-        for (int j = lo[u]; j < hi[u]; ++j) {
-          const uint16_t r2 = b[j];
-          rank += (((unsigned long long)key[r2] << 16) | r2) < kk;
-        }
-      }
-      lo[u] += rank;
-    }
-#pragma unroll
-    for (int u = 0; u < kRowIlp; ++u)
-      if (q0 + u * nthr < m) a[lo[u]] = row[u];
+    a[lo + rank] = row;
   }
   __syncthreads();
   return a;
@@ -1543,7 +1483,7 @@ __device__ uint16_t *sort_rows(const uint32_t *key, uint16_t *a, uint16_t *b, ui
       sort_small<1>(key, a, m, scratch);
     return a;
   }
-  if (uint16_t *o = bucket_sort(key, a, b, bid, m, hist, complemented)) return o;
+  if (uint16_t *o = bucket_sort(key, a, b, m, hist, complemented)) return o;
   if (m <= 2 * kSelectThreads) {
     __syncthreads();
     sort_small<2>(key, a, m, scratch);
@@ -1581,13 +1521,9 @@ __device__ uint32_t select_rank(const uint32_t *key, int n, int r, uint32_t *his
     uint32_t *h = hist + warp * 256;
     for (int d = lane; d < 256; d += 32) h[d] = 0u;
     __syncwarp();
-    for (int i0 = tid; i0 < n; i0 += kRowIlp * blockDim.x) {
-      uint32_t k[kRowIlp];
-#pragma unroll
-      for (int u = 0; u < kRowIlp; ++u) k[u] = key[min(i0 + u * (int)blockDim.x, n - 1)];
-#pragma unroll
-      for (int u = 0; u < kRowIlp; ++u)
-        if (i0 + u * (int)blockDim.x < n && (k[u] & mask) == pre) atomicAdd(&h[(k[u] >> shift) & 0xffu], 1u);
+    for (int i = tid; i < n; i += blockDim.x) {
+      const uint32_t k = key[i];
+      if ((k & mask) == pre) atomicAdd(&h[(k >> shift) & 0xffu], 1u);
     }
     __syncthreads();
     if (tid < 256) {  // column tid: only this thread reads or writes it here
@@ -1631,6 +1567,102 @@ __device__ uint32_t select_rank(const uint32_t *key, int n, int r, uint32_t *his
   *lt = r - rr;
   *eq = sh_eq;
   return pre;
+}
+
+// The same selection by value buckets, in one pass over the keys instead of
+// four: the value each key encodes (-R for the complemented importance
+// keys, so ascending keys are ascending values) is mapped linearly from
+// [vmin, vmax] onto nb buckets (a monotone map: equal keys share a bucket,
+// and a smaller key never lands in a later bucket); a scan of the bucket
+// counts finds the bucket holding position r, and one warp ranks its
+// members.  Returns false, having set nothing, when the values span no
+// usable range or that bucket holds more than 32 keys (the caller then
+// takes the radix selection).  hist: at least kBuckets words.
+__device__ bool select_rank_buckets(const uint32_t *key, int n, int r, uint32_t *hist, float vmin, float vmax,
+                                    uint32_t *t_out, int *lt, int *eq) {
+  __shared__ int sh_c, sh_before, sh_cnt, sh_lt, sh_eq;
+  __shared__ uint32_t sh_mem[32], sh_t;
+  const int tid = threadIdx.x, nthr = blockDim.x, lane = tid & 31;
+  int nb = 64;
+  while (nb < n && nb < kBuckets) nb <<= 1;
+  const float span = vmax - vmin, scale = (float)nb / span;
+  if (!(span > 0.f) || !isfinite(span) || !isfinite(scale)) return false;  // uniform
+  auto bucket = [&](uint32_t k) { return min(nb - 1, max(0, (int)((key_value(k, true) - vmin) * scale))); };
+  __syncthreads();  // hist may still be read by the caller's previous step
+  for (int c = tid; c < nb; c += nthr) hist[c] = 0u;
+  if (tid == 0) sh_cnt = 0;
+  __syncthreads();
+  for (int i = tid; i < n; i += nthr) atomicAdd(&hist[bucket(key[i])], 1u);
+  __syncthreads();
+  // the bucket holding position r: each thread sums a stretch of buckets
+  const int per = (nb + nthr - 1) / nthr;
+  const int c0 = min(nb, tid * per), c1 = min(nb, c0 + per);
+  int run = 0;
+  for (int c = c0; c < c1; ++c) run += (int)hist[c];
+  int total = 0;
+  int base = block_exclusive_scan(run, &total);
+  if (base <= r && r < base + run) {
+    for (int c = c0; c < c1; ++c) {
+      const int h = (int)hist[c];
+      if (r < base + h) {
+        sh_c = c;
+        sh_before = base;
+        break;
+      }
+      base += h;
+    }
+  }
+  __syncthreads();
+  const int cstar = sh_c, before = sh_before, members = (int)hist[cstar];
+  if (members > 32) return false;  // uniform
+  for (int i = tid; i < n; i += nthr) {
+    const uint32_t k = key[i];
+    if (bucket(k) == cstar) sh_mem[atomicAdd(&sh_cnt, 1)] = k;
+  }
+  __syncthreads();
+  if (tid < 32) {
+    const uint32_t mk = lane < members ? sh_mem[lane] : 0xffffffffu;
+    int less = 0, same = 0;
+    for (int j = 0; j < members; ++j) {
+      const uint32_t o = __shfl_sync(0xffffffffu, mk, j);
+      less += o < mk;
+      same += o == mk;
+    }
+    const int rr = r - before;  // position r inside the bucket
+    if (lane < members && less <= rr && rr < less + same) {  // lanes holding equal keys write the same
+      sh_t = mk;
+      sh_lt = before + less;
+      sh_eq = same;
+    }
+  }
+  __syncthreads();
+  *t_out = sh_t;
+  *lt = sh_lt;
+  *eq = sh_eq;
+  return true;
+}
+
+// Block-wide minimum and maximum (every thread receives both).
+__device__ void block_min_max(float &vmin, float &vmax) {
+  __shared__ float smin[32], smax[32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nwarps = blockDim.x >> 5;
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    vmin = fminf(vmin, __shfl_xor_sync(0xffffffffu, vmin, o));
+    vmax = fmaxf(vmax, __shfl_xor_sync(0xffffffffu, vmax, o));
+  }
+  __syncthreads();  // smin / smax may still be read by a previous call
+  if (lane == 0) {
+    smin[warp] = vmin;
+    smax[warp] = vmax;
+  }
+  __syncthreads();
+  vmin = smin[0];
+  vmax = smax[0];
+  for (int w = 1; w < nwarps; ++w) {
+    vmin = fminf(vmin, smin[w]);
+    vmax = fmaxf(vmax, smax[w]);
+  }
 }
 
 // Smallest key[i] (i < n) above t, or 0xffffffff when there is none.
@@ -1692,6 +1724,8 @@ struct ImageCtx {
   long long off;
   int n, k, k1, k2, ko;
   bool need_r, need_s, primary;
+  bool any_exact;    // some row was settled exactly up front
+  float vmin, vmax;  // range of -R32 over the rows with a float key
   uint32_t *key, *hist;
   uint16_t *ia, *ib, *bid;
   uint8_t *fl;
@@ -1760,6 +1794,8 @@ __device__ __forceinline__ void settle_unreliable(const SelectArgs &a, ImageCtx 
   ExactRec *rec = c.rec;
   const bool primary = c.primary;
   const bool need_r = c.need_r, need_s = c.need_s;
+  bool any = false;
+  float vmin = INFINITY, vmax = -INFINITY;
   for (int i0 = tid; i0 < n; i0 += kKeyIlp * nthr) {
     float2 kk[kKeyIlp];
 #pragma unroll
@@ -1774,16 +1810,25 @@ __device__ __forceinline__ void settle_unreliable(const SelectArgs &a, ImageCtx 
         uint8_t f = 0;
         if (want_l && (need_r || a.h2) && isnan(kk[u].x)) f |= F_NEEDL;
         if (want_s && (need_s || a.s) && isnan(kk[u].y)) f |= F_NEEDS;
+        any |= f != 0;
         fl[i] = f;
         key[i] = ~ord32(kk[u].x);
         ia[i] = (uint16_t)i;
+        if (kk[u].x == kk[u].x) {  // the value stage I's bucket map sees: -R
+          vmin = fminf(vmin, -kk[u].x);
+          vmax = fmaxf(vmax, -kk[u].x);
+        }
       }
     }
   }
-  __syncthreads();
-  refine_pending(a, off, n, fl, rec, primary);
-  __syncthreads();
-
+  block_min_max(vmin, vmax);  // its barriers also publish fl, key and ia
+  c.vmin = vmin;
+  c.vmax = vmax;
+  c.any_exact = __syncthreads_or(any);
+  if (c.any_exact) {
+    refine_listed(a, off, n, fl, rec, primary);
+    __syncthreads();
+  }
 }
 
 // Stage I when the K1-th and (K1+1)-th keys are not certainly ordered (t1:
@@ -1948,33 +1993,28 @@ __device__ __forceinline__ void stage_one(const SelectArgs &a, ImageCtx &c) {
   const int k1 = c.k1;
   const bool need_r = c.need_r;
   if (need_r) {
-    for (int i = tid; i < n; i += nthr)  // rows settled exactly carry their exact key
-      if (fl[i] & F_XL) key[i] = ~ord32(exact_r_key(rec[i]));
-    __syncthreads();
-    // Fast path: the K1-th and (K1+1)-th keys by radix selection; when they
-    // differ and their order is certain, the top K1 are exactly the rows
-    // with a key up to the K1-th, and no order is needed.
+    if (c.any_exact) {  // rows settled exactly carry their exact key (the
+                        // bucket map clamps it into range: still monotone)
+      for (int i = tid; i < n; i += nthr)
+        if (fl[i] & F_XL) key[i] = ~ord32(exact_r_key(rec[i]));
+      __syncthreads();
+    }
+    const float vmin = c.vmin, vmax = c.vmax;
+    // Fast path: the K1-th and (K1+1)-th keys (by value buckets, else radix
+    // selection); when they differ and their order is certain, the top K1
+    // are exactly the rows with a key up to the K1-th, and no order is needed.
     int lt = 0, eq = 0;
-    const uint32_t t1 = select_rank(key, n, k1 - 1, hist, &lt, &eq);
+    uint32_t t1 = 0u;
+    if (!select_rank_buckets(key, n, k1 - 1, hist, vmin, vmax, &t1, &lt, &eq))
+      t1 = select_rank(key, n, k1 - 1, hist, &lt, &eq);
     bool settled = false;
     if (lt + eq == k1) {
       const uint32_t t2 = block_min_above(key, n, t1);
       settled = cert_r_val(unord32(~t1), unord32(~t2), a.bounds);
     }
     if (settled) {
-      for (int i0 = tid; i0 < n; i0 += kRowIlp * nthr) {
-        uint32_t k[kRowIlp];
-        uint8_t f[kRowIlp];
-#pragma unroll
-        for (int u = 0; u < kRowIlp; ++u) {
-          const int i = min(i0 + u * nthr, n - 1);
-          k[u] = key[i];
-          f[u] = fl[i];
-        }
-#pragma unroll
-        for (int u = 0; u < kRowIlp; ++u)
-          if (i0 + u * nthr < n && k[u] <= t1) fl[i0 + u * nthr] = (uint8_t)(f[u] | F_IMP);
-      }
+      for (int i = tid; i < n; i += nthr)
+        if (key[i] <= t1) fl[i] |= F_IMP;
       __syncthreads();
     } else {
       resolve_cut(a, c, t1);
@@ -2015,38 +2055,19 @@ __device__ __forceinline__ void consistency_keys(const SelectArgs &a, ImageCtx &
   }
 }
 
-// Row passes in index order give each thread a contiguous stretch of rows,
-// a multiple of 4 long (at most 32), whose flags it loads as 32-bit words
-// before using any (the flags array is 16-byte aligned).
-constexpr int kStretchWords = 8;
-static_assert(TR_MAX_N <= 4 * kStretchWords * kSelectThreads, "a stretch holds at most 32 rows");
-__device__ __forceinline__ int stretch_rows(int n) { return 4 * ((n + 4 * kSelectThreads - 1) / (4 * kSelectThreads)); }
-__device__ __forceinline__ void load_stretch(const uint8_t *fl, int i0, int i1, uint32_t (&w)[kStretchWords]) {
-  const uint32_t *fw = reinterpret_cast<const uint32_t *>(fl + i0);
-#pragma unroll
-  for (int j = 0; j < kStretchWords; ++j) w[j] = i0 + 4 * j < i1 ? fw[j] : 0u;
-}
-__device__ __forceinline__ uint8_t stretch_flag(const uint32_t (&w)[kStretchWords], int j) {
-  return (uint8_t)((w[j >> 2] >> (8 * (j & 3))) & 0xffu);
-}
-
 // The rows of the image (all, or those outside X_imp) in ascending index
 // order -- the stable sort's tie order -- into dst; returns their number.
 __device__ __forceinline__ int list_rows(ImageCtx &c, uint16_t *dst, const bool skip_imp) {
-  const int tid = threadIdx.x, n = c.n;
-  const int per = stretch_rows(n);
+  const int tid = threadIdx.x, nthr = blockDim.x, n = c.n;
+  const uint8_t *fl = c.fl;
+  const int per = (n + nthr - 1) / nthr;
   const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
-  uint32_t w[kStretchWords];
-  load_stretch(c.fl, i0, i1, w);
   int cnt = 0;
-#pragma unroll
-  for (int j = 0; j < 4 * kStretchWords; ++j)
-    if (i0 + j < i1) cnt += !(skip_imp && (stretch_flag(w, j) & F_IMP));
+  for (int i = i0; i < i1; ++i) cnt += !(skip_imp && (fl[i] & F_IMP));
   int m = 0;
   int pos = block_exclusive_scan(cnt, &m);
-#pragma unroll
-  for (int j = 0; j < 4 * kStretchWords; ++j)
-    if (i0 + j < i1 && !(skip_imp && (stretch_flag(w, j) & F_IMP))) dst[pos++] = (uint16_t)(i0 + j);
+  for (int i = i0; i < i1; ++i)
+    if (!(skip_imp && (fl[i] & F_IMP))) dst[pos++] = (uint16_t)i;
   __syncthreads();
   return m;
 }
@@ -2245,48 +2266,24 @@ __device__ __forceinline__ void stage_two_picks(const SelectArgs &a, ImageCtx &c
 
 // 4. X* = X_imp union X_div in ascending token order (Eq. 7), plus outputs;
 //    the kept local indices are also left in ia (kept_rows).
-// The optional outputs of a row settled exactly (flags f): exact H2 and s,
-// and the non-finite / overflow counts.  Out of line: few rows have them.
-__device__ __noinline__ void emit_exact(const SelectArgs &a, const ExactRec &r, long long row, uint8_t f) {
-  int nonfinite = 0, overflow = 0;
-  if (f & F_XL) {
-    nonfinite |= (r.flags_l & kRecNonFiniteX) != 0;
-    overflow |= (r.flags_l & kRecOverflowL) != 0;
-    if (a.h2 && !(r.flags_l & kRecOverflowL)) a.h2[row] = exact_h2(r);
-  }
-  if (f & F_XS) {
-    nonfinite |= (r.flags_s & kRecNonFiniteS) != 0;
-    overflow |= (r.flags_s & kRecOverflowS) != 0;
-    if (a.s && !(r.flags_s & kRecOverflowS)) a.s[row] = (r.flags_s & kRecNonFiniteS) ? INFINITY : exact_s_key(r);
-  }
-  if (a.status) {
-    if (nonfinite) atomicAdd(&a.status[0], 1);
-    if (overflow) atomicAdd(&a.status[1], 1);
-  }
-}
-
 __device__ __forceinline__ void emit_outputs(const SelectArgs &a, ImageCtx &c) {
   const int tid = threadIdx.x;
+  const int nthr = blockDim.x;
   const int n = c.n;
   const long long off = c.off;
   uint16_t *ia = c.ia;
+  uint8_t *fl = c.fl;
+  ExactRec *rec = c.rec;
   const bool primary = c.primary;
   const int k = c.k, ko = c.ko;
-  const int per = stretch_rows(n);
+  const int per = (n + nthr - 1) / nthr;
   const int i0 = min(n, tid * per), i1 = min(n, i0 + per);
-  uint32_t w[kStretchWords];
-  load_stretch(c.fl, i0, i1, w);
   int cnt = 0;
-#pragma unroll
-  for (int j = 0; j < 4 * kStretchWords; ++j)
-    if (i0 + j < i1) cnt += (stretch_flag(w, j) & (F_IMP | F_DIV)) != 0;
+  for (int i = i0; i < i1; ++i) cnt += (fl[i] & (F_IMP | F_DIV)) != 0;
   int kept_total = 0;
   int pos = ko + block_exclusive_scan(cnt, &kept_total);
-#pragma unroll
-  for (int j = 0; j < 4 * kStretchWords; ++j) {
-    const int i = i0 + j;
-    if (i >= i1) break;
-    const uint8_t f = stretch_flag(w, j);
+  for (int i = i0; i < i1; ++i) {
+    const uint8_t f = fl[i];
     if ((f & (F_IMP | F_DIV)) && pos < ko + k) {  // never write past this image's slots
       if (primary) a.idx[pos] = i;
       ia[pos - ko] = (uint16_t)i;
@@ -2294,7 +2291,25 @@ __device__ __forceinline__ void emit_outputs(const SelectArgs &a, ImageCtx &c) {
     }
     if (!primary) continue;
     if (a.role) a.role[off + i] = (f & F_IMP) ? 1 : ((f & F_DIV) ? 2 : 0);
-    if (f & (F_XL | F_XS)) emit_exact(a, c.rec[i], off + i, f);
+    int nonfinite = 0, overflow = 0;
+    if (f & F_XL) {
+      const ExactRec &r = rec[i];
+      nonfinite |= (r.flags_l & kRecNonFiniteX) != 0;
+      overflow |= (r.flags_l & kRecOverflowL) != 0;
+      if (a.h2 && !(r.flags_l & kRecOverflowL))
+        a.h2[off + i] = exact_h2(r);
+    }
+    if (f & F_XS) {
+      const ExactRec &r = rec[i];
+      nonfinite |= (r.flags_s & kRecNonFiniteS) != 0;
+      overflow |= (r.flags_s & kRecOverflowS) != 0;
+      if (a.s && !(r.flags_s & kRecOverflowS))
+        a.s[off + i] = (r.flags_s & kRecNonFiniteS) ? INFINITY : exact_s_key(r);
+    }
+    if (a.status) {
+      if (nonfinite) atomicAdd(&a.status[0], 1);
+      if (overflow) atomicAdd(&a.status[1], 1);
+    }
   }
   if (tid == 0 && kept_total != k && a.status && primary) atomicAdd(&a.status[3], 1);
   __syncthreads();
