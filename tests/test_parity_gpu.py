@@ -686,6 +686,25 @@ def test_near_ties_beyond_fp32(dtype):
         assert 0 < st[2] <= 6, st
 
 
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float16, torch.float32], ids=["bf16", "f16", "f32"])
+def test_small_uniform_batches(dtype):
+    # Small uniform batches through tr_reduce (scoring, then the replicated
+    # selection and copy of k_select_gather): image sizes that are and are
+    # not multiples of the select kernel's 16 warps, three input types, and
+    # a second call on the same workspace and outputs.
+    for batch, n, d, k, k1 in [(5, 40, 256, 12, 4), (2, 16, 512, 6, 2), (3, 576, 1024, 64, 21)]:
+        x, xp, xq = _rows(batch * n, d, 40 + n, dtype)
+        seqlens = [n] * batch
+        budget = ([k] * batch, [k1] * batch, [k * b for b in range(batch + 1)])
+        altr = _alt()
+        red = altr.Reducer(seqlens, d, dtype, "cuda", budget=budget, scores=True)
+        dx, dp, dq = x.cuda(), xp.cuda(), xq.cuda()
+        for _ in range(2):
+            r = red.run(dx, dp, dq)
+            torch.cuda.synchronize()
+            compare_result(r, x, xp, xq, seqlens, budget)
+
+
 def test_fp32_wide_range():
     n, d = 300, 1024
     g = torch.Generator().manual_seed(5)
