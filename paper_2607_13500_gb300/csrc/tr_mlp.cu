@@ -29,14 +29,13 @@
 // The projector mode (tr_project_kept) is the hidden GEMM with its A rows
 // gathered: A row j is token idx[j] of the image that owns kept slot j, so
 // the first projector layer reads X* = X_imp union X_div (Eq. 7) straight
-// from x without a gathered copy.  Four more warps (10-13) move those rows
-// with 16-byte cp.async copies into the 128-byte-swizzled layout TMA would
-// have written (chunk c of row r at r * 128 + ((c ^ (r & 7)) << 4)), eight
-// threads to a row so that each warp copy reads whole 128-byte segments; a
-// copier waits for its copies of a stage and fences them into the async
-// proxy the tensor cores read through, and once its whole warp has, one lane
-// arrives on the stage's barrier -- some stages behind the issue, so that
-// copies stay in flight.
+// from x without a gathered copy.  Four more warps (10-13) bring those rows:
+// lane l of warp w issues, for row 32 w + l of each A k-block, a tiled TMA
+// load of one 64-element row of x (a one-row box, 128-byte swizzle, so the
+// row lands in the layout the tensor cores read: the swizzle follows the
+// shared-memory address); a slot past the kept rows loads row -1, which
+// reads zeros.  Each loader warp's lane 0 adds its rows' bytes to the
+// stage's transaction count and arrives once.
 //
 // The epilogue of tile i overlaps the main loop of tile i + 1 (two TMEM
 // accumulators).  A row's sums over its 2 n_tiles column halves are
@@ -63,14 +62,10 @@ constexpr int kBTile = kBN * kBK * 2;             // bytes of one B k-block
 constexpr int kStageBytes = kATile + kBTile;      // 48 KiB
 constexpr int kEpiWarps = 8;                      // two warpgroups: column halves of a tile
 enum { kModeHidden = 0, kModeScore = 1, kModeProject = 2 };
-// producer, MMA issuer, epilogue (+ the four A copiers of the projector mode)
-__host__ __device__ constexpr int gemm_threads(int mode) { return 64 + 32 * kEpiWarps + (mode == 2 ? 128 : 0); }
-// Stages a copier keeps in flight before it signals the oldest: two fewer
-// than the ring holds (a copier issues stage s + lag only after the MMAs have
-// released that slot, i.e. consumed stage s + lag - stages < s, which it has
-// already signalled).
-constexpr int kCopyLag = 2;     // one SM: 4-stage ring
-constexpr int kCopyLagP = 4;    // SM pair: 6-stage ring
+// producer, MMA issuer, epilogue (+ the A-row loaders of the projector mode)
+constexpr int kCopyWarps = 4;                      // projector: A-row loader warps, one row per lane
+static_assert(kCopyWarps * 32 == kBM, "the loaders' lanes cover a tile's rows");
+__host__ __device__ constexpr int gemm_threads(int mode) { return 64 + 32 * kEpiWarps + (mode == 2 ? 32 * kCopyWarps : 0); }
 constexpr int kTmemCols = 2 * kBN;                // two accumulators
 constexpr int kChunk = 16;                        // columns per tcgen05.ld
 constexpr int kPartWords = 10;                    // hi, lo of L1, S2, A, B, P
@@ -382,17 +377,6 @@ __device__ __forceinline__ void publish_rows(const GemmArgs &g, int rb, int nt, 
   if (lane == 0) g.arrivals[rb * 4 + q] = 0;  // ready for the next launch
 }
 
-// cp.async of 16 bytes (src_bytes = 0: zero fill, nothing read) and its groups.
-__device__ __forceinline__ void cp_async16(uint32_t dst, const void *src, uint32_t src_bytes) {
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes) : "memory");
-}
-__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int kN>
-__device__ __forceinline__ void cp_async_wait() {
-  asm volatile("cp.async.wait_group %0;" ::"n"(kN) : "memory");
-}
-__device__ __forceinline__ void fence_proxy_async() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
-
 // Row of x that kept slot j names (projector mode), or -1: the image b with
 // cu_k[b] <= j < cu_k[b + 1], its local index idx[j] checked against the
 // image's tokens (an index outside them gives a zero row, never another
@@ -435,7 +419,7 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      tc::mbar_init(full(s), kMode == kModeProject ? 1 + 4 : 1);  // + one arrival per copier warp
+      tc::mbar_init(full(s), kMode == kModeProject ? 1 + kCopyWarps : 1);  // + one arrival per loader warp
       tc::mbar_init(empty(s), 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -469,7 +453,7 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
           break;
         }
         if (lane == 0) {
-          if (kMode == kModeProject) {  // A comes from the copiers
+          if (kMode == kModeProject) {  // A comes from the row loaders
             tc::mbar_expect_tx(full(stage), kBTile);
           } else {
             tc::mbar_expect_tx(full(stage), kStageBytes);
@@ -533,38 +517,25 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
     __syncwarp();
     tc::mbar_wait_warp(done, 0);
   } else if (kMode == kModeProject && warp >= 2 + kEpiWarps) {
-    // ---------------------------------------------------------------- A copiers (projector mode)
-    const int t = (int)threadIdx.x - 32 * (2 + kEpiWarps);
-    const int c = t & 7;  // this thread's 16-byte unit of each row's 128-byte k-block segment
-    int stage = 0, pending = 0;  // stages copied into but not yet signalled: stage - pending ... stage - 1
+    // ---------------------------------------------------------------- A rows (projector mode)
+    // lane l of loader warp w brings row 32 w + l of each A k-block by a
+    // one-row TMA load (a row past the kept slots, coordinate -1, reads zeros)
+    const int r = (warp - 2 - kEpiWarps) * 32 + lane;
+    int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < g.tiles && ok; tile += gridDim.x) {
       const int rb = tile / g.n_tiles;
-      long long src[8];  // rows (t >> 3) + 16 i of the tile: 8 threads per row, whole 128-byte segments per warp
-#pragma unroll
-      for (int i = 0; i < 8; ++i) src[i] = kept_source_row(g, (long long)rb * kBM + (t >> 3) + 16 * i);
+      const long long src = kept_source_row(g, (long long)rb * kBM + r);
+      const int srow = src >= 0 ? (int)src : -1;
       for (int kb = 0; kb < g.kblocks; ++kb) {
         if (!tc::mbar_wait_warp(empty(stage), phase ^ 1u)) {
           ok = false;
           break;
         }
-        const int col = kb * kBK + c * 8;
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const int r = (t >> 3) + 16 * i;
-          const bool in = src[i] >= 0 && col < g.k;
-          cp_async16(sa(stage) + (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4)), in ? g.gx + src[i] * g.k + col : g.gx,
-                     in ? 16u : 0u);
-        }
-        cp_async_commit();
-        if (++pending > kCopyLag) {  // the copies of the stage issued kCopyLag stages ago are complete
-          cp_async_wait<kCopyLag>();
-          fence_proxy_async();
-          __syncwarp();  // the warp's copies of that stage are complete and fenced: one arrival
-          if (lane == 0) tc::mbar_arrive(full((stage - kCopyLag + kStages) % kStages));
-          --pending;
-        }
+        if (lane == 0) tc::mbar_expect_tx(full(stage), 32 * kBK * 2);  // this warp's 32 rows; one arrival
+        __syncwarp();
+        tc::tma_load_2d(sa(stage) + (uint32_t)(r * kBK * 2), &map_a, kb * kBK, srow, full(stage));
         if (++stage == kStages) {
           stage = 0;
           phase ^= 1u;
@@ -572,11 +543,6 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
       }
     }
     if (!ok && lane == 0) flag_error(g, 8);
-    cp_async_wait<0>();
-    fence_proxy_async();
-    __syncwarp();
-    if (lane == 0)
-      for (int i = pending; i > 0; --i) tc::mbar_arrive(full((stage - i + kStages) % kStages));
   } else {
     // ---------------------------------------------------------------- epilogue
     const int q = warp & 3;            // TMEM lane quadrant this warp may read
@@ -630,7 +596,6 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
 // brings 32 KiB of operands for a 128 x 256 x 64 product, against 48 KiB on
 // one SM, so six stages in flight hide the load latency that four did not.
 constexpr int kStagesP = 6;
-static_assert(kCopyLagP < kStagesP && kCopyLag < kStages, "a copier must signal a stage before it needs its slot again");
 constexpr int kHalfTile = 128 * kBK * 2;          // 128 rows of a k-block (A or B)
 constexpr int kStagePBytes = 2 * kHalfTile;       // this CTA's A rows + B rows
 constexpr uint32_t kIdescPair = tc::idesc_bf16(2 * kBM, kBN);
@@ -664,7 +629,7 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
   constexpr uint32_t kTx = kMode == kModeProject ? 2 * kHalfTile : 2 * kStagePBytes;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStagesP; ++s) {
-      tc::mbar_init(full(s), kMode == kModeProject ? 1 + 2 * 4 : 1);  // + both CTAs' copier warps
+      tc::mbar_init(full(s), kMode == kModeProject ? 1 + kCopyWarps : 1);  // + the even CTA's loader warps
       tc::mbar_init(empty(s), 1);
     }
     for (int a = 0; a < 2; ++a) {
@@ -767,39 +732,26 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
     }
     tc::mbar_wait_warp(done, 0);  // every pair MMA has completed (both CTAs' TMEM)
   } else if (kMode == kModeProject && warp >= 2 + kEpiWarps) {
-    // ---------------------------------------------------------------- A copiers (projector mode)
-    const int t = (int)threadIdx.x - 32 * (2 + kEpiWarps);
-    const int c = t & 7;  // as in the one-SM kernel: 8 threads per row
-    int stage = 0, pending = 0;
+    // ---------------------------------------------------------------- A rows (projector mode)
+    // as in the one-SM kernel, into this CTA's half of the pair's rows; the
+    // loads land on the even CTA's barrier, whose loader warps expect both
+    // CTAs' bytes (the odd CTA's loader warps do not arrive)
+    const int r = (warp - 2 - kEpiWarps) * 32 + lane;
+    int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
     for (int tile = cluster; tile < tiles && ok; tile += clusters) {
       const int rb = tile / g.n_tiles;
-      long long src[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i)
-        src[i] = kept_source_row(g, (long long)rb * 2 * kBM + (long long)rank * kBM + (t >> 3) + 16 * i);
+      const long long src = kept_source_row(g, (long long)rb * 2 * kBM + (long long)rank * kBM + r);
+      const int srow = src >= 0 ? (int)src : -1;
       for (int kb = 0; kb < g.kblocks; ++kb) {
         if (!tc::mbar_wait_warp(empty(stage), phase ^ 1u)) {
           ok = false;
           break;
         }
-        const int col = kb * kBK + c * 8;
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const int r = (t >> 3) + 16 * i;
-          const bool in = src[i] >= 0 && col < g.k;
-          cp_async16(sa(stage) + (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4)), in ? g.gx + src[i] * g.k + col : g.gx,
-                     in ? 16u : 0u);
-        }
-        cp_async_commit();
-        if (++pending > kCopyLagP) {
-          cp_async_wait<kCopyLagP>();
-          fence_proxy_async();
-          __syncwarp();
-          if (lane == 0) tc::mbar_arrive_cluster(full_even((stage - kCopyLagP + kStagesP) % kStagesP));
-          --pending;
-        }
+        if (lane == 0 && leader) tc::mbar_expect_tx(full(stage), 2 * 32 * kBK * 2);
+        __syncwarp();
+        tc::tma_load_2d_pair(sa(stage) + (uint32_t)(r * kBK * 2), &map_a, kb * kBK, srow, full_even(stage));
         if (++stage == kStagesP) {
           stage = 0;
           phase ^= 1u;
@@ -807,11 +759,6 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
       }
     }
     if (!ok && lane == 0) flag_error(g, 8);
-    cp_async_wait<0>();
-    fence_proxy_async();
-    __syncwarp();
-    if (lane == 0)
-      for (int i = pending; i > 0; --i) tc::mbar_arrive_cluster(full_even((stage - i + kStagesP) % kStagesP));
   } else {
     // ---------------------------------------------------------------- epilogue (both CTAs)
     const int q = warp & 3;
@@ -1082,6 +1029,7 @@ tr_status tr_project_kept(const tr_tokens *in, const int32_t *d_cu_k, const int3
     total_rows = (long long)in->batch * in->n;
   }
   if (total_k < 0 || total_k > total_rows) return TR_ERR_BUDGET;
+  if (total_rows > INT_MAX) return TR_ERR_UNSUPPORTED;  // TMA row coordinates are 32-bit
   if (total_k == 0) return TR_OK;
   if (in->batch == 0 || !d_cu_k || !idx) return TR_ERR_ARG;
   const long long rblocks = ((long long)total_k + kBM - 1) / kBM;
@@ -1104,9 +1052,12 @@ tr_status tr_project_kept(const tr_tokens *in, const int32_t *d_cu_k, const int3
   g.cu_seqlens = in->cu_seqlens;
   g.cu_k = d_cu_k;
   g.idx = idx;
-  CUtensorMap mb, mo;
-  if (!make_map(&mb, w, d_out, in->d, b_box_rows(g.m)) || !make_map(&mo, z, total_k, d_out, 32)) return TR_ERR_CUDA;
-  return launch_gemm<kModeProject>(mb, mb, mo, g, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TR_OK
+  // A: x, one row per box (the loaders gather rows by kept index)
+  CUtensorMap ma, mb, mo;
+  if (!make_map(&ma, in->x, total_rows, in->d, 1) || !make_map(&mb, w, d_out, in->d, b_box_rows(g.m)) ||
+      !make_map(&mo, z, total_k, d_out, 32))
+    return TR_ERR_CUDA;
+  return launch_gemm<kModeProject>(ma, mb, mo, g, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TR_OK
                                                                                                      : TR_ERR_CUDA;
 }
 

@@ -707,7 +707,7 @@ template <int kDt>
 __device__ __noinline__ bool df_row_block(const SelectArgs &a, long long row, int mode, ExactRec *rec, PartDf &part,
                                           const Group g) {
   constexpr int kPer = kDt == TR_F32 ? 4 : 8;  // elements per 16-byte chunk
-  constexpr int kLoads = 4;                    // chunks per stream in flight per thread
+  constexpr int kLoads = 2;                    // chunks per stream in flight per thread
   const int nchunks = a.d / kPer;
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   bool ok = true;
