@@ -21,11 +21,13 @@
 //               accumulators) and issues tcgen05.mma (M 128, N 256, K 16)
 //               from one thread, committing each stage back to the
 //               producer and each finished accumulator to the epilogue;
-//   warps 2-9   epilogue: one thread per accumulator row (TMEM lane) and
-//               column half (warps 2-5 columns 0-127, warps 6-9 128-255),
-//               16 columns per tcgen05.ld; the hidden GEMM applies
-//               bias + activation and stores H, the score GEMM stores x''
-//               and x and accumulates the row sums.
+//   warps 2-    epilogue: one thread per accumulator row (TMEM lane: a
+//               warp reads the lane quarter warp % 4) and column part, 16
+//               columns per tcgen05.ld.  The score GEMM runs 8 warps (2-9,
+//               column halves): it stores x'' and x and accumulates the row
+//               sums.  The hidden GEMM runs 16 (2-17, column quarters):
+//               bias + activation, and H through TMA stores of 32 x 32
+//               blocks; the projector 8 (halves, 32 x 64 blocks).
 // The projector mode (tr_project_kept) is the hidden GEMM with its A rows
 // gathered: A row j is token idx[j] of the image that owns kept slot j, so
 // the first projector layer reads X* = X_imp union X_div (Eq. 7) straight
@@ -35,7 +37,8 @@
 // row lands in the layout the tensor cores read: the swizzle follows the
 // shared-memory address); a slot past the kept rows loads row -1, which
 // reads zeros.  Each loader warp's lane 0 adds its rows' bytes to the
-// stage's transaction count and arrives once.
+// stage's transaction count and arrives once.  (One warp issuing all 128
+// row loads was too slow: 769 against 273 us.)
 //
 // The epilogue of tile i overlaps the main loop of tile i + 1 (two TMEM
 // accumulators).  A row's sums over its 2 n_tiles column halves are
@@ -60,20 +63,31 @@ constexpr int kBM = 128, kBN = 256, kBK = 64, kStages = 4;
 constexpr int kATile = kBM * kBK * 2;             // bytes of one A k-block
 constexpr int kBTile = kBN * kBK * 2;             // bytes of one B k-block
 constexpr int kStageBytes = kATile + kBTile;      // 48 KiB
-constexpr int kEpiWarps = 8;                      // two warpgroups: column halves of a tile
+constexpr int kEpiWarps = 8;                      // score mode: two warpgroups, column halves of a tile
 enum { kModeHidden = 0, kModeScore = 1, kModeProject = 2 };
+// Epilogue warps per mode: the hidden GEMM's epilogue (activation and a TMA
+// store) runs four warpgroups, one per column quarter, so that more warps
+// hide the latencies of its TMEM loads and activation arithmetic; the score
+// and projector epilogues run two (column halves) -- the projector's threads
+// also include its row loaders.
+__host__ __device__ constexpr int epi_warps(int mode) { return mode == kModeHidden ? 2 * kEpiWarps : kEpiWarps; }
+__host__ __device__ constexpr int epi_parts(int mode) { return epi_warps(mode) / 4; }  // column parts of a tile
 // producer, MMA issuer, epilogue (+ the A-row loaders of the projector mode)
-constexpr int kCopyWarps = 4;                      // projector: A-row loader warps, one row per lane
-static_assert(kCopyWarps * 32 == kBM, "the loaders' lanes cover a tile's rows");
-__host__ __device__ constexpr int gemm_threads(int mode) { return 64 + 32 * kEpiWarps + (mode == 2 ? 32 * kCopyWarps : 0); }
+constexpr int kLoadWarps = 4;                      // projector: A-row loader warps, one row per lane
+static_assert(kLoadWarps * 32 == kBM, "the loaders' lanes cover a tile's rows");
+__host__ __device__ constexpr int gemm_threads(int mode) {
+  return 64 + 32 * epi_warps(mode) + (mode == kModeProject ? 32 * kLoadWarps : 0);
+}
 constexpr int kTmemCols = 2 * kBN;                // two accumulators
 constexpr int kChunk = 16;                        // columns per tcgen05.ld
 constexpr int kPartWords = 10;                    // hi, lo of L1, S2, A, B, P
 constexpr uint32_t kIdesc = tc::idesc_bf16(kBM, kBN);
-// Per epilogue warp, a 32-row x 64-column bf16 output block staged for a TMA
-// store (hidden and projector modes), 128-byte rows in the swizzled layout.
-constexpr int kStageOut = 32 * 128;
-constexpr int kStageOutAll = kEpiWarps * kStageOut;  // 32 KiB
+// Per epilogue warp of the hidden and projector modes, a 32-row bf16 output
+// block staged for a TMA store: 32 columns (64-byte rows, 64-byte swizzle)
+// with four column parts, 64 (128-byte rows and swizzle) with two; 32 KiB in
+// all either way.
+constexpr int kStageOutAll = 32 * 1024;
+__host__ __device__ constexpr int stage_out(int mode) { return kStageOutAll / epi_warps(mode); }
 constexpr size_t kGemmSmem = (size_t)kStages * kStageBytes + kStageOutAll + 1024 + 256;
 
 struct GemmArgs {
@@ -222,25 +236,30 @@ __device__ __forceinline__ void epi_score(const GemmArgs &g, long long row, int 
   dx[1] = make_uint4(xo[4], xo[5], xo[6], xo[7]);
 }
 
-// One accumulator tile's worth of this warp's epilogue: the 8 chunks of 16
-// columns of its column half, each chunk's TMEM load (and, for the score
-// epilogue, its x' and residual loads) issued while the chunk before it is
-// processed.
-// Hidden / projector epilogue of one tile half for this warp: 8 chunks of
-// 16 columns, H = bf16(act(acc + bias)), staged per 64 columns in this
-// warp's 32 x 64 swizzled block (unit u of row r at r * 128 +
-// ((u ^ (r & 7)) << 4): the 32 lanes' 16-byte writes fall in distinct banks)
-// and written by one TMA store per 64 columns, so global memory sees whole
-// 128-byte row segments instead of one 32-byte piece per row and lane.  The
-// next chunk's TMEM load and bias are in flight while a chunk is processed;
-// a block is rewritten only after its previous store has read it.  Rows and
-// columns past the output are computed from zero operands and clipped by
-// the store.
+// Score epilogue of one tile half for this warp: the 8 chunks of 16 columns
+// of its column half, each chunk's TMEM load (and its x' and residual
+// loads) issued while the chunk before it is processed.
+//
+// Hidden / projector epilogue of one of a tile's kParts column parts for
+// this warp: chunks of 16 columns, H = bf16(act(acc + bias)), staged in this
+// warp's 32-row block of kBlk = 64 / (kParts / 2) columns, whose rows are
+// kBlk * 2 bytes with the swizzle of that span (unit u of row r at
+// r * 2 kBlk + ((u ^ ((r / (8 / (kBlk / 8))) % (kBlk / 8))) << 4): the 32
+// lanes' 16-byte writes take the fewest shared-memory wavefronts), and
+// written by one TMA store per block, so global memory sees whole row
+// segments.  The next chunk's TMEM load and bias are in flight while a chunk
+// is processed; the block is rewritten only after its previous store has
+// read it.  Rows and columns past the output are computed from zero operands
+// and clipped by the store.
+template <int kParts>
 __device__ __forceinline__ void drain_tile_store(const GemmArgs &g, const CUtensorMap *map_out, uint32_t buf,
-                                                 uint32_t taddr, int half, int nt, long long row0) {
-  constexpr int kChunks = kBN / 2 / kChunk;
+                                                 uint32_t taddr, int part, int nt, long long row0) {
+  constexpr int kChunks = kBN / kParts / kChunk;  // 8 (halves) or 4 (quarters)
+  constexpr int kBlk = 128 / kParts;              // block columns: 64 or 32
+  constexpr int kUnits = kBlk / 8;                // 16-byte units per block row: 8 or 4
+  constexpr int kPerBlk = kBlk / kChunk;          // chunks per block: 4 or 2
   const int lane = threadIdx.x & 31;
-  const int col_first = nt * kBN + half * (kBN / 2);
+  const int col_first = nt * kBN + part * (kBN / kParts);
   int chunks = 0;
   while (chunks < kChunks && col_first + chunks * kChunk < g.n) ++chunks;
   if (chunks == 0) return;
@@ -256,15 +275,17 @@ __device__ __forceinline__ void drain_tile_store(const GemmArgs &g, const CUtens
       for (int i = 0; i < 4; ++i) b[i] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
   };
-  tc::tmem_ld16_issue(taddr + (uint32_t)(half * (kBN / 2)), cur);
+  const uint32_t tcol = taddr + (uint32_t)(part * (kBN / kParts));
+  tc::tmem_ld16_issue(tcol, cur);
   load_bias(col_first, bc);
   tc::tmem_ld_wait(cur);
-  const uint32_t rowbuf = buf + (uint32_t)(lane * 128);
+  const uint32_t rowbuf = buf + (uint32_t)(lane * kBlk * 2);
+  const uint32_t sw = (uint32_t)((lane / (8 / kUnits)) % kUnits);  // the swizzle's row term
   for (int c = 0; c < chunks; ++c) {
     const int col0 = col_first + c * kChunk;
     const bool more = c + 1 < chunks;
     if (more) {
-      tc::tmem_ld16_issue(taddr + (uint32_t)(half * (kBN / 2) + (c + 1) * kChunk), nxt);
+      tc::tmem_ld16_issue(tcol + (uint32_t)((c + 1) * kChunk), nxt);
       load_bias(col0 + kChunk, bn);
     }
     const float bias[16] = {bc[0].x, bc[0].y, bc[0].z, bc[0].w, bc[1].x, bc[1].y, bc[1].z, bc[1].w,
@@ -274,18 +295,18 @@ __device__ __forceinline__ void drain_tile_store(const GemmArgs &g, const CUtens
     for (int i = 0; i < 8; ++i)
       w[i] = pack_bf16x2(activate(__uint_as_float(cur[2 * i]) + bias[2 * i], g.act),
                          activate(__uint_as_float(cur[2 * i + 1]) + bias[2 * i + 1], g.act));
-    if ((c & 3) == 0 && c > 0) {  // the block's previous store must have read it
+    if (c % kPerBlk == 0 && c > 0) {  // the block's previous store must have read it
       if (lane == 0) tc::bulk_wait_read();
       __syncwarp();
     }
-    const int u = 2 * (c & 3);
-    tc::st_shared_v4(rowbuf + (uint32_t)((u ^ (lane & 7)) << 4), w[0], w[1], w[2], w[3]);
-    tc::st_shared_v4(rowbuf + (uint32_t)(((u + 1) ^ (lane & 7)) << 4), w[4], w[5], w[6], w[7]);
-    if ((c & 3) == 3 || !more) {  // a 64-column block is complete: one TMA store for the warp's 32 rows
+    const uint32_t u = 2u * (uint32_t)(c % kPerBlk);
+    tc::st_shared_v4(rowbuf + ((u ^ sw) << 4), w[0], w[1], w[2], w[3]);
+    tc::st_shared_v4(rowbuf + (((u + 1u) ^ sw) << 4), w[4], w[5], w[6], w[7]);
+    if (c % kPerBlk == kPerBlk - 1 || !more) {  // a block is complete: one TMA store for the warp's 32 rows
       tc::fence_async_shared();
       __syncwarp();
       if (lane == 0 && row0 < g.m) {  // a block wholly past the last row is not stored
-        tc::tma_store_2d(map_out, col_first + 64 * (c >> 2), (int)row0, buf);
+        tc::tma_store_2d(map_out, col_first + kBlk * (c / kPerBlk), (int)row0, buf);
         tc::bulk_commit();
       }
     }
@@ -419,12 +440,12 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStages; ++s) {
-      tc::mbar_init(full(s), kMode == kModeProject ? 1 + kCopyWarps : 1);  // + one arrival per loader warp
+      tc::mbar_init(full(s), kMode == kModeProject ? 1 + kLoadWarps : 1);  // + one arrival per loader warp
       tc::mbar_init(empty(s), 1);
     }
     for (int a = 0; a < 2; ++a) {
       tc::mbar_init(tfull(a), 1);
-      tc::mbar_init(tempty(a), 32 * kEpiWarps);
+      tc::mbar_init(tempty(a), 32 * epi_warps(kMode));
     }
     tc::mbar_init(done, 1);
     tc::mbar_fence_init();
@@ -516,11 +537,11 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
     if (lane == 0) tc::mma_commit(done);
     __syncwarp();
     tc::mbar_wait_warp(done, 0);
-  } else if (kMode == kModeProject && warp >= 2 + kEpiWarps) {
+  } else if (kMode == kModeProject && warp >= 2 + epi_warps(kMode)) {
     // ---------------------------------------------------------------- A rows (projector mode)
     // lane l of loader warp w brings row 32 w + l of each A k-block by a
     // one-row TMA load (a row past the kept slots, coordinate -1, reads zeros)
-    const int r = (warp - 2 - kEpiWarps) * 32 + lane;
+    const int r = (warp - 2 - epi_warps(kMode)) * 32 + lane;
     int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
@@ -546,7 +567,7 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
   } else {
     // ---------------------------------------------------------------- epilogue
     const int q = warp & 3;            // TMEM lane quadrant this warp may read
-    const int half = (warp - 2) >> 2;  // column half of the tile
+    const int half = (warp - 2) >> 2;  // column half (score) or quarter (hidden, projector) of the tile
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = blockIdx.x; tile < g.tiles; tile += gridDim.x) {
@@ -563,7 +584,8 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
       if (kMode == kModeScore)
         drain_tile<kMode>(g, taddr, half, nt, row, row_ok, sums);
       else
-        drain_tile_store(g, &map_out, out_stage + (uint32_t)((warp - 2) * kStageOut), taddr, half, nt,
+        drain_tile_store<epi_parts(kMode)>(g, &map_out, out_stage + (uint32_t)((warp - 2) * stage_out(kMode)), taddr,
+                                           half, nt,
                          row - lane);
       tc::fence_before_sync();
       tc::mbar_arrive(tempty(acc));  // the MMA warp may refill this accumulator
@@ -629,12 +651,12 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
   constexpr uint32_t kTx = kMode == kModeProject ? 2 * kHalfTile : 2 * kStagePBytes;
   if (threadIdx.x == 0) {
     for (int s = 0; s < kStagesP; ++s) {
-      tc::mbar_init(full(s), kMode == kModeProject ? 1 + kCopyWarps : 1);  // + the even CTA's loader warps
+      tc::mbar_init(full(s), kMode == kModeProject ? 1 + kLoadWarps : 1);  // + the even CTA's loader warps
       tc::mbar_init(empty(s), 1);
     }
     for (int a = 0; a < 2; ++a) {
       tc::mbar_init(tfull(a), 1);
-      tc::mbar_init(tempty(a), 2 * kEpiWarps);  // one arrival per epilogue warp of either CTA
+      tc::mbar_init(tempty(a), 2 * epi_warps(kMode));  // one arrival per epilogue warp of either CTA
     }
     tc::mbar_init(done, 1);
     tc::mbar_fence_init();
@@ -731,12 +753,12 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
       __syncwarp();
     }
     tc::mbar_wait_warp(done, 0);  // every pair MMA has completed (both CTAs' TMEM)
-  } else if (kMode == kModeProject && warp >= 2 + kEpiWarps) {
+  } else if (kMode == kModeProject && warp >= 2 + epi_warps(kMode)) {
     // ---------------------------------------------------------------- A rows (projector mode)
     // as in the one-SM kernel, into this CTA's half of the pair's rows; the
     // loads land on the even CTA's barrier, whose loader warps expect both
     // CTAs' bytes (the odd CTA's loader warps do not arrive)
-    const int r = (warp - 2 - kEpiWarps) * 32 + lane;
+    const int r = (warp - 2 - epi_warps(kMode)) * 32 + lane;
     int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
@@ -762,7 +784,7 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
   } else {
     // ---------------------------------------------------------------- epilogue (both CTAs)
     const int q = warp & 3;
-    const int half = (warp - 2) >> 2;
+    const int half = (warp - 2) >> 2;  // column half (score) or quarter of the tile
     int acc = 0;
     uint32_t acc_phase = 0;
     for (int tile = cluster; tile < tiles; tile += clusters) {
@@ -780,7 +802,8 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
       if (kMode == kModeScore)
         drain_tile<kMode>(g, taddr, half, nt, row, row_ok, sums);
       else
-        drain_tile_store(g, &map_out, out_stage + (uint32_t)((warp - 2) * kStageOut), taddr, half, nt,
+        drain_tile_store<epi_parts(kMode)>(g, &map_out, out_stage + (uint32_t)((warp - 2) * stage_out(kMode)), taddr,
+                                           half, nt,
                          row - lane);
       tc::fence_before_sync();
       __syncwarp();
@@ -821,15 +844,19 @@ EncodeTiled encode_fn() {
 
 // Row-major bf16 [rows, cols] read in boxes of box_rows x 64 columns with the
 // 128-byte swizzle; out-of-range rows and columns read as zeros.
-bool make_map(CUtensorMap *map, const void *base, long long rows, long long cols, int box_rows) {
+// A bf16 [rows, cols] row-major tensor in boxes of box_rows x box_cols
+// (box_cols x 2 bytes = the swizzle span: 64 columns with the 128-byte
+// swizzle for operands, 32 with the 64-byte swizzle for the output staging).
+bool make_map(CUtensorMap *map, const void *base, long long rows, long long cols, int box_rows, int box_cols = kBK,
+              CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
   EncodeTiled fn = encode_fn();
   if (!fn) return false;
   const cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
   const cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
-  const cuuint32_t box[2] = {(cuuint32_t)kBK, (cuuint32_t)box_rows};
+  const cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
   const cuuint32_t estr[2] = {1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -961,7 +988,7 @@ tr_status tr_mlp_hidden(const tr_mlp *m, void *h, int32_t *d_error, void *stream
   g.err = d_error;
   CUtensorMap ma, mb, mo;
   if (!make_map(&ma, m->x_pre, m->t, m->d, kBM) || !make_map(&mb, m->w1, m->d_hidden, m->d, b_box_rows(g.m)) ||
-      !make_map(&mo, h, m->t, m->d_hidden, 32))
+      !make_map(&mo, h, m->t, m->d_hidden, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B))
     return TR_ERR_CUDA;
   return launch_gemm<kModeHidden>(ma, mb, mo, g, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TR_OK
                                                                                                     : TR_ERR_CUDA;
