@@ -31,14 +31,17 @@
 // The projector mode (tr_project_kept) is the hidden GEMM with its A rows
 // gathered: A row j is token idx[j] of the image that owns kept slot j, so
 // the first projector layer reads X* = X_imp union X_div (Eq. 7) straight
-// from x without a gathered copy.  Four more warps (10-13) bring those rows:
-// lane l of warp w issues, for row 32 w + l of each A k-block, a tiled TMA
-// load of one 64-element row of x (a one-row box, 128-byte swizzle, so the
-// row lands in the layout the tensor cores read: the swizzle follows the
-// shared-memory address); a slot past the kept rows loads row -1, which
-// reads zeros.  Each loader warp's lane 0 adds its rows' bytes to the
-// stage's transaction count and arrives once.  (One warp issuing all 128
-// row loads was too slow: 769 against 273 us.)
+// from x without a gathered copy.  Four more warps (10-13) bring those
+// rows: lanes 0-7 of each load four rows of each A k-block with one TMA
+// tile::gather4 load (four 64-element rows of x by index, one-row box,
+// 128-byte swizzle -- the rows land in the layout the tensor cores read: the
+// swizzle follows the shared-memory address); a group with a row past the
+// kept slots (or a k-block past x's columns) takes four one-row tiled loads
+// instead, an outside row at coordinate -1, which reads zeros.  Each loader
+// warp's lane 0 adds its rows' bytes to the stage's transaction count and
+// arrives once.  The rate at which one warp issues TMA loads sets the pace:
+// 128 one-row loads per stage took 769 us from one warp and 273 us from
+// four, the gather4 loads 314 us from one warp and 200 us from four.
 //
 // The epilogue of tile i overlaps the main loop of tile i + 1 (two TMEM
 // accumulators).  A row's sums over its 2 n_tiles column halves are
@@ -68,13 +71,17 @@ enum { kModeHidden = 0, kModeScore = 1, kModeProject = 2 };
 // Epilogue warps per mode: the hidden GEMM's epilogue (activation and a TMA
 // store) runs four warpgroups, one per column quarter, so that more warps
 // hide the latencies of its TMEM loads and activation arithmetic; the score
-// and projector epilogues run two (column halves) -- the projector's threads
-// also include its row loaders.
+// and projector epilogues run two (column halves) -- the projector's
+// threads also include its four row-loader warps (measured on clip_mlp576's
+// projector: four loader warps with 8 epilogue warps 200 us, with 16 195 us
+// but spilling; two loader warps with 16, 226 us; eight with 8, 212 us).
 __host__ __device__ constexpr int epi_warps(int mode) { return mode == kModeHidden ? 2 * kEpiWarps : kEpiWarps; }
 __host__ __device__ constexpr int epi_parts(int mode) { return epi_warps(mode) / 4; }  // column parts of a tile
-// producer, MMA issuer, epilogue (+ the A-row loaders of the projector mode)
-constexpr int kLoadWarps = 4;                      // projector: A-row loader warps, one row per lane
-static_assert(kLoadWarps * 32 == kBM, "the loaders' lanes cover a tile's rows");
+// producer, MMA issuer, epilogue (+ the A-row loader warps of the projector mode)
+constexpr int kLoadRows = 4;   // projector: rows per loader lane and k-block, one tile::gather4
+constexpr int kLoadWarps = 4;  // projector: loader warps, kBM / (kLoadRows kLoadWarps) lanes each
+constexpr int kLoadLanes = kBM / (kLoadRows * kLoadWarps);
+static_assert(kLoadLanes * kLoadRows * kLoadWarps == kBM && kLoadLanes <= 32, "the loaders cover a tile's rows");
 __host__ __device__ constexpr int gemm_threads(int mode) {
   return 64 + 32 * epi_warps(mode) + (mode == kModeProject ? 32 * kLoadWarps : 0);
 }
@@ -539,24 +546,43 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
     tc::mbar_wait_warp(done, 0);
   } else if (kMode == kModeProject && warp >= 2 + epi_warps(kMode)) {
     // ---------------------------------------------------------------- A rows (projector mode)
-    // lane l of loader warp w brings row 32 w + l of each A k-block by a
-    // one-row TMA load (a row past the kept slots, coordinate -1, reads zeros)
-    const int r = (warp - 2 - epi_warps(kMode)) * 32 + lane;
+    // lane l < kLoadLanes of loader warp w brings rows 4 j .. 4 j + 3 (j = w
+    // kLoadLanes + l) of each A k-block with one tile::gather4 load; a group
+    // with a row outside x (past the kept slots) or a k-block past x's
+    // columns takes four one-row loads instead, an outside row at coordinate
+    // -1, which reads zeros
+    const int j = (warp - 2 - epi_warps(kMode)) * kLoadLanes + lane;
+    const bool loads = lane < kLoadLanes;
     int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
     for (int tile = blockIdx.x; tile < g.tiles && ok; tile += gridDim.x) {
       const int rb = tile / g.n_tiles;
-      const long long src = kept_source_row(g, (long long)rb * kBM + r);
-      const int srow = src >= 0 ? (int)src : -1;
+      int srow[kLoadRows];
+      bool whole = true;
+#pragma unroll
+      for (int i = 0; i < kLoadRows; ++i) {
+        const long long src = loads ? kept_source_row(g, (long long)rb * kBM + kLoadRows * j + i) : -1;
+        srow[i] = src >= 0 ? (int)src : -1;
+        whole &= src >= 0;
+      }
       for (int kb = 0; kb < g.kblocks; ++kb) {
         if (!tc::mbar_wait_warp(empty(stage), phase ^ 1u)) {
           ok = false;
           break;
         }
-        if (lane == 0) tc::mbar_expect_tx(full(stage), 32 * kBK * 2);  // this warp's 32 rows; one arrival
+        if (lane == 0) tc::mbar_expect_tx(full(stage), kATile / kLoadWarps);  // this warp's rows; one arrival
         __syncwarp();
-        tc::tma_load_2d(sa(stage) + (uint32_t)(r * kBK * 2), &map_a, kb * kBK, srow, full(stage));
+        const uint32_t dst = sa(stage) + (uint32_t)(kLoadRows * j * kBK * 2);
+        if (loads) {
+          if (whole && (kb + 1) * kBK <= g.k) {  // rows and columns inside x
+            tc::tma_gather4(dst, &map_a, kb * kBK, srow[0], srow[1], srow[2], srow[3], full(stage));
+          } else {
+#pragma unroll
+            for (int i = 0; i < kLoadRows; ++i)
+              tc::tma_load_2d(dst + (uint32_t)(i * kBK * 2), &map_a, kb * kBK, srow[i], full(stage));
+          }
+        }
         if (++stage == kStages) {
           stage = 0;
           phase ^= 1u;
@@ -758,22 +784,39 @@ __global__ void __launch_bounds__(gemm_threads(kMode), 1)
     // as in the one-SM kernel, into this CTA's half of the pair's rows; the
     // loads land on the even CTA's barrier, whose loader warps expect both
     // CTAs' bytes (the odd CTA's loader warps do not arrive)
-    const int r = (warp - 2 - epi_warps(kMode)) * 32 + lane;
+    const int j = (warp - 2 - epi_warps(kMode)) * kLoadLanes + lane;
+    const bool loads = lane < kLoadLanes;
     int stage = 0;
     uint32_t phase = 0;
     bool ok = true;
     for (int tile = cluster; tile < tiles && ok; tile += clusters) {
       const int rb = tile / g.n_tiles;
-      const long long src = kept_source_row(g, (long long)rb * 2 * kBM + (long long)rank * kBM + r);
-      const int srow = src >= 0 ? (int)src : -1;
+      int srow[kLoadRows];
+      bool whole = true;
+#pragma unroll
+      for (int i = 0; i < kLoadRows; ++i) {
+        const long long src =
+            loads ? kept_source_row(g, (long long)rb * 2 * kBM + (long long)rank * kBM + kLoadRows * j + i) : -1;
+        srow[i] = src >= 0 ? (int)src : -1;
+        whole &= src >= 0;
+      }
       for (int kb = 0; kb < g.kblocks; ++kb) {
         if (!tc::mbar_wait_warp(empty(stage), phase ^ 1u)) {
           ok = false;
           break;
         }
-        if (lane == 0 && leader) tc::mbar_expect_tx(full(stage), 2 * 32 * kBK * 2);
+        if (lane == 0 && leader) tc::mbar_expect_tx(full(stage), 2 * kHalfTile / kLoadWarps);
         __syncwarp();
-        tc::tma_load_2d_pair(sa(stage) + (uint32_t)(r * kBK * 2), &map_a, kb * kBK, srow, full_even(stage));
+        const uint32_t dst = sa(stage) + (uint32_t)(kLoadRows * j * kBK * 2);
+        if (loads) {
+          if (whole && (kb + 1) * kBK <= g.k) {  // rows and columns inside x
+            tc::tma_gather4_pair(dst, &map_a, kb * kBK, srow[0], srow[1], srow[2], srow[3], full_even(stage));
+          } else {
+#pragma unroll
+            for (int i = 0; i < kLoadRows; ++i)
+              tc::tma_load_2d_pair(dst + (uint32_t)(i * kBK * 2), &map_a, kb * kBK, srow[i], full_even(stage));
+          }
+        }
         if (++stage == kStagesP) {
           stage = 0;
           phase ^= 1u;
@@ -988,7 +1031,9 @@ tr_status tr_mlp_hidden(const tr_mlp *m, void *h, int32_t *d_error, void *stream
   g.err = d_error;
   CUtensorMap ma, mb, mo;
   if (!make_map(&ma, m->x_pre, m->t, m->d, kBM) || !make_map(&mb, m->w1, m->d_hidden, m->d, b_box_rows(g.m)) ||
-      !make_map(&mo, h, m->t, m->d_hidden, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B))
+      !make_map(&mo, h, m->t, m->d_hidden, 32, 128 / epi_parts(kModeHidden),
+                                                           epi_parts(kModeHidden) == 2 ? CU_TENSOR_MAP_SWIZZLE_128B
+                                                                                       : CU_TENSOR_MAP_SWIZZLE_64B))
     return TR_ERR_CUDA;
   return launch_gemm<kModeHidden>(ma, mb, mo, g, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TR_OK
                                                                                                     : TR_ERR_CUDA;
@@ -1082,7 +1127,8 @@ tr_status tr_project_kept(const tr_tokens *in, const int32_t *d_cu_k, const int3
   // A: x, one row per box (the loaders gather rows by kept index)
   CUtensorMap ma, mb, mo;
   if (!make_map(&ma, in->x, total_rows, in->d, 1) || !make_map(&mb, w, d_out, in->d, b_box_rows(g.m)) ||
-      !make_map(&mo, z, total_k, d_out, 32))
+      !make_map(&mo, z, total_k, d_out, 32, 128 / epi_parts(kModeProject),
+                epi_parts(kModeProject) == 2 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B))
     return TR_ERR_CUDA;
   return launch_gemm<kModeProject>(ma, mb, mo, g, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TR_OK
                                                                                                      : TR_ERR_CUDA;

@@ -210,6 +210,26 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr) {
 }
 // 2-D tiled load into this CTA's shared memory completing on a barrier that
 // may sit in the peer CTA (bar: shared::cluster address).
+// Four rows r0..r3 of a 2D tensor at column c0 (tile::gather4: the map's
+// box is one row high), written one after another from dst with the map's
+// swizzle, completing on bar.  The rows must lie inside the tensor.
+__device__ __forceinline__ void tma_gather4(uint32_t dst, const CUtensorMap *map, int c0, int r0, int r1, int r2,
+                                            int r3, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes [%0], [%1, {%2, "
+      "%3, %4, %5, %6}], [%7];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(r0), "r"(r1), "r"(r2), "r"(r3), "r"(bar)
+      : "memory");
+}
+// The same for an SM pair: completion may be signalled on the peer CTA's barrier.
+__device__ __forceinline__ void tma_gather4_pair(uint32_t dst, const CUtensorMap *map, int c0, int r0, int r1,
+                                                 int r2, int r3, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile::gather4.mbarrier::complete_tx::bytes.cta_group::2 [%0], "
+      "[%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(r0), "r"(r1), "r"(r2), "r"(r3), "r"(bar)
+      : "memory");
+}
 __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap *map, int c0, int c1,
                                                  uint32_t bar) {
   asm volatile(

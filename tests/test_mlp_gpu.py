@@ -206,7 +206,8 @@ def _hidden_on(altr, y, w, bias, act):
 @pytest.mark.parametrize("name,over,bud,d_out,act", [
     ("llava576", dict(batch=3, d=1024), dict(k=192), 4096, "gelu"),           # LLaVA-1.5's 1024 -> 4096 layer
     ("ragged_dynres", dict(batch=5, n=(256, 3000), d=1152), dict(ratio=(2, 9)), 1280, "quick_gelu"),
-], ids=["llava576", "ragged_dynres"])
+    ("llava576", dict(batch=2, d=1040), dict(k=64), 512, "gelu"),              # a partial last k-block
+], ids=["llava576", "ragged_dynres", "partial_kblock"])
 def test_project_kept(name, over, bud, d_out, act):
     # Selection, then the projector's first layer on the kept tokens read
     # from x by index: bit for bit the hidden GEMM on the gathered copy y,
