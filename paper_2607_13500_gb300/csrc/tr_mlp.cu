@@ -44,10 +44,16 @@
 // four, the gather4 loads 314 us from one warp and 200 us from four.
 //
 // The epilogue of tile i overlaps the main loop of tile i + 1 (two TMEM
-// accumulators).  A row's sums over its 2 n_tiles column halves are
-// combined by the last of the warps that worked on them (an arrival
-// counter; no warp or CTA waits for another), in column order, so the
-// record does not depend on which finished first.
+// accumulators), but not for free: epilogue arithmetic on the SM
+// sub-partitions that also hold the producer and MMA warps slows the main
+// loop.  In a modified copy of the score GEMM with the sums' arithmetic
+// skipped on sub-partitions 0-1 it took 224 us, on 2-3 254 us, on all four
+// 193 us, against 257 us with none skipped.  So the epilogues do their fp32
+// arithmetic on packed pairs (add / mul / fma.f32x2, one instruction per two
+// columns): 6-7 % off all three modes.  A row's sums over its 2 n_tiles
+// column halves are combined by the last of the warps that worked on them
+// (an arrival counter; no warp or CTA waits for another), in column order,
+// so the record does not depend on which finished first.
 #include <cuda.h>
 #include <cuda_bf16.h>
 
@@ -119,25 +125,58 @@ struct GemmArgs {
 
 __device__ __forceinline__ float bf16_val(uint32_t bits16) { return __uint_as_float(bits16 << 16); }
 
-// erf(z) for z >= 0 by Abramowitz and Stegun, Handbook of Mathematical
-// Functions (1964), formula 7.1.26: 1 - (a1 t + ... + a5 t^5) exp(-z^2) with
-// t = 1 / (1 + p z), |error| <= 1.5e-7; evaluated with the fast exponential
-// and reciprocal intrinsics (a few ulp each), so GELU below stays within
-// ~2e-7 |v| of x Phi(x), far inside the bf16 rounding of its result.
-__device__ __forceinline__ float erf_as(float z) {
-  const float t = __fdividef(1.f, fmaf(0.3275911f, z, 1.f));
-  const float poly =
-      t * fmaf(t, fmaf(t, fmaf(t, fmaf(t, 1.061405429f, -1.453152027f), 1.421413741f), -0.284496736f), 0.254829592f);
-  return 1.f - poly * __expf(-z * z);
+// 2^x and 1/x by the hardware approximations (PTX ex2.approx, rcp.approx:
+// relative error about 2^-22 and 2^-23), a few fp32 ulp, far inside the bf16
+// rounding of the activations below.
+__device__ __forceinline__ float ex2_approx(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+__device__ __forceinline__ float rcp_approx(float x) {
+  float y;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
 }
 
-__device__ __forceinline__ float activate(float v, int act) {
+// Packed fp32 pairs (one instruction for two lanes of arithmetic, each
+// rounded to nearest like its scalar form).
+__device__ __forceinline__ float2 f2(float v) { return make_float2(v, v); }
+__device__ __forceinline__ float2 sub2(float2 a, float2 b) {  // a - b, one rounding
+  return __ffma2_rn(b, f2(-1.f), a);
+}
+__device__ __forceinline__ float2 ex2_2(float2 x) { return make_float2(ex2_approx(x.x), ex2_approx(x.y)); }
+__device__ __forceinline__ float2 rcp_2(float2 x) { return make_float2(rcp_approx(x.x), rcp_approx(x.y)); }
+
+// erf(z) for z >= 0 by Abramowitz and Stegun, Handbook of Mathematical
+// Functions (1964), formula 7.1.26: 1 - (a1 t + ... + a5 t^5) exp(-z^2) with
+// t = 1 / (1 + p z), |error| <= 1.5e-7; with the approximate exponential and
+// reciprocal GELU below stays within ~2e-7 |v| of x Phi(x), far inside the
+// bf16 rounding of its result.  Two arguments at a time.
+__device__ __forceinline__ float2 erf_as2(float2 z) {
+  const float2 t = rcp_2(__ffma2_rn(z, f2(0.3275911f), f2(1.f)));
+  float2 poly = __ffma2_rn(t, f2(1.061405429f), f2(-1.453152027f));
+  poly = __ffma2_rn(t, poly, f2(1.421413741f));
+  poly = __ffma2_rn(t, poly, f2(-0.284496736f));
+  poly = __ffma2_rn(t, poly, f2(0.254829592f));
+  poly = __fmul2_rn(t, poly);
+  const float2 ez = ex2_2(__fmul2_rn(__fmul2_rn(z, z), f2(-1.4426950408889634f)));  // exp(-z^2)
+  return sub2(f2(1.f), __fmul2_rn(poly, ez));
+}
+
+// The activation sigma of the hidden layer (and the projector) on a pair of
+// pre-activations.
+__device__ __forceinline__ float2 activate2(float2 v, int act) {
   if (act == TR_ACT_GELU) {  // v Phi(v) = v (1 + erf(v / sqrt 2)) / 2
-    const float e = erf_as(fabsf(v) * 0.70710678118654752f);
-    return 0.5f * v * (1.f + copysignf(e, v));
+    const float2 e = erf_as2(__fmul2_rn(make_float2(fabsf(v.x), fabsf(v.y)), f2(0.70710678118654752f)));
+    return __fmul2_rn(__fmul2_rn(v, f2(0.5f)), __fadd2_rn(f2(1.f), make_float2(copysignf(e.x, v.x), copysignf(e.y, v.y))));
   }
-  if (act == TR_ACT_QUICK_GELU)  // v sigma(1.702 v); the exponent is capped so the divisor stays finite
-    return __fdividef(v, 1.f + __expf(fminf(-1.702f * v, 80.f)));
+  if (act == TR_ACT_QUICK_GELU) {  // v sigma(1.702 v) = v / (1 + 2^(-1.702 log2(e) v)), the exponent capped
+    float2 z = __fmul2_rn(v, f2(-2.4554669595930156f));
+    z.x = fminf(z.x, 126.f);
+    z.y = fminf(z.y, 126.f);
+    return __fmul2_rn(v, rcp_2(__fadd2_rn(ex2_2(z), f2(1.f))));
+  }
   return v;
 }
 
@@ -152,23 +191,24 @@ __device__ __forceinline__ void flag_error(const GemmArgs &g, int code) {
 
 // Hidden GEMM epilogue for 16 columns of one row: H = bf16(act(acc + b1)).
 __device__ __forceinline__ void epi_hidden(const GemmArgs &g, long long row, int col0, const float (&v)[16]) {
-  float a[16];
+  float2 a[8];
 #pragma unroll
-  for (int i = 0; i < 16; ++i) a[i] = v[i];
+  for (int i = 0; i < 8; ++i) a[i] = make_float2(v[2 * i], v[2 * i + 1]);
   if (g.bias) {  // the same 16 values in every lane: four broadcast loads
     const float4 *bp = reinterpret_cast<const float4 *>(g.bias + col0);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const float4 b = __ldg(bp + i);
-      a[4 * i] += b.x;
-      a[4 * i + 1] += b.y;
-      a[4 * i + 2] += b.z;
-      a[4 * i + 3] += b.w;
+      a[2 * i] = __fadd2_rn(a[2 * i], make_float2(b.x, b.y));
+      a[2 * i + 1] = __fadd2_rn(a[2 * i + 1], make_float2(b.z, b.w));
     }
   }
   uint32_t w[8];
 #pragma unroll
-  for (int i = 0; i < 8; ++i) w[i] = pack_bf16x2(activate(a[2 * i], g.act), activate(a[2 * i + 1], g.act));
+  for (int i = 0; i < 8; ++i) {
+    const float2 h = activate2(a[i], g.act);
+    w[i] = pack_bf16x2(h.x, h.y);
+  }
   uint4 *dst = reinterpret_cast<uint4 *>(g.out + row * g.n + col0);
   dst[0] = make_uint4(w[0], w[1], w[2], w[3]);
   dst[1] = make_uint4(w[4], w[5], w[6], w[7]);
@@ -193,47 +233,83 @@ __device__ __forceinline__ void load_score_in(const GemmArgs &g, long long row, 
   }
 }
 
+// The score epilogue keeps its five double-float sums as fp32 pairs:
+// component x takes the even columns, component y the odd ones, merged once
+// per tile.
+__device__ __forceinline__ float2 bf16x2_f2(uint32_t w) {  // the two bf16 of a word as fp32
+  return make_float2(bf16_val(w & 0xffffu), bf16_val(w >> 16));
+}
+struct DF2 {
+  float2 hi, lo;
+};
+struct Acc2 {
+  DF2 l1, s2, a, b, p;
+};
+// acc += v with Knuth's TwoSum per component: s = hi + v, and the rounding
+// error (hi - (s - (s - hi))) + (v - (s - hi)) joins lo.  With nb = hi - s
+// (= -(s - hi) exactly, rounding being symmetric) the steps are the scalar
+// df_add's, two lanes at a time.
+__device__ __forceinline__ void df2_add(DF2 &acc, float2 v) {
+  const float2 s = __fadd2_rn(acc.hi, v);
+  const float2 nb = sub2(acc.hi, s);
+  const float2 aa = __fadd2_rn(s, nb);
+  acc.lo = __fadd2_rn(acc.lo, __fadd2_rn(sub2(acc.hi, aa), __fadd2_rn(v, nb)));
+  acc.hi = s;
+}
+// acc += u v for products exact in fp32 (bf16 times bf16): the fused
+// multiply-add rounds hi + u v once, as the sum of the exact product would.
+__device__ __forceinline__ void df2_add_prod(DF2 &acc, float2 u, float2 v) {
+  const float2 s = __ffma2_rn(u, v, acc.hi);
+  const float2 nb = sub2(acc.hi, s);
+  const float2 aa = __fadd2_rn(s, nb);
+  acc.lo = __fadd2_rn(acc.lo, __fadd2_rn(sub2(acc.hi, aa), __ffma2_rn(u, v, nb)));
+  acc.hi = s;
+}
+__device__ __forceinline__ void df2_fold(DF &out, const DF2 &in) {  // even + odd columns
+  out.hi = in.hi.x;
+  out.lo = in.lo.x;
+  df_merge(out, in.hi.y, in.lo.y);
+}
+
 // Score GEMM epilogue for 16 columns of one row: x'' = bf16(acc + b2),
 // x = bf16(resid + x''), both stored; the five sums take the stored values
 // (products and squares of bf16 values are exact in fp32; each term enters
 // its double-float sum through TwoSum).
 __device__ __forceinline__ void epi_score(const GemmArgs &g, long long row, int col0, const float (&v)[16],
-                                          const ScoreIn &in, Acc &acc) {
+                                          const ScoreIn &in, Acc2 &acc) {
   const long long base = row * g.n + col0;
   const uint32_t pw[8] = {in.p0.x, in.p0.y, in.p0.z, in.p0.w, in.p1.x, in.p1.y, in.p1.z, in.p1.w};
   const uint32_t rw[8] = {in.r0.x, in.r0.y, in.r0.z, in.r0.w, in.r1.x, in.r1.y, in.r1.z, in.r1.w};
-  float a[16];
+  float2 a[8];
 #pragma unroll
-  for (int i = 0; i < 16; ++i) a[i] = v[i];
+  for (int i = 0; i < 8; ++i) a[i] = make_float2(v[2 * i], v[2 * i + 1]);
   if (g.bias) {
     const float4 *bp = reinterpret_cast<const float4 *>(g.bias + col0);
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
       const float4 b = __ldg(bp + i);
-      a[4 * i] += b.x;
-      a[4 * i + 1] += b.y;
-      a[4 * i + 2] += b.z;
-      a[4 * i + 3] += b.w;
+      a[2 * i] = __fadd2_rn(a[2 * i], make_float2(b.x, b.y));
+      a[2 * i + 1] = __fadd2_rn(a[2 * i + 1], make_float2(b.z, b.w));
     }
   }
   uint32_t qo[8], xo[8];
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
-    qo[i] = pack_bf16x2(a[2 * i], a[2 * i + 1]);  // x''
-    const float q0 = bf16_val(qo[i] & 0xffffu), q1 = bf16_val(qo[i] >> 16);
-    xo[i] = g.resid ? pack_bf16x2(bf16_val(rw[i] & 0xffffu) + q0, bf16_val(rw[i] >> 16) + q1) : qo[i];
-    const float x0 = bf16_val(xo[i] & 0xffffu), x1 = bf16_val(xo[i] >> 16);
-    const float p0 = bf16_val(pw[i] & 0xffffu), p1 = bf16_val(pw[i] >> 16);  // x'
-    df_add(acc.l1, fabsf(x0));
-    df_add(acc.l1, fabsf(x1));
-    df_add(acc.s2, x0 * x0);
-    df_add(acc.s2, x1 * x1);
-    df_add(acc.a, p0 * p0);
-    df_add(acc.a, p1 * p1);
-    df_add(acc.b, q0 * q0);
-    df_add(acc.b, q1 * q1);
-    df_add(acc.p, p0 * q0);
-    df_add(acc.p, p1 * q1);
+    qo[i] = pack_bf16x2(a[i].x, a[i].y);  // x''
+    const float2 q = bf16x2_f2(qo[i]);
+    if (g.resid) {
+      const float2 xs = __fadd2_rn(bf16x2_f2(rw[i]), q);
+      xo[i] = pack_bf16x2(xs.x, xs.y);
+    } else {
+      xo[i] = qo[i];
+    }
+    const float2 xa = bf16x2_f2(xo[i] & 0x7fff7fffu);  // |x|
+    const float2 p = bf16x2_f2(pw[i]);                 // x'
+    df2_add(acc.l1, xa);
+    df2_add_prod(acc.s2, xa, xa);
+    df2_add_prod(acc.a, p, p);
+    df2_add_prod(acc.b, q, q);
+    df2_add_prod(acc.p, p, q);
   }
   uint4 *dq = reinterpret_cast<uint4 *>(g.out + base);
   dq[0] = make_uint4(qo[0], qo[1], qo[2], qo[3]);
@@ -271,7 +347,7 @@ __device__ __forceinline__ void drain_tile_store(const GemmArgs &g, const CUtens
   while (chunks < kChunks && col_first + chunks * kChunk < g.n) ++chunks;
   if (chunks == 0) return;
   uint32_t cur[16], nxt[16];
-  float4 bc[4], bn[4];
+  float4 bc[4];
   auto load_bias = [&](int col0, float4 (&b)[4]) {
     if (g.bias) {
       const float4 *bp = reinterpret_cast<const float4 *>(g.bias + col0);
@@ -284,24 +360,24 @@ __device__ __forceinline__ void drain_tile_store(const GemmArgs &g, const CUtens
   };
   const uint32_t tcol = taddr + (uint32_t)(part * (kBN / kParts));
   tc::tmem_ld16_issue(tcol, cur);
-  load_bias(col_first, bc);
   tc::tmem_ld_wait(cur);
   const uint32_t rowbuf = buf + (uint32_t)(lane * kBlk * 2);
   const uint32_t sw = (uint32_t)((lane / (8 / kUnits)) % kUnits);  // the swizzle's row term
   for (int c = 0; c < chunks; ++c) {
     const int col0 = col_first + c * kChunk;
     const bool more = c + 1 < chunks;
-    if (more) {
-      tc::tmem_ld16_issue(tcol + (uint32_t)((c + 1) * kChunk), nxt);
-      load_bias(col0 + kChunk, bn);
-    }
+    if (more) tc::tmem_ld16_issue(tcol + (uint32_t)((c + 1) * kChunk), nxt);
+    load_bias(col0, bc);  // the same 16 values in every lane (broadcast loads, cached)
     const float bias[16] = {bc[0].x, bc[0].y, bc[0].z, bc[0].w, bc[1].x, bc[1].y, bc[1].z, bc[1].w,
                             bc[2].x, bc[2].y, bc[2].z, bc[2].w, bc[3].x, bc[3].y, bc[3].z, bc[3].w};
     uint32_t w[8];
 #pragma unroll
-    for (int i = 0; i < 8; ++i)
-      w[i] = pack_bf16x2(activate(__uint_as_float(cur[2 * i]) + bias[2 * i], g.act),
-                         activate(__uint_as_float(cur[2 * i + 1]) + bias[2 * i + 1], g.act));
+    for (int i = 0; i < 8; ++i) {
+      const float2 h = activate2(__fadd2_rn(make_float2(__uint_as_float(cur[2 * i]), __uint_as_float(cur[2 * i + 1])),
+                                            make_float2(bias[2 * i], bias[2 * i + 1])),
+                                 g.act);
+      w[i] = pack_bf16x2(h.x, h.y);
+    }
     if (c % kPerBlk == 0 && c > 0) {  // the block's previous store must have read it
       if (lane == 0) tc::bulk_wait_read();
       __syncwarp();
@@ -321,8 +397,6 @@ __device__ __forceinline__ void drain_tile_store(const GemmArgs &g, const CUtens
       tc::tmem_ld_wait(nxt);
 #pragma unroll
       for (int i = 0; i < 16; ++i) cur[i] = nxt[i];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) bc[i] = bn[i];
     }
   }
   if (lane == 0) tc::bulk_wait_read();  // the block may be rewritten by the next tile
@@ -338,6 +412,7 @@ __device__ __forceinline__ void drain_tile(const GemmArgs &g, uint32_t taddr, in
   if (chunks == 0) return;
   uint32_t cur[16], nxt[16];
   ScoreIn in_cur{}, in_nxt{};
+  Acc2 acc2{};
   const int col_first = nt * kBN + half * (kBN / 2);
   tc::tmem_ld16_issue(taddr + (uint32_t)(half * (kBN / 2)), cur);
   if (kMode == kModeScore && row_ok) load_score_in(g, row, col_first, in_cur);
@@ -354,7 +429,7 @@ __device__ __forceinline__ void drain_tile(const GemmArgs &g, uint32_t taddr, in
 #pragma unroll
       for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(cur[i]);
       if (kMode == kModeScore)
-        epi_score(g, row, col0, v, in_cur, sums);
+        epi_score(g, row, col0, v, in_cur, acc2);
       else
         epi_hidden(g, row, col0, v);
     }
@@ -364,6 +439,13 @@ __device__ __forceinline__ void drain_tile(const GemmArgs &g, uint32_t taddr, in
       for (int i = 0; i < 16; ++i) cur[i] = nxt[i];
       in_cur = in_nxt;
     }
+  }
+  if (kMode == kModeScore) {
+    df2_fold(sums.l1, acc2.l1);
+    df2_fold(sums.s2, acc2.s2);
+    df2_fold(sums.a, acc2.a);
+    df2_fold(sums.b, acc2.b);
+    df2_fold(sums.p, acc2.p);
   }
 }
 

@@ -86,6 +86,7 @@ CASES = [
     ("clip_l", 300, 1024, 4096, "gelu", True, True),           # 3 row blocks, the last ragged
     ("ragged_dims", 200, 1152, 4304, "quick_gelu", True, False),  # a half column block, a K tail of 16
     ("one_row", 1, 256, 512, "none", False, True),              # x = x'' (no residual)
+    ("even_tiles_ragged", 600, 1296, 4400, "gelu", True, True),  # even column tile counts, every edge ragged
 ]
 
 
