@@ -631,11 +631,13 @@ def _bf16_peak():
 def measure_mlp(args, dev, altr, reps=20, batch=None):
     """The vision encoder's final-layer MLP with the scoring fused into its
     second GEMM (Eq. 5, Section IV-B), then the selection, the gather and
-    the projector's first layer on the kept tokens read by index, on the
-    CLIP-ViT-L/14-shaped batch: 64 images x 576 tokens, D = 1024, hidden
+    the projector's first layer on the gathered kept tokens (tr_project), on
+    the CLIP-ViT-L/14-shaped batch: 64 images x 576 tokens, D = 1024, hidden
     4096, K = 192.  Each kernel timed with CUDA events on the current stream
-    (median of `reps` steps, inputs larger than L2); beside it, the unfused
-    route through the same library (cuBLAS MLP, tr_score pass) for context."""
+    (median of `reps` steps, inputs larger than L2); beside it the projector
+    reading the kept rows from x by index (tr_project_kept, the same z bit for
+    bit) and the unfused route through the same library (cuBLAS MLP, tr_score
+    pass), for context."""
     w = synth.make_mlp("clip_mlp576", seed=args.seed, device=dev, **({"batch": batch} if batch else {}))
     t, d, dh = w.total, w.x_pre.shape[1], w.w1.shape[0]
     wp, bp = synth.make_projector(d, w.d_proj, seed=args.seed, device=dev)
@@ -643,16 +645,21 @@ def measure_mlp(args, dev, altr, reps=20, batch=None):
     ks, k1s, cu = budget
     m = altr.Mlp(t, w.w1, w.w2, w.b1, w.b2, act=w.act)
     red = altr.Reducer(w.seqlens, d, torch.bfloat16, dev, budget=budget)
-    # events: 0 | hidden | 1 | score | 2 (status zeroed) 3 | select | 4 | gather | 5 | project | 6
-    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(7)] for _ in range(reps + 3)]
+    # events: 0 | hidden | 1 | score | 2 (status zeroed) 3 | select | 4 | gather | 5 | project | 6,
+    # then (outside the step) 7 | project_kept | 8
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(9)] for _ in range(reps + 3)]
     spans = {"tr_mlp_hidden": (0, 1), "tr_mlp_score": (1, 2), "tr_select": (3, 4), "tr_gather": (4, 5),
-             "tr_project_kept": (5, 6)}
+             "tr_project": (5, 6), "tr_project_kept": (7, 8)}
+    z = torch.empty(cu[-1], w.d_proj, dtype=torch.bfloat16, device=dev)
     clocks = ClockSampler(dev)
     for ev in evs:
         out = m.run(w.x_pre, w.resid, events=ev[0:3])
         r = red.run_select_gather(out.x, w.x_pre, out.x_post, out.stats, events=ev[3:6])
-        z, err = altr.project_kept(out.x, r.idx, cu, wp, bp, act="gelu", seqlens=w.seqlens, error=m.error)
+        altr.project(r.y, wp, bp, act="gelu", error=m.error, out=z)
         ev[6].record()
+        ev[7].record()
+        altr.project_kept(out.x, r.idx, cu, wp, bp, act="gelu", seqlens=w.seqlens, error=m.error)
+        ev[8].record()
     torch.cuda.synchronize()
     clk = clocks.stop()
     med = {n: statistics.median(ev[i].elapsed_time(ev[j]) for ev in evs[3:]) for n, (i, j) in spans.items()}
@@ -691,10 +698,14 @@ def measure_mlp(args, dev, altr, reps=20, batch=None):
                      "peak_source": f"{kind} cuBLAS bf16 GEMM (burst)", "traffic": None,
                      "algorithmic_flops": flop},
         "gemm_tflops": {"tr_mlp_hidden": tf(flop, med["tr_mlp_hidden"]), "tr_mlp_score": tf(flop, med["tr_mlp_score"]),
+                        "tr_project": tf(flop_p, med["tr_project"]),
                         "tr_project_kept": tf(flop_p, med["tr_project_kept"]),
                         "frac_of_measured_peak": {"tr_mlp_hidden": tf(flop, med["tr_mlp_hidden"]) / peak,
                                                   "tr_mlp_score": tf(flop, med["tr_mlp_score"]) / peak,
+                                                  "tr_project": tf(flop_p, med["tr_project"]) / peak,
                                                   "tr_project_kept": tf(flop_p, med["tr_project_kept"]) / peak}},
+        "projector_note": "the step projects the gathered rows y (tr_project); tr_project_kept, timed outside the "
+                          "step, reads the same rows from x by index and gives the same z bit for bit",
         "scoring_bytes": {"fused_extra_reads": t * d * e, "separate_pass_reads": 3 * t * d * e,
                           "note": "the fused epilogue reads x' (its P and A terms); x'' and x are written by the "
                                   "MLP in both routes; the separate pass reads x, x', x'' again"},

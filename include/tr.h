@@ -374,6 +374,23 @@ tr_status tr_project_kept(const tr_tokens *in, const int32_t *d_cu_k, const int3
                           const void *w, const float *bias, int32_t d_out, int32_t act, void *z, int32_t *d_error,
                           void *stream);
 
+/*
+ * The same first projector layer (Section III-A) on rows already gathered --
+ * tr_gather's y, or any dense rows:
+ *   y:        device bf16 [rows, d]
+ *   w, bias, d_out, act: as for tr_project_kept
+ *   z:        device bf16 [rows, d_out], row r from y's row r
+ * z = sigma(y W^T + bias) by the kernel of tr_mlp_hidden; for y = the rows
+ * that tr_project_kept reads, the two give the same z bit for bit (the same
+ * MMA order and epilogue arithmetic).  Gathering first and projecting the
+ * dense rows is the faster route on GB300: tr_project_kept's row loads are
+ * TMA gathers whose issue rate sets its pace, while the copy costs one write
+ * and one read of rows * d * 2 bytes.  d and d_out multiples of 16, pointers
+ * 16-byte aligned; rows = 0 does nothing.  d_error as for tr_mlp_hidden.
+ */
+tr_status tr_project(const void *y, int32_t rows, int32_t d, const void *w, const float *bias, int32_t d_out,
+                     int32_t act, void *z, int32_t *d_error, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -10,10 +10,11 @@ The work runs in libtr.so (hand-written CUDA for sm_103a, C ABI in
 include/tr.h); this package is its Python binding.  ``mlp`` runs the vision
 encoder's final-layer MLP (Eq. 5) on the tensor cores with the scoring fused
 into its second GEMM, for callers that own that MLP; ``project_kept`` runs the
-projector's first layer on the kept tokens, reading them from x by index.
+projector's first layer on the kept tokens, reading them from x by index, and
+``project`` the same layer on the gathered rows y (the faster route).
 """
-from .api import (Mlp, MlpResult, Pipeline, Reducer, ReduceResult, budgets, mlp, project_kept, reduce, score,
-                  select, workspace_bytes)
+from .api import (Mlp, MlpResult, Pipeline, Reducer, ReduceResult, budgets, mlp, project, project_kept, reduce,
+                  score, select, workspace_bytes)
 
-__all__ = ["Mlp", "MlpResult", "Pipeline", "Reducer", "ReduceResult", "budgets", "mlp", "project_kept", "reduce",
-           "score", "select", "workspace_bytes"]
+__all__ = ["Mlp", "MlpResult", "Pipeline", "Reducer", "ReduceResult", "budgets", "mlp", "project", "project_kept",
+           "reduce", "score", "select", "workspace_bytes"]

@@ -101,6 +101,8 @@ def load() -> ctypes.CDLL:
     lib.tr_mlp_score.restype = I32
     lib.tr_project_kept.argtypes = [tok, VP, VP, I32, VP, VP, I32, I32, VP, VP, VP]
     lib.tr_project_kept.restype = I32
+    lib.tr_project.argtypes = [VP, I32, I32, VP, VP, I32, I32, VP, VP, VP]
+    lib.tr_project.restype = I32
     _lib = lib
     return lib
 

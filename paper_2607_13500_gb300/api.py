@@ -668,3 +668,27 @@ def project_kept(x, idx, cu_k, w, bias=None, act="gelu", seqlens=None, error=Non
     check("tr_project_kept", lib.tr_project_kept(tok.ref(), _ptr(d_cu), _ptr(idx), total_k, _ptr(w.contiguous()),
                                                  _ptr(b), d_out, TR_ACT[act], _ptr(z), _ptr(err), _stream(dev)))
     return z[:total_k], err
+
+
+def project(y, w, bias=None, act="gelu", error=None, out=None):
+    """tr_project: z = sigma(y W^T + bias) for rows already gathered (tr_gather's
+    y, bf16 [rows, D]); ``w`` bf16 [d_out, D], ``bias`` fp32 [d_out] or None;
+    ``out`` an optional bf16 [rows, d_out] buffer.  Returns (z, error)."""
+    lib = load()
+    if y.dtype != torch.bfloat16 or w.dtype != torch.bfloat16:
+        raise TypeError("y and w must be bf16")
+    if act not in TR_ACT:
+        raise ValueError(f"act must be one of {sorted(TR_ACT)}")
+    if y.dim() != 2 or not y.is_contiguous() or w.dim() != 2 or w.shape[1] != y.shape[1]:
+        raise ValueError("y must be contiguous [rows, D] and w [d_out, D]")
+    rows, d = int(y.shape[0]), int(y.shape[1])
+    d_out = int(w.shape[0])
+    dev = y.device
+    b = None if bias is None else bias.float().contiguous()
+    z = out if out is not None else torch.empty(max(rows, 1), d_out, dtype=torch.bfloat16, device=dev)
+    if z.dtype != torch.bfloat16 or not z.is_contiguous() or z.shape[1] != d_out or z.shape[0] < rows:
+        raise ValueError(f"out must be contiguous bf16 [>= {rows}, {d_out}]")
+    err = torch.zeros(1, dtype=torch.int32, device=dev) if error is None else error
+    check("tr_project", lib.tr_project(_ptr(y), rows, d, _ptr(w.contiguous()), _ptr(b), d_out, TR_ACT[act], _ptr(z),
+                                       _ptr(err), _stream(dev)))
+    return z[:rows], err

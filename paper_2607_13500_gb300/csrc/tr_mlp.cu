@@ -1087,6 +1087,31 @@ MlpWs mlp_ws(const tr_mlp *m) {
   return w;
 }
 
+// out = act(a W^T + bias) for dense bf16 rows a [rows, k] and W [n, k]: the
+// hidden-mode GEMM (bias + activation epilogue, TMA stores), arguments
+// checked by the caller.
+tr_status dense_act_gemm(const void *a, int rows, int k, const void *w, const float *bias, int n, int act, void *out,
+                         int32_t *d_error, cudaStream_t st) {
+  if (rows == 0) return TR_OK;
+  GemmArgs g{};
+  g.m = rows;
+  g.n = n;
+  g.k = k;
+  g.n_tiles = (g.n + kBN - 1) / kBN;
+  g.tiles = ((g.m + kBM - 1) / kBM) * g.n_tiles;
+  g.kblocks = (g.k + kBK - 1) / kBK;
+  g.bias = bias;
+  g.act = act;
+  g.out = static_cast<uint16_t *>(out);
+  g.err = d_error;
+  CUtensorMap ma, mb, mo;
+  if (!make_map(&ma, a, rows, k, kBM) || !make_map(&mb, w, n, k, b_box_rows(g.m)) ||
+      !make_map(&mo, out, rows, n, 32, 128 / epi_parts(kModeHidden),
+                epi_parts(kModeHidden) == 2 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B))
+    return TR_ERR_CUDA;
+  return launch_gemm<kModeHidden>(ma, mb, mo, g, st) == cudaSuccess ? TR_OK : TR_ERR_CUDA;
+}
+
 }  // namespace
 }  // namespace tr
 
@@ -1099,26 +1124,19 @@ tr_status tr_mlp_hidden(const tr_mlp *m, void *h, int32_t *d_error, void *stream
   if (rc != TR_OK) return rc;
   if (!h) return TR_ERR_ARG;
   if (misaligned16(h)) return TR_ERR_ALIGN;
-  if (m->t == 0) return TR_OK;
-  GemmArgs g{};
-  g.m = m->t;
-  g.n = m->d_hidden;
-  g.k = m->d;
-  g.n_tiles = (g.n + kBN - 1) / kBN;
-  g.tiles = ((g.m + kBM - 1) / kBM) * g.n_tiles;
-  g.kblocks = (g.k + kBK - 1) / kBK;
-  g.bias = m->b1;
-  g.act = m->act;
-  g.out = static_cast<uint16_t *>(h);
-  g.err = d_error;
-  CUtensorMap ma, mb, mo;
-  if (!make_map(&ma, m->x_pre, m->t, m->d, kBM) || !make_map(&mb, m->w1, m->d_hidden, m->d, b_box_rows(g.m)) ||
-      !make_map(&mo, h, m->t, m->d_hidden, 32, 128 / epi_parts(kModeHidden),
-                                                           epi_parts(kModeHidden) == 2 ? CU_TENSOR_MAP_SWIZZLE_128B
-                                                                                       : CU_TENSOR_MAP_SWIZZLE_64B))
-    return TR_ERR_CUDA;
-  return launch_gemm<kModeHidden>(ma, mb, mo, g, static_cast<cudaStream_t>(stream)) == cudaSuccess ? TR_OK
-                                                                                                    : TR_ERR_CUDA;
+  return dense_act_gemm(m->x_pre, m->t, m->d, m->w1, m->b1, m->d_hidden, m->act, h, d_error,
+                        static_cast<cudaStream_t>(stream));
+}
+
+tr_status tr_project(const void *y, int32_t rows, int32_t d, const void *w, const float *bias, int32_t d_out,
+                     int32_t act, void *z, int32_t *d_error, void *stream) {
+  if (!y || !w || !z || rows < 0 || d <= 0 || d_out <= 0) return TR_ERR_ARG;
+  if (act != TR_ACT_GELU && act != TR_ACT_QUICK_GELU && act != TR_ACT_NONE) return TR_ERR_ARG;
+  if (d % 16 != 0 || d_out % 16 != 0) return TR_ERR_ALIGN;
+  if (d > TR_MAX_D || d_out > TR_MLP_MAX_HIDDEN) return TR_ERR_UNSUPPORTED;
+  if (((long long)rows + kBM - 1) / kBM * ((d_out + kBN - 1) / kBN) > INT_MAX) return TR_ERR_UNSUPPORTED;
+  if (misaligned16(y) || misaligned16(w) || misaligned16(bias) || misaligned16(z)) return TR_ERR_ALIGN;
+  return dense_act_gemm(y, rows, d, w, bias, d_out, act, z, d_error, static_cast<cudaStream_t>(stream));
 }
 
 size_t tr_mlp_workspace_bytes(const tr_mlp *m) {

@@ -94,6 +94,19 @@ def test_host_argument_checks(lib):
     assert lib.tr_gather(ctypes.byref(t), v(0x40200), v(0x50000), 1153, v(0x70000), None) == 2
     assert lib.tr_gather(ctypes.byref(t), None, v(0x50000), 10, v(0x70000), None) == 1
     assert lib.tr_gather(ctypes.byref(t), v(0x40200), v(0x50000), 10, v(0x70004), None) == 4
+    # tr_project: every check comes before any CUDA call; no rows is a no-op
+    p = lambda y=v(0x40000), rows=64, d=1024, w=v(0x80000), b=None, d_out=4096, act=0, z=v(0x90000): \
+        lib.tr_project(y, rows, d, w, b, d_out, act, z, None, None)
+    assert p(rows=0) == 0
+    assert p(y=None, rows=0) == 1
+    assert p(z=None, rows=0) == 1
+    assert p(rows=-1) == 1
+    assert p(act=9, rows=0) == 1
+    assert p(d=1000, rows=0) == 4             # not a multiple of 16
+    assert p(d_out=4100, rows=0) == 4
+    assert p(d=20000, rows=0) == 7
+    assert p(y=v(0x40008), rows=0) == 4       # base not 16-byte aligned
+    assert p(b=v(0x50004), rows=0) == 4
 
 
 def test_pipeline_host_argument_checks(lib):

@@ -196,14 +196,6 @@ def test_fused_selection_full_size():
 
 
 # ---------------------------------------------------------------- projector on the kept tokens
-def _hidden_on(altr, y, w, bias, act):
-    """The hidden-GEMM kernel run on an explicit gathered copy y (TMA loads):
-    the same MMA inputs as tr_project_kept, which reads the rows by index."""
-    m = altr.Mlp(y.shape[0], w, w.t().contiguous(), bias, None, act=act)
-    out = m.run(y.contiguous())
-    return out.h, out.error
-
-
 @pytest.mark.parametrize("name,over,bud,d_out,act", [
     ("llava576", dict(batch=3, d=1024), dict(k=192), 4096, "gelu"),           # LLaVA-1.5's 1024 -> 4096 layer
     ("ragged_dynres", dict(batch=5, n=(256, 3000), d=1152), dict(ratio=(2, 9)), 1280, "quick_gelu"),
@@ -211,8 +203,9 @@ def _hidden_on(altr, y, w, bias, act):
 ], ids=["llava576", "ragged_dynres", "partial_kblock"])
 def test_project_kept(name, over, bud, d_out, act):
     # Selection, then the projector's first layer on the kept tokens read
-    # from x by index: bit for bit the hidden GEMM on the gathered copy y,
-    # and within the GEMM tolerance of float64 on the kept rows.
+    # from x by index: bit for bit tr_project on the gathered copy y (the
+    # hidden-GEMM kernel with plain TMA loads), and within the GEMM tolerance
+    # of float64 on the kept rows.
     altr = _alt()
     w_in = synth.make(name, seed=17, device="cuda", **over)
     budget = altr.budgets(w_in.seqlens, **bud)
@@ -221,7 +214,7 @@ def test_project_kept(name, over, bud, d_out, act):
     w = (torch.randn(d_out, w_in.d, generator=g, device="cuda") / math.sqrt(w_in.d)).to(torch.bfloat16)
     bias = 0.05 * torch.randn(d_out, generator=g, device="cuda")
     z, err = altr.project_kept(w_in.x, r.idx, budget[2], w, bias, act=act, seqlens=w_in.seqlens)
-    zh, err_h = _hidden_on(altr, r.y, w, bias, act)
+    zh, err_h = altr.project(r.y, w, bias, act=act)
     torch.cuda.synchronize()
     assert err.item() == 0 and err_h.item() == 0
     assert torch.equal(z.view(torch.int16), zh.view(torch.int16))
