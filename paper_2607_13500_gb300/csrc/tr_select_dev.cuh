@@ -780,17 +780,24 @@ __device__ __noinline__ bool df_row_block(const SelectArgs &a, long long row, in
   }
   g.sync();
   const int gi = g.bar - 1;
+  const int w0 = g.first >> 5, nw = g.size >> 5;
+  if (g.tid() < (mode == 0 ? 2 : 3)) {
+    // thread j of the group's first warp merges sum j's warp partials in
+    // turn, into the first warp's slot (only thread j touches index j)
+    const int j = g.tid();
+    float h = part.h[w0 * 3 + j], l = part.l[w0 * 3 + j];
+    for (int w = w0 + 1; w < w0 + nw; ++w) df_join(h, l, part.h[w * 3 + j], part.l[w * 3 + j]);
+    const df::F2 n = df::two_sum(h, l);
+    part.h[w0 * 3 + j] = n.h;
+    part.l[w0 * 3 + j] = n.l;
+  }
+  if (g.tid() < 32) __syncwarp();
   if (g.tid() == 0) {
-    // the group's first thread merges the warps' partials in turn
-    const int w0 = g.first >> 5, nw = g.size >> 5;
     float s[3][2];
 #pragma unroll
     for (int j = 0; j < 3; ++j) {
-      float h = part.h[w0 * 3 + j], l = part.l[w0 * 3 + j];
-      for (int w = w0 + 1; w < w0 + nw; ++w) df_join(h, l, part.h[w * 3 + j], part.l[w * 3 + j]);
-      const df::F2 n = df::two_sum(h, l);
-      s[j][0] = n.h;
-      s[j][1] = n.l;
+      s[j][0] = part.h[w0 * 3 + j];
+      s[j][1] = part.l[w0 * 3 + j];
     }
     bool fine;
     if (mode == 0) {
@@ -1869,6 +1876,9 @@ __device__ __noinline__ void resolve_cut(const SelectArgs &a, const ImageCtx c, 
       const uint32_t k = key[i];
       c_in += k >= kw_lo && k <= kw_hi;
       c_lt += k < kw_lo;
+      // above the window, R exceeds the K1-th key's by far more than the
+      // keys' bound: certainly among the K1 kept, whichever order follows
+      if (k < kw_lo) fl[i] |= F_IMP;
     }
     // one scan of both counts (each total is at most n < 2^16)
     int both = 0;
@@ -1899,27 +1909,41 @@ __device__ __noinline__ void resolve_cut(const SelectArgs &a, const ImageCtx c, 
       len = n;
     }
     const bool whole = base == 0 && len == n;
+    // The uncertain run around position p = k1 - base: from the last
+    // certified boundary at or before p (0 if none) to the first at or after
+    // p (len if none), found by all threads at once; a certified p gives
+    // lo = hi = p, no run.
+    const int p = k1 - base;
+    const bool outside = p < 1 || p >= len;  // uniform
     if (tid == 0) {
-      int lo = k1 - base, hi = k1 - base;
-      bool escaped = lo < 1 || lo >= len;
-      if (!escaped && !cert_r(key, ord, lo, a.bounds)) {
-        --lo;
-        while (lo > 0 && !cert_r(key, ord, lo, a.bounds)) --lo;
-        ++hi;
-        while (hi < len && !cert_r(key, ord, hi, a.bounds)) ++hi;
-        escaped = !whole && (lo == 0 || hi == len);  // the run may go on outside the list
+      sh_lo = 0;
+      sh_hi = len;
+    }
+    __syncthreads();
+    if (!outside) {
+      int my_lo = 0, my_hi = len;
+      for (int q = 1 + tid; q < len; q += nthr)
+        if (cert_r(key, ord, q, a.bounds)) {
+          if (q <= p) my_lo = q;  // q rises: the last one wins
+          if (q >= p && my_hi == len) my_hi = q;
+        }
+      if (my_lo > 0) atomicMax(&sh_lo, my_lo);
+      if (my_hi < len) atomicMin(&sh_hi, my_hi);
+    }
+    __syncthreads();
+    if (tid == 0) {
+      if (outside) {
+        sh_lo = -1;
+        sh_hi = p;
+      } else if (sh_lo != sh_hi && !whole && (sh_lo == 0 || sh_hi == len)) {
+        sh_lo = -1;  // the run may go on outside the list
       }
-      sh_lo = escaped ? -1 : lo;
-      sh_hi = hi;
     }
     __syncthreads();
     if (sh_lo >= 0) break;
     ord = nullptr;  // the window was not enough: sort everything
   }
   const int lo = sh_lo, hi = sh_hi;
-  if (base > 0)
-    for (int i = tid; i < n; i += nthr)
-      if (key[i] < kw_lo) fl[i] |= F_IMP;
   for (int q = tid; q < lo; q += nthr) fl[ord[q]] |= F_IMP;
   if (hi > lo) {
     // The run's rows: double-float keys first (short runs), and exact
