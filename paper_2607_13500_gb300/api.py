@@ -32,6 +32,15 @@ def _ptr(t):
     return None if t is None else ctypes.c_void_p(t.data_ptr())
 
 
+def _check_buf(t, device, dtype, min_numel, name):
+    """A caller's buffer the library reads or writes: on the tokens' device,
+    of the expected dtype, contiguous and large enough (None passes)."""
+    if t is None:
+        return
+    if t.device != device or t.dtype != dtype or not t.is_contiguous() or t.numel() < min_numel:
+        raise ValueError(f"{name} must be a contiguous {dtype} tensor of at least {min_numel} elements on {device}")
+
+
 def _stream(device) -> ctypes.c_void_p:
     return ctypes.c_void_p(torch.cuda.current_stream(device).cuda_stream)
 
@@ -135,6 +144,10 @@ def select(x, x_pre, x_post, stats, k=None, ratio=None, lam=(1, 3), seqlens=None
     interval, TR_STRIDE_INTERVAL)."""
     lib = load()
     x, x_pre, x_post, seqlens = _flatten(x, x_pre, x_post, seqlens)
+    t = x.shape[0]
+    _check_buf(stats, x.device, torch.float32, t * TR_STATS_WORDS, "stats")
+    _check_buf(h2, x.device, torch.float32, t, "h2")
+    _check_buf(s, x.device, torch.float32, t, "s")
     tok = _Tokens(x, x_pre, x_post, seqlens, stride)
     ks, k1s, cu_k = budget if budget is not None else budgets(seqlens, k, ratio, lam)
     dev = x.device
@@ -248,6 +261,7 @@ class Reducer:
         by Mlp's fused scoring), on the current stream; ``events`` (three
         torch.cuda.Event or None) recorded before, between and after."""
         tok = self._bind(x, x_pre, x_post)
+        _check_buf(stats, tok.x.device, torch.float32, tok.x.shape[0] * TR_STATS_WORDS, "stats")
         st = _stream(self.device)
         lib = self.lib
         self.status.zero_()
@@ -578,6 +592,9 @@ class Mlp:
 
     def __init__(self, t, w1, w2, b1=None, b2=None, act="gelu", scores=False):
         self.lib = load()
+        if w1.device.type != "cuda" or w2.device != w1.device or any(
+                b is not None and b.device != w1.device for b in (b1, b2)):
+            raise ValueError("the MLP weights and biases must live on one CUDA device (libtr has no CPU path)")
         if w1.dtype != torch.bfloat16 or w2.dtype != torch.bfloat16:
             raise TypeError("the MLP weights must be bf16")
         dh, d = w1.shape
@@ -657,6 +674,9 @@ def project_kept(x, idx, cu_k, w, bias=None, act="gelu", seqlens=None, error=Non
     if act not in TR_ACT:
         raise ValueError(f"act must be one of {sorted(TR_ACT)}")
     x2, _, _, seqlens = _flatten(x, None, x, seqlens)
+    if w.device != x2.device or idx.device != x2.device or (bias is not None and bias.device != x2.device) or \
+            (error is not None and error.device != x2.device):
+        raise ValueError("w, idx, bias and error must live on x's device")
     tok = _Tokens(x2, None, x2, seqlens)
     total_k = int(cu_k[-1])
     d_out = int(w.shape[0])
@@ -675,6 +695,9 @@ def project(y, w, bias=None, act="gelu", error=None, out=None):
     y, bf16 [rows, D]); ``w`` bf16 [d_out, D], ``bias`` fp32 [d_out] or None;
     ``out`` an optional bf16 [rows, d_out] buffer.  Returns (z, error)."""
     lib = load()
+    if y.device.type != "cuda" or w.device != y.device or (bias is not None and bias.device != y.device) or \
+            (out is not None and out.device != y.device):
+        raise ValueError("y, w, bias and out must live on one CUDA device (libtr has no CPU path)")
     if y.dtype != torch.bfloat16 or w.dtype != torch.bfloat16:
         raise TypeError("y and w must be bf16")
     if act not in TR_ACT:

@@ -146,3 +146,35 @@ def test_missing_library_raises(monkeypatch, tmp_path):
         altr.reduce(x, x, x, k=2)
     with pytest.raises(RuntimeError, match="missing"):
         altr.budgets([8], k=2)
+
+
+def test_binding_refuses_bad_buffers_before_any_launch(lib, monkeypatch):
+    # Caller-supplied buffers are checked in Python before the library sees a
+    # pointer: host tensors for the MLP and the projector, and statistics of
+    # the wrong dtype, size or layout for the selection (the token tensors'
+    # own device check is bypassed here so that host tensors reach it).
+    import torch
+
+    from paper_2607_13500_gb300 import api
+    w = torch.zeros(64, 32, dtype=torch.bfloat16)
+    with pytest.raises(ValueError, match="CUDA"):
+        api.Mlp(4, w, w.t().contiguous())
+    with pytest.raises(ValueError, match="CUDA"):
+        api.project(torch.zeros(4, 32, dtype=torch.bfloat16), w)
+    monkeypatch.setattr(api, "_flatten", lambda x, xp, xq, sl: (x, xp, xq, sl or [x.shape[0]]))
+    x = torch.zeros(16, 64, dtype=torch.bfloat16)
+    good = torch.zeros(16, 8)
+    for bad in (good.double(), good[:8], good.t()):
+        with pytest.raises(ValueError, match="stats"):
+            api.select(x, x, x, bad, k=4)
+    with pytest.raises(ValueError, match="h2"):
+        api.select(x, x, x, good, k=4, h2=torch.zeros(3))
+    with pytest.raises(ValueError, match="s must"):
+        api.select(x, x, x, good, k=4, s=torch.zeros(16, dtype=torch.float64))
+    # and good buffers go through to the entry point (stubbed: no GPU here)
+    calls = []
+    monkeypatch.setattr(lib, "tr_select", lambda *args: calls.append(len(args)) or 0)
+    monkeypatch.setattr(api, "_stream", lambda device: None)
+    monkeypatch.setattr(api, "_workspace", lambda lib_, tok, device: (torch.empty(256, dtype=torch.uint8), 256))
+    idx, role, cu_k, status = api.select(x, x, x, good, k=4, h2=torch.zeros(16), s=torch.zeros(16))
+    assert calls == [13] and cu_k == [0, 4] and idx.shape == (4,) and role.shape == (16,)
